@@ -1,0 +1,336 @@
+"""Benchmark of the MTP decode path on one VALL-E-sized workload.
+
+Workload (one "step"): batch 1, prompt = 64 phonemes + 225 acoustic codes,
+prefill, then decode 750 codec tokens with n = 4 heads and top_k = 4
+(ceil(750 / 4) = 188 decode steps) -- whole-job codec tokens/s.  Synthetic
+seeded weights and prompts (synth); the 302 MB of weights per decode step
+are larger than L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line.  --impl reference times the CPU oracle on the host
+cores (a bounded sample of the same workload).  Under torchrun (N > 1) every
+rank runs an independent replica (no collective on the data path); the
+value is all ranks' tokens over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+N_PH, N_AC, GEN, N_HEADS, TOP_K, BATCH = 64, 225, 750, 4, 4, 1
+WORKLOAD = "VALL-E-sized AR decode: 12 layers, d=1024, 16 heads, FFN 4096, bf16; B=1, prompt 64+225, 750 tokens, n=4, top_k=4"
+METRIC = "codec tokens/s at B=1 (n=4 heads, top_k=4)"
+MODEL = synth.VALLE
+MAX_CTX = N_PH + N_AC + GEN + MODEL.n_heads_max + 8
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        p = json.load(open(path))
+        return float(p["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def _config():
+    return {"workload": WORKLOAD, "batch": BATCH, "prompt": [N_PH, N_AC], "generate": GEN,
+            "n_heads": N_HEADS, "top_k": TOP_K, "page_size": 64,
+            "l2": "inputs larger than L2: 302 MB of weights streamed per decode step (L2 129 MB)",
+            "parallelism": "replicas"}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def _kernel_bytes(d, F, V, L, n, wb, ctx_keys):
+    """Algorithmic bytes per launch of each kernel class (weights + params; KV for attention)."""
+    return {
+        "qkv": 3 * d * d * wb + 3 * d * 4 + 2 * d * 4,
+        "oproj": d * d * wb + d * 4,
+        "ffn1": F * d * wb + F * 4 + 2 * d * 4,
+        "ffn2": d * F * wb + d * 4,
+        "heads": n * V * d * wb + n * V * 4 + 2 * d * 4,
+        "attn": ctx_keys * d * 2 * 2,
+    }
+
+
+def _decode_bytes_total(d, F, V, L, n, wb, prompt_len, gen):
+    """Algorithmic bytes of all decode steps of one generation (weights, heads, KV read + write)."""
+    weights = L * ((3 * d * d + d * d + 2 * d * F) * wb + (3 * d + d + F + d + 4 * d) * 4)
+    heads = n * V * d * wb + n * V * 4 + 2 * d * 4
+    total, cached, produced = 0, prompt_len, 0
+    fed = 0
+    while produced < gen:
+        step = heads
+        if fed:
+            step += weights + L * (cached + fed) * d * 4 + L * fed * d * 4
+            cached += fed
+        a = min(n, gen - produced)
+        produced += a
+        fed = a
+        total += step
+    return total
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = [r.split(",") for r in (self.out or "").strip().splitlines() if r.count(",") >= 8]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        sm = [float(r[1]) for r in rows]
+        smax = max(float(r[2]) for r in rows)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": reasons, "samples": len(rows)}
+
+
+def cpu_baseline(max_steps: int = 60):
+    """The oracle as it stands on this host: prefill + the first decode steps of the workload."""
+    from oracle.mtp import MTPOracle
+    w = synth.make_weights(MODEL)
+    ph, ac = synth.make_prompt(0, N_PH, N_AC, MODEL.phone_vocab)
+    o = MTPOracle(MODEL, w)
+    t0 = time.perf_counter()
+    o.prefill(ph, ac, GEN)
+    recs = o.generate(N_HEADS, TOP_K, max_steps=max_steps)
+    dt = time.perf_counter() - t0
+    toks = sum(r.accepted for r in recs)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": toks / dt, "unit": "codec tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"prefill of the {N_PH + N_AC}-token prompt + first {len(recs)} decode steps "
+                      f"({toks} tokens), float64 numpy, {dt:.1f} s"}
+
+
+def _traffic_for(kind: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    entry = json.load(open(path)).get(kind)
+    if not entry:
+        return None
+    src = os.path.join(ROOT, entry["source"])
+    if not os.path.exists(src) or hashlib.sha1(open(src, "rb").read()).hexdigest() != entry["source_sha1"]:
+        return None
+    return entry["dram_bytes_per_launch"]
+
+
+def run_reference(args):
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    from oracle.mtp import MTPOracle
+    w = synth.make_weights(MODEL)
+    ph, ac = synth.make_prompt(0, N_PH, N_AC, MODEL.phone_vocab)
+    o = MTPOracle(MODEL, w)
+    o.prefill(ph, ac, GEN)
+    per_step = 8    # decode steps per bench step: a bounded sample of the generation
+    times, toks = [], 0
+    for i in range(args.warmup + args.steps):
+        if o.done:
+            o.prefill(ph, ac, GEN)
+        t0 = time.perf_counter()
+        recs = o.generate(N_HEADS, TOP_K, max_steps=per_step)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+            toks += sum(r.accepted for r in recs)
+    total = sum(times)
+    value = toks / total
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "codec tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config(),
+            "cpu_baseline": {"value": value, "unit": "codec tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{per_step} decode steps ({per_step * N_HEADS} tokens) per bench step "
+                                       "after one untimed prefill; float64 numpy oracle"},
+            "e2e": {"value": value, "unit": "codec tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    cpu = cpu_baseline() if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
+
+    from paper_2410_13839_gb300 import build
+    build.build()
+    from paper_2410_13839_gb300 import mtp
+
+    stream = torch.cuda.Stream()
+    w = synth.make_weights(MODEL)
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, BATCH, MAX_CTX, stream=stream)
+    ctx = dec.ctx
+    ph, ac = synth.make_prompt(rank, N_PH, N_AC, MODEL.phone_vocab)
+    with torch.cuda.stream(stream):
+        ph_d = torch.from_numpy(ph).cuda()
+        ac_d = torch.from_numpy(ac).cuda()
+    stream.synchronize()
+    lens = torch.zeros(BATCH, dtype=torch.int32, device="cuda")
+
+    def one_step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        mtp.mtp_prefill(ctx, 0, ph_d, ac_d, GEN)
+        if ev:
+            ev[1].record(stream)
+        steps = mtp.mtp_generate(ctx, N_HEADS, TOP_K, None, 0, lens)
+        if ev:
+            ev[2].record(stream)
+        return steps
+
+    def barrier():
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        one_step()
+    barrier()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        start = torch.cuda.Event(enable_timing=True)
+        stop = torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        decode_steps = 0
+        for i in range(args.steps):
+            decode_steps += one_step(evs[i])
+        stop.record(stream)
+        barrier()
+    ms = start.elapsed_time(stop)
+    tokens_done = int(lens.cpu()[0])
+    assert tokens_done == GEN, f"generation stopped at {tokens_done} tokens"
+    prefill_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    decode_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * args.steps * GEN * BATCH / (ms / 1e3)
+
+    # end to end through the public API with host buffers (pinned), copies inside the timed region
+    ph_h = torch.from_numpy(ph).pin_memory()
+    ac_h = torch.from_numpy(ac).pin_memory()
+    out_h = torch.zeros((BATCH, GEN), dtype=torch.int32).pin_memory()
+    lens_h = torch.zeros(BATCH, dtype=torch.int32).pin_memory()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        mtp.mtp_prefill(ctx, 0, ph_h, ac_h, GEN)
+        mtp.mtp_generate(ctx, N_HEADS, TOP_K, out_h, GEN, lens_h)
+    barrier()
+    e2e_s = time.perf_counter() - t0
+    if dist:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = {"value": world * args.steps * GEN * BATCH / e2e_s, "unit": "codec tokens/s",
+           "h2d_bytes_per_step": (N_PH + N_AC) * 4, "d2h_bytes_per_step": BATCH * GEN * 4 + BATCH * 4}
+
+    # per-kernel durations: one eager step mid-generation, events around every launch
+    mtp.mtp_prefill(ctx, 0, ph_d, ac_d, GEN)
+    for _ in range(GEN // N_HEADS // 2):
+        mtp.mtp_decode_step(ctx, N_HEADS, TOP_K)
+    state = mtp.mtp_seq_state(ctx, 0)
+    prof = mtp.mtp_profile_step(ctx, N_HEADS, TOP_K)
+    d, F, V, L = MODEL.d_model, MODEL.d_ffn, MODEL.codec_vocab, MODEL.layers
+    kb = _kernel_bytes(d, F, V, L, N_HEADS, 2, state["len"] + state["pending"])
+    dom = max(kb, key=lambda kind: prof[kind][0])
+    per_launch_ms = prof[dom][0] / max(1, prof[dom][1])
+    peak, peak_kind = _peaks()
+    achieved = kb[dom] / (per_launch_ms / 1e3) / 1e9
+    traffic = _traffic_for(dom)
+    roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic, "peak_source": peak_kind,
+                "algorithmic_bytes_per_launch": kb[dom], "avg_launch_us": per_launch_ms * 1e3,
+                "timing": "one eager decode step at context %d, CUDA events around each launch" % state["len"]}
+    dec_bytes = _decode_bytes_total(d, F, V, L, N_HEADS, 2, N_PH + N_AC, GEN)
+    step_roof = {"decode_bytes": dec_bytes, "decode_ms": decode_ms,
+                 "achieved_gbs": dec_bytes / (decode_ms / 1e3) / 1e9,
+                 "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak}
+    launches_per_step = 2 + ((N_PH + N_AC + 7) // 8) * (1 + 5 * L) + decode_steps // args.steps * (3 + 5 * L)
+
+    line = {"metric": METRIC, "value": value, "unit": "codec tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": _config(),
+            "roofline": roofline, "decode_roofline": step_roof,
+            "prefill_ms": prefill_ms, "decode_ms": decode_ms,
+            "decode_tokens_per_s": GEN / (decode_ms / 1e3),
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk.summary(), "kernel_ms": {k: v[0] for k, v in prof.items()}}
+    dec.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

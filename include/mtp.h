@@ -1,0 +1,264 @@
+/*
+ * mtp.h -- C ABI of the GB300 (sm_103a) multi-token-prediction decode path.
+ *
+ * The operation: accelerated inference of an autoregressive codec-token
+ * language model (Sec. III-A, Eq. 1) extended with n multi-token-prediction
+ * heads (Sec. III-B) and Viterbi-based selection of the token sequence to
+ * accept from the heads' top-k candidates (Sec. III-C).  Every step of the
+ * path runs in this library's CUDA kernels; the caller supplies memory
+ * (host or device pointers, as each call states) and a CUDA stream.
+ *
+ * Conventions for every call:
+ *   - return value: MTP_OK (0) or a negative mtp_status; mtp_last_error()
+ *     then gives a message (per thread, valid until the next call);
+ *   - pointers marked "host or device" are classified with
+ *     cudaPointerGetAttributes; device pointers must be on the context's GPU;
+ *   - the caller owns every buffer it passes; the library owns only the
+ *     device state inside an mtp_ctx and frees it in mtp_destroy;
+ *   - calls on one context are not thread-safe; calls on different contexts are;
+ *   - work is ordered on the stream given to mtp_create (or, for the
+ *     stand-alone operators, the stream passed in); calls that return data
+ *     to host memory synchronise that stream first.
+ */
+#ifndef MTP_H
+#define MTP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MTP_API __attribute__((visibility("default")))
+#define MTP_ABI_VERSION 1
+
+typedef enum mtp_status {
+    MTP_OK = 0,
+    MTP_ERR_INVALID = -1,   /* bad argument, size or handle                          */
+    MTP_ERR_NO_PAGES = -2,  /* KV page pool cannot hold the requested sequence        */
+    MTP_ERR_CUDA = -3,      /* a CUDA runtime call failed (message has the CUDA text) */
+    MTP_ERR_WEIGHTS = -4,   /* weight blob malformed or inconsistent with the config  */
+    MTP_ERR_DEVICE = -5     /* a kernel set the device error word (bounded wait ran
+                               out or an index failed its check); the context must be
+                               destroyed */
+} mtp_status;
+
+typedef enum mtp_dtype { MTP_F32 = 0, MTP_BF16 = 1 } mtp_dtype;
+
+/* Acceptance of the selected path (Sec. III-C): the paper accepts the whole
+ * Viterbi path each step; it is cut after the first EOS and at the
+ * sequence's remaining token budget. */
+typedef enum mtp_accept { MTP_ACCEPT_ALL = 0 } mtp_accept;
+
+/* Model and capacity.  The model is a decoder-only transformer over one
+ * concatenated sequence [phonemes ; acoustic prompt ; generated codes]
+ * (Sec. III-A) with sinusoidal absolute positions, pre-LN blocks (exact-erf
+ * GELU MLP, biased linears), a final LayerNorm and n_heads_max linear heads
+ * d_model -> codec_vocab; head i (1-based) predicts the token i positions
+ * ahead (Sec. III-B). */
+typedef struct mtp_config {
+    int32_t layers;        /* transformer blocks                                   */
+    int32_t d_model;       /* multiple of 256                                      */
+    int32_t n_attn_heads;  /* d_model / n_attn_heads must be 64                    */
+    int32_t d_ffn;         /* multiple of 256                                      */
+    int32_t phone_vocab;   /* phoneme table rows                                   */
+    int32_t codec_vocab;   /* codec ids + EOS (1025 in the paper's setting), <= 1056 */
+    int32_t eos_id;        /* EOS id inside [0, codec_vocab)                        */
+    int32_t n_heads_max;   /* heads stored in the blob, 1..8                        */
+    int32_t top_k_max;     /* largest top_k a call may ask for, 1..32               */
+    int32_t max_batch;     /* sequence slots, 1..1024                               */
+    int32_t max_ctx;       /* longest prompt + generation + n_heads_max per slot    */
+    int32_t page_size;     /* KV tokens per page: 16, 32, 64 or 128                 */
+    int32_t n_pages;       /* pages in the pool; 0 = max_batch * ceil(max_ctx/page) */
+    int32_t weight_dtype;  /* mtp_dtype of matrices and embedding tables            */
+    int32_t accept_policy; /* mtp_accept                                            */
+    float ln_eps;          /* LayerNorm epsilon                                     */
+} mtp_config;
+
+/*
+ * Weight blob (host memory, read during mtp_create only):
+ *   bytes 0..7   magic "MTPWGT01"
+ *   u32          version (1)
+ *   u32          n_tensors = 5 + 12 * layers + 2
+ *   u64          reserved (0)
+ *   n_tensors x { u64 offset_from_blob_start; u64 nbytes; }
+ *   tensor data; every offset a multiple of 256.
+ * Tensors in this order (row-major; "W" = weight_dtype, "f" = fp32):
+ *   tok_phone [phone_vocab, d] W      tok_codec [codec_vocab, d] W
+ *   per layer: ln1_g [d] f, ln1_b [d] f, wqkv [3d, d] W (rows q | k | v, head h
+ *              at rows h*64..h*64+63 of each part), bqkv [3d] f, wo [d, d] W,
+ *              bo [d] f, ln2_g [d] f, ln2_b [d] f, w1 [d_ffn, d] W,
+ *              b1 [d_ffn] f, w2 [d, d_ffn] W, b2 [d] f
+ *   lnf_g [d] f, lnf_b [d] f, w_heads [n_heads_max, codec_vocab, d] W,
+ *   b_heads [n_heads_max, codec_vocab] f,
+ *   log_q [codec_vocab, codec_vocab] f  -- log of the token transition matrix
+ *              Q of Sec. III-C, log_q[i][j] = log Q(i -> j).
+ * A linear layer computes y = x W^T + b.
+ */
+
+typedef struct mtp_ctx mtp_ctx;
+
+/* Create a context on the current CUDA device: validates config and blob,
+ * copies the weights to the device (the caller keeps the blob), allocates
+ * the KV page pool and all step buffers.  `cuda_stream` is a cudaStream_t
+ * (NULL = legacy default stream) used by every later call on the context.
+ * Errors: MTP_ERR_INVALID (config), MTP_ERR_WEIGHTS (blob), MTP_ERR_CUDA. */
+MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_t blob_bytes,
+                       void* cuda_stream, mtp_ctx** out);
+
+/* Free every device resource of the context (NULL is ignored). */
+MTP_API void mtp_destroy(mtp_ctx* ctx);
+
+/* Message of the last failed call on this thread ("" if none). */
+MTP_API const char* mtp_last_error(void);
+
+/* Admit a sequence into slot `seq_slot` and run the prompt through the model
+ * (Sec. III-A: [phonemes ; acoustic prompt] as one sequence).  Reserves
+ * ceil((n_ph + n_ac + max_new_tokens + n_heads_max) / page_size) pages for
+ * the slot (released by mtp_release or the next prefill of the slot), fills
+ * their keys/values and keeps the last position's hidden state, from which
+ * the next mtp_decode_step selects the first tokens.  `phonemes` and
+ * `acoustic` are int32 ids, host or device; n_ph + n_ac >= 1.
+ * Errors: MTP_ERR_INVALID (slot, ids out of range, length > max_ctx),
+ * MTP_ERR_NO_PAGES, MTP_ERR_CUDA. */
+MTP_API int mtp_prefill(mtp_ctx* ctx, int seq_slot, const int32_t* phonemes, int n_ph,
+                        const int32_t* acoustic, int n_ac, int max_new_tokens);
+
+/* Return the slot's pages to the pool and mark it inactive. */
+MTP_API int mtp_release(mtp_ctx* ctx, int seq_slot);
+
+/* One decode step for every active, unfinished slot (Fig. 1 caption,
+ * Sec. III-B/C): feed the tokens accepted by the previous step (appending
+ * their keys/values), apply the first `n_heads` heads to the last fed
+ * position, take each head's `top_k` candidates (log-softmax descending,
+ * lower id first on ties), select a path with Viterbi over that n x k
+ * lattice and accept it under the context's policy.
+ * Outputs (each may be NULL; host or device):
+ *   out_tokens   int32 [max_batch][n_heads]: accepted tokens, -1 after them
+ *   out_accepted int32 [max_batch]: tokens accepted this step (0 if idle)
+ *   out_done     int32 [max_batch]: 1 once the slot has finished
+ * Errors: MTP_ERR_INVALID (n_heads, top_k), MTP_ERR_CUDA, MTP_ERR_DEVICE. */
+MTP_API int mtp_decode_step(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_tokens,
+                            int32_t* out_accepted, int32_t* out_done);
+
+/* Run decode steps until every active slot has finished, with no host
+ * synchronisation between steps.  out_tokens (host or device, may be NULL)
+ * receives each slot's generated tokens in row b at stride `out_stride`
+ * (>= the slot's max_new_tokens); out_lens (may be NULL) their counts.
+ * Returns the number of steps run (>= 0) or an error. */
+MTP_API int mtp_generate(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_tokens,
+                         int out_stride, int32_t* out_lens);
+
+/* Remove the last `n_tokens` cached positions of a slot (rejected tokens).
+ * The pages stay reserved for the slot and are reused by later appends. */
+MTP_API int mtp_rollback(mtp_ctx* ctx, int seq_slot, int n_tokens);
+
+/* Replace the tokens the next step feeds for a slot (teacher forcing for
+ * parity tests): `tokens` (host, int32) of length 1..n_heads_max. */
+MTP_API int mtp_set_teacher_tokens(mtp_ctx* ctx, int seq_slot, const int32_t* tokens, int n);
+
+/* Slot state (host int32[6]): cached length, tokens pending to be fed,
+ * remaining budget, done flag, active flag, tokens generated so far. */
+MTP_API int mtp_seq_state(mtp_ctx* ctx, int seq_slot, int32_t* out6);
+
+/* Logits and log-sum-exp of the last decode step (host or device):
+ * out_logits float [max_batch][n_heads][codec_vocab] and out_lse float
+ * [max_batch][n_heads] (either may be NULL), for the n_heads of that step.
+ * The kernels rank candidates by logp = logits - lse rounded to fp32. */
+MTP_API int mtp_debug_logits(mtp_ctx* ctx, float* out_logits, float* out_lse);
+
+/* Candidate lattice and selected path of the last decode step (host or
+ * device, may be NULL): out_ids int32 and out_logp float [max_batch][n][k],
+ * out_path int32 [max_batch][n]. */
+MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, int32_t* out_path);
+
+/* Options: MTP_OPT_GRAPHS (1 = capture each (n_heads, top_k) step into a
+ * CUDA graph, default) and MTP_OPT_PDL (1 = programmatic dependent launch
+ * between the step's kernels, default). */
+typedef enum mtp_option { MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1 } mtp_option;
+MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
+
+/* Kernel classes reported by mtp_profile_step. */
+typedef enum mtp_kernel_kind {
+    MTP_K_EMBED = 0, MTP_K_QKV = 1, MTP_K_ATTN = 2, MTP_K_OPROJ = 3, MTP_K_FFN1 = 4,
+    MTP_K_FFN2 = 5, MTP_K_HEADS = 6, MTP_K_SELECT = 7, MTP_K_COUNT = 8
+} mtp_kernel_kind;
+
+/* Run one decode step with each kernel launched alone (no graph, no PDL)
+ * and bracketed by CUDA events on the context's stream.  out_ms[kind]
+ * receives the summed device time (ms) and out_launches[kind] the launch
+ * count, for kinds 0..MTP_K_COUNT-1 (host arrays).  The step's effect on
+ * the slots is the same as mtp_decode_step. */
+MTP_API int mtp_profile_step(mtp_ctx* ctx, int n_heads, int top_k, float* out_ms,
+                             int32_t* out_launches);
+
+/* Algorithmic bytes of one decode step: weights read (all blocks and the
+ * first n_heads heads) plus keys/values read and written for every active
+ * slot, from the current slot state (host uint64 out). */
+MTP_API int mtp_step_bytes(mtp_ctx* ctx, int n_heads, uint64_t* out_bytes);
+
+/* ---- stand-alone operators (device pointers, caller's stream) ---------- */
+
+/* Viterbi selection over candidate lattices (Sec. III-C, reading A: the
+ * states at position t are head t's top-k candidates).  In the log domain,
+ * delta_1(j) = s_1(j) and
+ *   delta_t(j) = max_i [ delta_{t-1}(i) + log_q(c_{t-1,i}, c_{t,j}) ] + s_t(j),
+ * each add one fp32 add in that order, the lowest i taking ties; the path
+ * ends in the lowest j maximising delta_n.  Then ACCEPT_ALL: accepted =
+ * min(n, first EOS index + 1, remaining[b]) and rollback = 0.
+ *   cand_ids  int32 [batch][n][k], ids in [0, vocab)
+ *   cand_logp float [batch][n][k]
+ *   log_q     float [vocab][vocab]
+ *   remaining int32 [batch] or NULL (no budget)
+ * Outputs int32 out_path [batch][n], float out_score [batch] (may be NULL),
+ * int32 out_accepted [batch], int32 out_rollback [batch] (may be NULL).
+ * Limits: 1 <= n <= 8, 1 <= k <= 32.  Errors: MTP_ERR_INVALID, MTP_ERR_CUDA. */
+MTP_API int mtp_viterbi(int batch, int n, int k, int vocab, int eos_id,
+                        const int32_t* cand_ids, const float* cand_logp, const float* log_q,
+                        const int32_t* remaining, int32_t* out_path, float* out_score,
+                        int32_t* out_accepted, int32_t* out_rollback, void* cuda_stream);
+
+/* The context's heads on `batch` hidden states (Sec. III-B): z = LN_f(h),
+ * logits_i = z W_i^T + b_i for i < n_heads, logp = logits - lse, top-k.
+ *   hidden     [batch][d_model], dtype hidden_dtype (mtp_dtype), device
+ *   out_ids    int32 [batch][n_heads][top_k]; out_logp float, same shape
+ *   out_logits float [batch][n_heads][codec_vocab] or NULL
+ *   out_lse    float [batch][n_heads] or NULL
+ * Uses the context's stream.  Errors: MTP_ERR_INVALID, MTP_ERR_CUDA. */
+MTP_API int mtp_heads_topk(mtp_ctx* ctx, int batch, const void* hidden, int hidden_dtype,
+                           int n_heads, int top_k, int32_t* out_ids, float* out_logp,
+                           float* out_logits, float* out_lse);
+
+/* Causal attention of `rows` query rows over a paged bf16 KV pool (the
+ * attention of one block, Sec. III-A), split over the key axis with a
+ * log-sum-exp merge.  Pool layout: bf16 [n_pages][layers][2][n_heads][page_size][64],
+ * index 0 of the "2" axis keys, 1 values.  Rows are grouped: group g is rows
+ * g*rows_per_group ..; all active rows of a group belong to one slot.
+ *   q          float [rows][n_heads*64] (unscaled)
+ *   row_seq    int32 [rows]: slot of the row, < 0 = inactive row (skipped)
+ *   row_pos    int32 [rows]: position; the row sees keys 0..row_pos
+ *   block_table int32 [slots][bt_stride]: page of each page_size span
+ *   out        float [rows][n_heads*64]
+ *   workspace  device scratch of mtp_attention_workspace_bytes(...) bytes;
+ *              its counters must be zero on the first call and are left zero.
+ *   max_keys   upper bound of (row_pos + 1) over all rows; sets the split count
+ * Keys/values for positions 0..max row_pos of each group must be present.
+ * Errors: MTP_ERR_INVALID, MTP_ERR_CUDA. */
+typedef struct mtp_attention_args {
+    int32_t rows, rows_per_group, n_heads, page_size, layers, layer, bt_stride, max_keys;
+    const float* q;
+    const uint16_t* kv_pool;
+    const int32_t* block_table;
+    const int32_t* row_seq;
+    const int32_t* row_pos;
+    float* out;
+} mtp_attention_args;
+MTP_API size_t mtp_attention_workspace_bytes(const mtp_attention_args* args);
+MTP_API int mtp_attention(const mtp_attention_args* args, void* workspace, size_t workspace_bytes,
+                          void* cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MTP_H */

@@ -1,0 +1,128 @@
+// embed.cu -- rows of the concatenated sequence (Sec. III-A): token embedding
+// (phoneme table for the phoneme prefix, codec table for acoustic prompt and
+// generated codes) plus the sinusoidal position of the row.
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace mtp {
+namespace {
+
+__global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
+    __shared__ int s_tok, s_pos, s_act, s_phone;
+    const int r = blockIdx.x, tid = threadIdx.x;
+    pdl_launch_dependents();
+    pdl_wait();
+    if (tid == 0) {
+        int seq = -1, pos = 0, tok = 0, phone = 0, last = 0;
+        if (a.mode == 0) {  // decode: row r is fed token j of slot seq_base + r / n
+            const int b = a.seq_base + r / a.n_heads, j = r % a.n_heads;
+            if (r < a.rows && b < a.slots && a.active[b] && !a.done[b] && j < a.n_pending[b]) {
+                seq = b;
+                pos = a.seq_len[b] + j;
+                tok = a.pending[b * a.n_max + j];
+                last = (j == a.n_pending[b] - 1);
+            }
+        } else {  // prefill chunk: positions p0 .. p0 + rows - 1 of one slot
+            pos = a.p0 + r;
+            if (r < a.rows && pos < a.total) {
+                seq = a.slot;
+                tok = a.prompt[(size_t)a.slot * a.prompt_stride + pos];
+                phone = pos < a.n_ph;
+                last = (pos == a.total - 1);
+            }
+        }
+        if (seq >= 0 && (pos >= a.max_pos || tok < 0 || tok >= (phone ? a.phone_vocab : a.codec_vocab))) {
+            atomicOr(a.err, ERR_BOUNDS);
+            seq = -1;
+        }
+        a.row_seq[r] = seq;
+        a.row_pos[r] = seq >= 0 ? pos : -1;
+        a.row_last[r] = seq >= 0 ? last : 0;
+        s_act = seq >= 0;
+        s_tok = tok;
+        s_pos = pos;
+        s_phone = phone;
+    }
+    __syncthreads();
+    float* x = a.x + (size_t)r * a.d;
+    if (!s_act) {
+        for (int i = tid; i < a.d; i += blockDim.x) x[i] = 0.f;
+        return;
+    }
+    const float* pe = a.pe + (size_t)s_pos * a.d;
+    const void* table = s_phone ? a.tok_phone : a.tok_codec;
+    for (int i = tid; i < a.d; i += blockDim.x) {
+        float e;
+        if (a.w_bf16) {
+            const uint16_t bits = reinterpret_cast<const uint16_t*>(table)[(size_t)s_tok * a.d + i];
+            e = __uint_as_float((uint32_t)bits << 16);
+        } else {
+            e = reinterpret_cast<const float*>(table)[(size_t)s_tok * a.d + i];
+        }
+        x[i] = e + pe[i];
+    }
+}
+
+// PE[p, 2i] = sin(p * 10000^(-2i/d)), PE[p, 2i+1] = cos(same), in double, stored fp32.
+__global__ void pe_kernel(float* pe, int max_ctx, int d) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)max_ctx * (d / 2)) return;
+    const int p = (int)(idx / (d / 2)), i = (int)(idx % (d / 2));
+    const double inv_freq = pow(10000.0, -2.0 * i / d);
+    const double ang = (double)p * inv_freq;
+    pe[(size_t)p * d + 2 * i] = (float)sin(ang);
+    pe[(size_t)p * d + 2 * i + 1] = (float)cos(ang);
+}
+
+__global__ void convert_rows_kernel(const void* src, int src_bf16, float* dst, long long n) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    dst[i] = src_bf16 ? __uint_as_float((uint32_t)reinterpret_cast<const uint16_t*>(src)[i] << 16)
+                      : reinterpret_cast<const float*>(src)[i];
+}
+
+__global__ void slot_set_kernel(SlotSet s) {
+    if (threadIdx.x != 0) return;
+    pdl_wait();
+    const int b = s.slot;
+    if (s.set_len >= 0) s.seq_len[b] = s.set_len;
+    if (s.set_pending >= 0) s.n_pending[b] = s.set_pending;
+    if (s.set_remaining >= 0) s.remaining[b] = s.set_remaining;
+    if (s.set_done >= 0) s.done[b] = s.set_done;
+    if (s.set_active >= 0) s.active[b] = s.set_active;
+    if (s.set_gen >= 0) s.gen_count[b] = s.set_gen;
+}
+
+}  // namespace
+
+cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(MAX_ROWS);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, embed_kernel, a);
+}
+
+cudaError_t launch_pe_table(float* pe, int max_ctx, int d, cudaStream_t s) {
+    const long long n = (long long)max_ctx * (d / 2);
+    pe_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(pe, max_ctx, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert_rows(const void* src, int src_bf16, float* dst, int rows, int d, cudaStream_t s) {
+    const long long n = (long long)rows * d;
+    convert_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(src, src_bf16, dst, n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s) {
+    slot_set_kernel<<<1, 32, 0, s>>>(set);
+    return cudaGetLastError();
+}
+
+}  // namespace mtp

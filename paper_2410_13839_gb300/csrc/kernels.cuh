@@ -1,0 +1,130 @@
+// kernels.cuh -- argument blocks and host launchers of libmtp's kernels.
+//
+// Each launcher enqueues one kernel on `stream`.  With `pdl` set the launch
+// carries the programmatic-stream-serialisation attribute: the kernel may
+// start while its predecessor is still running, prefetches what does not
+// depend on it (weights, old keys/values), then waits (griddepcontrol.wait).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace mtp {
+
+constexpr int HEAD_DIM = 64;     // attention head width (fixed by the kernels)
+constexpr int MAX_ROWS = 8;      // rows per weight-streaming pass (B * n_heads per chunk)
+constexpr int MAX_TOPK = 32;     // one warp lane per candidate
+constexpr int MAX_NHEADS = 8;    // prediction heads
+constexpr int MAX_VOCAB = 1056;  // 33 logits per lane in the top-k warp
+
+// ---------------------------------------------------------------- GEMV ----
+// y[m, f] = epilogue( sum_k A'[m, k] W[f, k] + bias[f] ),  A' = LN(A) if ln_g.
+enum Epilogue : int {
+    EPI_QKV = 0,     // f < d: q[m, f];  d <= f < 3d: key/value into the KV page pool
+    EPI_RESID = 1,   // out[m, f] += y   (residual stream); optional h_last copy
+    EPI_GELU = 2,    // out[m, f] = GELU(y)
+    EPI_LOGITS = 3,  // out[m, f] = y
+};
+
+struct GemvArgs {
+    const float* A; int lda;             // input rows [M][K] fp32
+    const float* ln_g; const float* ln_b; float ln_eps;  // LayerNorm prologue (ln_g null: none)
+    const void* W;                       // [N][K] row-major, bf16 or fp32
+    const float* bias;                   // [N]
+    int N, K, M;                         // M <= rows of the instantiation
+    int rows_per_cta;
+    const int* row_seq;                  // [M] slot of each row, < 0 inactive (null: all active)
+    const int* row_pos;                  // [M] position of each row (EPI_QKV)
+    const int* row_last;                 // [M] 1 if the row is its slot's last fed row
+    float* out; int ldo;                 // q / residual / hidden / logits
+    float* h_last; int ld_h;             // EPI_RESID: copy of the final row per slot (may be null)
+    // EPI_QKV key/value placement
+    uint16_t* kv_pool; long long page_elems; long long layer_off; int n_heads, page_size, d_model;
+    const int* block_table; int bt_stride;
+    int* err;
+};
+
+size_t gemv_smem_bytes(int rows_per_cta, int K, int wbytes, int M);
+cudaError_t launch_gemv(const GemvArgs& a, int epi, bool ln, bool w_bf16, int grid, cudaStream_t s, bool pdl);
+
+// ----------------------------------------------------------- attention ----
+enum AttnPlan : int {
+    PLAN_ROWS = 0,    // slot and key count read from row_seq/row_pos after the wait
+    PLAN_DEVICE = 1,  // slot = seq_base + group; old length and new count from device state
+    PLAN_VALUE = 2,   // one group: slot, old length and new count passed by value
+};
+
+struct AttnArgs {
+    const float* q; int ldq;                   // [rows][H*64]
+    const __nv_bfloat16* kv_pool; long long page_elems; long long layer_off;
+    const int* block_table; int bt_stride;
+    const int* row_seq; const int* row_pos;
+    float* out; int ldo;
+    float* ws_part; int* ws_count;             // split partials and per-(group, head) counters
+    int rows_per_group, n_heads, page_size, n_splits;
+    int plan;
+    const int* seq_len; const int* seq_new; int seq_base;   // PLAN_DEVICE
+    int val_seq, val_old, val_new;                           // PLAN_VALUE
+    int* err;
+};
+
+size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
+size_t attn_smem_bytes(int page_size);
+int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms);
+cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl);
+
+// --------------------------------------------------------------- embed ----
+struct EmbedArgs {
+    int mode;                  // 0 = decode rows from slot state, 1 = prefill chunk
+    const void* tok_phone; const void* tok_codec; int w_bf16;
+    int phone_vocab, codec_vocab;
+    const float* pe; int d; int max_pos;   // positional table [max_pos][d]
+    float* x;                  // [MAX_ROWS][d]
+    int* row_seq; int* row_pos; int* row_last;
+    int rows;                  // rows in this pass (<= MAX_ROWS); the rest are inactive
+    // decode
+    int seq_base, n_heads, n_max, slots;
+    const int* active; const int* done; const int* n_pending; const int* pending; const int* seq_len;
+    // prefill
+    int slot, p0, n_ph, total, prompt_stride; const int* prompt;
+    int* err;
+};
+cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_pe_table(float* pe, int max_ctx, int d, cudaStream_t s);
+
+// -------------------------------------------------------------- select ----
+struct SelectArgs {
+    const float* logits;      // [B][n][V]
+    float* lse;               // [B][n]
+    int32_t* cand_ids; float* cand_logp;   // [B][n][k]
+    int32_t* path;            // [B][n]
+    const float* log_q;       // [V][V]
+    int n, k, V, eos_id, n_max, seq_base;
+    // slot state (decode); null for the stand-alone heads call
+    int* active; int* done; int* n_pending; int* pending; int* seq_len; int* remaining;
+    int* gen_count; int* gen_tokens; int gen_stride;
+    int* out_tokens; int* out_accepted;   // [B][n_max], [B]
+    int* err;
+};
+cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
+
+struct ViterbiArgs {
+    int batch, n, k, vocab, eos_id;
+    const int32_t* cand_ids; const float* cand_logp; const float* log_q; const int32_t* remaining;
+    int32_t* path; float* score; int32_t* accepted; int32_t* rollback;
+};
+cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s);
+
+// --------------------------------------------------------------- misc ----
+cudaError_t launch_convert_rows(const void* src, int src_bf16, float* dst, int rows, int d, cudaStream_t s);
+
+// set fields of one slot's device state (a field is left alone when its value is < 0)
+struct SlotSet {
+    int slot;
+    int* seq_len; int* n_pending; int* remaining; int* done; int* active; int* gen_count;
+    int set_len, set_pending, set_remaining, set_done, set_active, set_gen;
+};
+cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s);
+
+}  // namespace mtp

@@ -1,0 +1,919 @@
+// mtp_api.cu -- the C ABI of include/mtp.h over libmtp's kernels.
+//
+// Host runtime: weight upload, KV page allocator (host free list, device
+// block table), slot state kept on the device, and the step orchestration:
+//   decode step = for each chunk of <= 8 fed rows: embed, then per layer
+//                 [LN1+QKV+KV append, attention, O-proj+residual,
+//                  LN2+FFN1+GELU, FFN2+residual]; then the heads
+//                 (LN_f + n x V logits) and one select kernel (log-softmax,
+//                 top-k, Viterbi, acceptance, slot bookkeeping);
+//   prefill      = the same layer stack over the prompt in chunks of 8 rows.
+// Within a pass the kernels are chained with programmatic dependent launch;
+// each (n_heads, top_k) decode step is captured once into a CUDA graph.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "kernels.cuh"
+#include "mtp.h"
+
+using namespace mtp;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+#define CUDA_TRY(expr)                                                                                  \
+    do {                                                                                                \
+        cudaError_t e_ = (expr);                                                                        \
+        if (e_ != cudaSuccess)                                                                          \
+            return fail(MTP_ERR_CUDA, "%s: %s (%s:%d)", #expr, cudaGetErrorString(e_), __FILE__, __LINE__); \
+    } while (0)
+
+#define MTP_TRY(expr)              \
+    do {                           \
+        int r_ = (expr);           \
+        if (r_ != MTP_OK) return r_; \
+    } while (0)
+
+struct Layer {
+    const float *ln1_g, *ln1_b, *bqkv, *bo, *ln2_g, *ln2_b, *b1, *b2;
+    const void *wqkv, *wo, *w1, *w2;
+};
+
+struct Prof {
+    std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev;
+};
+
+bool is_device_ptr(const void* p) {
+    if (!p) return false;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace
+
+struct mtp_ctx {
+    mtp_config cfg{};
+    cudaStream_t stream = nullptr;
+    cudaStream_t cap_stream = nullptr;
+    int device = 0, num_sms = 0, wbytes = 2;
+    bool use_graphs = true, use_pdl = true;
+    std::vector<void*> allocs;
+    // weights
+    void* d_weights = nullptr;
+    const void *tok_phone = nullptr, *tok_codec = nullptr, *w_heads = nullptr;
+    const float *lnf_g = nullptr, *lnf_b = nullptr, *b_heads = nullptr, *log_q = nullptr;
+    std::vector<Layer> layers;
+    float* d_pe = nullptr;
+    // KV cache
+    uint16_t* d_kv = nullptr;
+    int n_pages = 0, pages_per_seq = 0;
+    long long page_elems = 0;
+    std::vector<int> free_pages;
+    std::vector<std::vector<int>> slot_pages;
+    std::vector<int> h_block_table;
+    int* d_block_table = nullptr;
+    // slot state
+    int *d_len = nullptr, *d_npend = nullptr, *d_pending = nullptr, *d_remaining = nullptr, *d_done = nullptr,
+        *d_active = nullptr, *d_gen_count = nullptr, *d_gen_tokens = nullptr, *d_prompt = nullptr;
+    float* d_h_last = nullptr;
+    // step buffers
+    float *d_x = nullptr, *d_q = nullptr, *d_attn = nullptr, *d_u = nullptr, *d_logits = nullptr, *d_lse = nullptr,
+          *d_cand_logp = nullptr;
+    int *d_row_seq = nullptr, *d_row_pos = nullptr, *d_row_last = nullptr, *d_cand_ids = nullptr, *d_path = nullptr,
+        *d_out_tokens = nullptr, *d_out_accepted = nullptr;
+    float* d_ws = nullptr;
+    int* d_ws_count = nullptr;
+    int* d_err = nullptr;
+    std::map<std::pair<int, int>, cudaGraphExec_t> graphs;
+    int last_n = 0, last_k = 0;
+
+    template <typename T>
+    int alloc(T** p, size_t count) {
+        void* q = nullptr;
+        CUDA_TRY(cudaMalloc(&q, std::max<size_t>(count * sizeof(T), 16)));
+        allocs.push_back(q);
+        CUDA_TRY(cudaMemset(q, 0, std::max<size_t>(count * sizeof(T), 16)));
+        *p = static_cast<T*>(q);
+        return MTP_OK;
+    }
+};
+
+namespace {
+
+// ------------------------------------------------------------ launching ----
+
+int record(Prof* prof, int kind, cudaStream_t s, bool start) {
+    if (!prof) return MTP_OK;
+    if (start) {
+        cudaEvent_t a, b;
+        CUDA_TRY(cudaEventCreate(&a));
+        CUDA_TRY(cudaEventCreate(&b));
+        prof->ev.push_back({kind, {a, b}});
+        CUDA_TRY(cudaEventRecord(a, s));
+    } else {
+        CUDA_TRY(cudaEventRecord(prof->ev.back().second.second, s));
+    }
+    return MTP_OK;
+}
+
+#define LAUNCH(kind, expr)                                                                                  \
+    do {                                                                                                   \
+        MTP_TRY(record(prof, kind, s, true));                                                              \
+        cudaError_t e_ = (expr);                                                                           \
+        if (e_ != cudaSuccess)                                                                             \
+            return fail(MTP_ERR_CUDA, "launch %s: %s (%s:%d)", #kind, cudaGetErrorString(e_), __FILE__, __LINE__); \
+        MTP_TRY(record(prof, kind, s, false));                                                             \
+    } while (0)
+
+// CTAs and rows per CTA of a projection: one wave over the SMs while the
+// weight slice fits the shared-memory budget, else more CTAs.
+int gemv_grid(const mtp_ctx* c, int N, int K, int M, int* rpc) {
+    int ctas = c->num_sms;
+    for (;;) {
+        *rpc = (N + ctas - 1) / ctas;
+        if (gemv_smem_bytes(*rpc, K, c->wbytes, M) <= 112 * 1024 || *rpc == 1) break;
+        ctas *= 2;
+    }
+    return (N + *rpc - 1) / *rpc;
+}
+
+GemvArgs gemv_base(mtp_ctx* c) {
+    GemvArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.ln_eps = c->cfg.ln_eps;
+    a.err = c->d_err;
+    a.row_seq = c->d_row_seq;
+    a.row_pos = c->d_row_pos;
+    a.row_last = c->d_row_last;
+    return a;
+}
+
+// The layer stack over the M rows currently in d_x (G groups of rpg rows).
+int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int val_seq, int val_old, int val_new,
+               int max_keys, cudaStream_t s, bool pdl, Prof* prof) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
+    const bool bf = cf.weight_dtype == MTP_BF16;
+    const int S = attn_splits_for(G, H, P, max_keys, c->num_sms);
+    for (int l = 0; l < cf.layers; ++l) {
+        const Layer& L = c->layers[l];
+        const long long layer_off = (long long)l * 2 * H * P * HEAD_DIM;
+        int rpc, grid;
+
+        GemvArgs q = gemv_base(c);
+        q.A = c->d_x; q.lda = d; q.ln_g = L.ln1_g; q.ln_b = L.ln1_b;
+        q.W = L.wqkv; q.bias = L.bqkv; q.N = 3 * d; q.K = d; q.M = M;
+        grid = gemv_grid(c, q.N, q.K, M, &rpc); q.rows_per_cta = rpc;
+        q.out = c->d_q; q.ldo = d;
+        q.kv_pool = c->d_kv; q.page_elems = c->page_elems; q.layer_off = layer_off;
+        q.n_heads = H; q.page_size = P; q.d_model = d;
+        q.block_table = c->d_block_table; q.bt_stride = c->pages_per_seq;
+        LAUNCH(MTP_K_QKV, launch_gemv(q, EPI_QKV, true, bf, grid, s, pdl));
+
+        AttnArgs at;
+        std::memset(&at, 0, sizeof(at));
+        at.q = c->d_q; at.ldq = d;
+        at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(c->d_kv);
+        at.page_elems = c->page_elems; at.layer_off = layer_off;
+        at.block_table = c->d_block_table; at.bt_stride = c->pages_per_seq;
+        at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
+        at.out = c->d_attn; at.ldo = d;
+        at.ws_part = c->d_ws; at.ws_count = c->d_ws_count;
+        at.rows_per_group = rpg; at.n_heads = H; at.page_size = P; at.n_splits = S;
+        at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = seq_base;
+        at.val_seq = val_seq; at.val_old = val_old; at.val_new = val_new;
+        at.err = c->d_err;
+        LAUNCH(MTP_K_ATTN, launch_attention(at, G, s, pdl));
+
+        GemvArgs o = gemv_base(c);
+        o.A = c->d_attn; o.lda = d; o.W = L.wo; o.bias = L.bo; o.N = d; o.K = d; o.M = M;
+        grid = gemv_grid(c, o.N, o.K, M, &rpc); o.rows_per_cta = rpc;
+        o.out = c->d_x; o.ldo = d;
+        LAUNCH(MTP_K_OPROJ, launch_gemv(o, EPI_RESID, false, bf, grid, s, pdl));
+
+        GemvArgs f1 = gemv_base(c);
+        f1.A = c->d_x; f1.lda = d; f1.ln_g = L.ln2_g; f1.ln_b = L.ln2_b;
+        f1.W = L.w1; f1.bias = L.b1; f1.N = F; f1.K = d; f1.M = M;
+        grid = gemv_grid(c, f1.N, f1.K, M, &rpc); f1.rows_per_cta = rpc;
+        f1.out = c->d_u; f1.ldo = F;
+        LAUNCH(MTP_K_FFN1, launch_gemv(f1, EPI_GELU, true, bf, grid, s, pdl));
+
+        GemvArgs f2 = gemv_base(c);
+        f2.A = c->d_u; f2.lda = F; f2.W = L.w2; f2.bias = L.b2; f2.N = d; f2.K = F; f2.M = M;
+        grid = gemv_grid(c, f2.N, f2.K, M, &rpc); f2.rows_per_cta = rpc;
+        f2.out = c->d_x; f2.ldo = d;
+        if (l == cf.layers - 1) {
+            f2.h_last = c->d_h_last;
+            f2.ld_h = d;
+        }
+        LAUNCH(MTP_K_FFN2, launch_gemv(f2, EPI_RESID, false, bf, grid, s, pdl));
+    }
+    return MTP_OK;
+}
+
+EmbedArgs embed_base(mtp_ctx* c) {
+    EmbedArgs e;
+    std::memset(&e, 0, sizeof(e));
+    e.tok_phone = c->tok_phone; e.tok_codec = c->tok_codec;
+    e.w_bf16 = c->cfg.weight_dtype == MTP_BF16;
+    e.phone_vocab = c->cfg.phone_vocab; e.codec_vocab = c->cfg.codec_vocab;
+    e.pe = c->d_pe; e.d = c->cfg.d_model; e.max_pos = c->cfg.max_ctx;
+    e.x = c->d_x; e.row_seq = c->d_row_seq; e.row_pos = c->d_row_pos; e.row_last = c->d_row_last;
+    e.n_max = c->cfg.n_heads_max; e.slots = c->cfg.max_batch;
+    e.active = c->d_active; e.done = c->d_done; e.n_pending = c->d_npend; e.pending = c->d_pending;
+    e.seq_len = c->d_len; e.prompt = c->d_prompt; e.prompt_stride = c->cfg.max_ctx;
+    e.err = c->d_err;
+    return e;
+}
+
+// Heads on h_last of slots [b0, b0 + m) -> logits rows of those slots.
+int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, cudaStream_t s, bool pdl, Prof* prof) {
+    const int d = c->cfg.d_model, V = c->cfg.codec_vocab;
+    GemvArgs h = gemv_base(c);
+    h.A = A; h.lda = d; h.ln_g = c->lnf_g; h.ln_b = c->lnf_b;
+    h.W = c->w_heads; h.bias = c->b_heads; h.N = n * V; h.K = d; h.M = m;
+    int rpc;
+    const int grid = gemv_grid(c, h.N, h.K, m, &rpc);
+    h.rows_per_cta = rpc;
+    h.row_seq = nullptr;
+    h.out = logits; h.ldo = n * V;
+    LAUNCH(MTP_K_HEADS, launch_gemv(h, EPI_LOGITS, true, c->cfg.weight_dtype == MTP_BF16, grid, s, pdl));
+    return MTP_OK;
+}
+
+SelectArgs select_base(mtp_ctx* c, int n, int k) {
+    SelectArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.logits = c->d_logits; a.lse = c->d_lse; a.cand_ids = c->d_cand_ids; a.cand_logp = c->d_cand_logp;
+    a.path = c->d_path; a.log_q = c->log_q;
+    a.n = n; a.k = k; a.V = c->cfg.codec_vocab; a.eos_id = c->cfg.eos_id; a.n_max = c->cfg.n_heads_max;
+    a.active = c->d_active; a.done = c->d_done; a.n_pending = c->d_npend; a.pending = c->d_pending;
+    a.seq_len = c->d_len; a.remaining = c->d_remaining; a.gen_count = c->d_gen_count;
+    a.gen_tokens = c->d_gen_tokens; a.gen_stride = c->cfg.max_ctx;
+    a.out_tokens = c->d_out_tokens; a.out_accepted = c->d_out_accepted;
+    a.err = c->d_err;
+    return a;
+}
+
+int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof) {
+    const int B = c->cfg.max_batch, d = c->cfg.d_model, V = c->cfg.codec_vocab;
+    const int spc = std::max(1, MAX_ROWS / n);
+    for (int b0 = 0; b0 < B; b0 += spc) {
+        const int G = std::min(spc, B - b0), M = G * n;
+        EmbedArgs e = embed_base(c);
+        e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
+        LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));  // full dependency on the previous pass
+        MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, c->cfg.max_ctx, s, pdl, prof));
+    }
+    for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
+        const int m = std::min(MAX_ROWS, B - b0);
+        MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, s, pdl, prof));
+    }
+    SelectArgs sa = select_base(c, n, k);
+    LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
+    return MTP_OK;
+}
+
+int run_step(mtp_ctx* c, int n, int k) {
+    c->last_n = n;
+    c->last_k = k;
+    if (!c->use_graphs) return enqueue_step(c, n, k, c->stream, c->use_pdl, nullptr);
+    auto key = std::make_pair(n, k);
+    auto it = c->graphs.find(key);
+    if (it == c->graphs.end()) {
+        cudaGraph_t graph = nullptr;
+        cudaGraphExec_t exec = nullptr;
+        CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
+        const int r = enqueue_step(c, n, k, c->cap_stream, c->use_pdl, nullptr);
+        const cudaError_t ec = cudaStreamEndCapture(c->cap_stream, &graph);
+        if (r != MTP_OK) {
+            if (graph) cudaGraphDestroy(graph);
+            return r;
+        }
+        CUDA_TRY(ec);
+        const cudaError_t ei = cudaGraphInstantiate(&exec, graph, 0);
+        cudaGraphDestroy(graph);
+        CUDA_TRY(ei);
+        it = c->graphs.emplace(key, exec).first;
+    }
+    CUDA_TRY(cudaGraphLaunch(it->second, c->stream));
+    return MTP_OK;
+}
+
+int check_device_error(mtp_ctx* c) {
+    int err = 0;
+    CUDA_TRY(cudaMemcpyAsync(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    if (err) return fail(MTP_ERR_DEVICE, "device error word 0x%x (1 = bounded wait ran out, 2 = index check)", err);
+    return MTP_OK;
+}
+
+int copy_out(void* dst, const void* src, size_t bytes, cudaStream_t s) {
+    if (!dst || bytes == 0) return MTP_OK;
+    CUDA_TRY(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, s));
+    return MTP_OK;
+}
+
+int slot_set(mtp_ctx* c, int slot, int len, int pend, int rem, int done, int active, int gen) {
+    SlotSet ss;
+    ss.slot = slot;
+    ss.seq_len = c->d_len; ss.n_pending = c->d_npend; ss.remaining = c->d_remaining;
+    ss.done = c->d_done; ss.active = c->d_active; ss.gen_count = c->d_gen_count;
+    ss.set_len = len; ss.set_pending = pend; ss.set_remaining = rem;
+    ss.set_done = done; ss.set_active = active; ss.set_gen = gen;
+    CUDA_TRY(launch_slot_set(ss, c->stream));
+    return MTP_OK;
+}
+
+int read_slot_ints(mtp_ctx* c, const int* dptr, std::vector<int>& out) {
+    out.resize(c->cfg.max_batch);
+    CUDA_TRY(cudaMemcpyAsync(out.data(), dptr, out.size() * sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+int validate_config(const mtp_config& c) {
+    if (c.layers < 1 || c.layers > 256) return fail(MTP_ERR_INVALID, "layers %d out of range", c.layers);
+    if (c.d_model < 256 || c.d_model % 256 || c.d_model > 4096)
+        return fail(MTP_ERR_INVALID, "d_model %d: need a multiple of 256 up to 4096", c.d_model);
+    if (c.n_attn_heads * HEAD_DIM != c.d_model)
+        return fail(MTP_ERR_INVALID, "d_model / n_attn_heads must be %d", HEAD_DIM);
+    if (c.d_ffn < 256 || c.d_ffn % 256 || c.d_ffn > 4096)
+        return fail(MTP_ERR_INVALID, "d_ffn %d: need a multiple of 256 up to 4096", c.d_ffn);
+    if (c.phone_vocab < 1) return fail(MTP_ERR_INVALID, "phone_vocab %d", c.phone_vocab);
+    if (c.codec_vocab < 2 || c.codec_vocab > MAX_VOCAB)
+        return fail(MTP_ERR_INVALID, "codec_vocab %d: need 2..%d", c.codec_vocab, MAX_VOCAB);
+    if (c.eos_id < 0 || c.eos_id >= c.codec_vocab) return fail(MTP_ERR_INVALID, "eos_id %d", c.eos_id);
+    if (c.n_heads_max < 1 || c.n_heads_max > MAX_NHEADS)
+        return fail(MTP_ERR_INVALID, "n_heads_max %d: need 1..%d", c.n_heads_max, MAX_NHEADS);
+    if (c.top_k_max < 1 || c.top_k_max > MAX_TOPK || c.top_k_max > c.codec_vocab)
+        return fail(MTP_ERR_INVALID, "top_k_max %d: need 1..%d", c.top_k_max, MAX_TOPK);
+    if (c.max_batch < 1 || c.max_batch > 1024) return fail(MTP_ERR_INVALID, "max_batch %d", c.max_batch);
+    if (c.max_ctx < 2 || c.max_ctx > (1 << 20)) return fail(MTP_ERR_INVALID, "max_ctx %d", c.max_ctx);
+    if (c.page_size != 16 && c.page_size != 32 && c.page_size != 64 && c.page_size != 128)
+        return fail(MTP_ERR_INVALID, "page_size %d: need 16, 32, 64 or 128", c.page_size);
+    if (c.n_pages < 0) return fail(MTP_ERR_INVALID, "n_pages %d", c.n_pages);
+    if (c.weight_dtype != MTP_F32 && c.weight_dtype != MTP_BF16)
+        return fail(MTP_ERR_INVALID, "weight_dtype %d", c.weight_dtype);
+    if (c.accept_policy != MTP_ACCEPT_ALL) return fail(MTP_ERR_INVALID, "accept_policy %d", c.accept_policy);
+    if (!(c.ln_eps > 0.f)) return fail(MTP_ERR_INVALID, "ln_eps must be > 0");
+    return MTP_OK;
+}
+
+struct TensorSpec {
+    size_t numel;
+    bool matrix;
+};
+
+std::vector<TensorSpec> blob_specs(const mtp_config& c) {
+    const size_t d = c.d_model, F = c.d_ffn, V = c.codec_vocab;
+    std::vector<TensorSpec> t;
+    t.push_back({(size_t)c.phone_vocab * d, true});
+    t.push_back({V * d, true});
+    for (int l = 0; l < c.layers; ++l) {
+        t.push_back({d, false}); t.push_back({d, false});
+        t.push_back({3 * d * d, true}); t.push_back({3 * d, false});
+        t.push_back({d * d, true}); t.push_back({d, false});
+        t.push_back({d, false}); t.push_back({d, false});
+        t.push_back({F * d, true}); t.push_back({F, false});
+        t.push_back({d * F, true}); t.push_back({d, false});
+    }
+    t.push_back({d, false}); t.push_back({d, false});
+    t.push_back({(size_t)c.n_heads_max * V * d, true});
+    t.push_back({(size_t)c.n_heads_max * V, false});
+    t.push_back({V * V, false});
+    return t;
+}
+
+int upload_weights(mtp_ctx* c, const void* blob, size_t bytes) {
+    const mtp_config& cf = c->cfg;
+    const unsigned char* b = static_cast<const unsigned char*>(blob);
+    if (!blob || bytes < 24) return fail(MTP_ERR_WEIGHTS, "weight blob missing or shorter than its header");
+    if (std::memcmp(b, "MTPWGT01", 8) != 0) return fail(MTP_ERR_WEIGHTS, "bad weight blob magic");
+    uint32_t version, n_t;
+    std::memcpy(&version, b + 8, 4);
+    std::memcpy(&n_t, b + 12, 4);
+    const std::vector<TensorSpec> specs = blob_specs(cf);
+    if (version != 1) return fail(MTP_ERR_WEIGHTS, "weight blob version %u (expected 1)", version);
+    if (n_t != specs.size()) return fail(MTP_ERR_WEIGHTS, "blob has %u tensors, config needs %zu", n_t, specs.size());
+    if (bytes < 24 + 16 * (size_t)n_t) return fail(MTP_ERR_WEIGHTS, "blob shorter than its tensor table");
+    std::vector<size_t> dev_off(n_t);
+    size_t total = 0;
+    for (uint32_t i = 0; i < n_t; ++i) {
+        uint64_t off, nb;
+        std::memcpy(&off, b + 24 + 16 * i, 8);
+        std::memcpy(&nb, b + 24 + 16 * i + 8, 8);
+        const size_t want = specs[i].numel * (specs[i].matrix ? c->wbytes : 4);
+        if (nb != want) return fail(MTP_ERR_WEIGHTS, "tensor %u has %llu bytes, config needs %zu", i,
+                                    (unsigned long long)nb, want);
+        if (off % 256 || off + nb > bytes) return fail(MTP_ERR_WEIGHTS, "tensor %u offset %llu invalid", i,
+                                                        (unsigned long long)off);
+        dev_off[i] = total;
+        total += align256(nb);
+    }
+    unsigned char* dw = nullptr;
+    MTP_TRY(c->alloc(&dw, total));
+    c->d_weights = dw;
+    for (uint32_t i = 0; i < n_t; ++i) {
+        uint64_t off, nb;
+        std::memcpy(&off, b + 24 + 16 * i, 8);
+        std::memcpy(&nb, b + 24 + 16 * i + 8, 8);
+        CUDA_TRY(cudaMemcpy(dw + dev_off[i], b + off, nb, cudaMemcpyHostToDevice));
+    }
+    size_t i = 0;
+    auto nxt = [&]() { return static_cast<const void*>(dw + dev_off[i++]); };
+    c->tok_phone = nxt();
+    c->tok_codec = nxt();
+    c->layers.resize(cf.layers);
+    for (int l = 0; l < cf.layers; ++l) {
+        Layer& L = c->layers[l];
+        L.ln1_g = (const float*)nxt(); L.ln1_b = (const float*)nxt();
+        L.wqkv = nxt(); L.bqkv = (const float*)nxt();
+        L.wo = nxt(); L.bo = (const float*)nxt();
+        L.ln2_g = (const float*)nxt(); L.ln2_b = (const float*)nxt();
+        L.w1 = nxt(); L.b1 = (const float*)nxt();
+        L.w2 = nxt(); L.b2 = (const float*)nxt();
+    }
+    c->lnf_g = (const float*)nxt();
+    c->lnf_b = (const float*)nxt();
+    c->w_heads = nxt();
+    c->b_heads = (const float*)nxt();
+    c->log_q = (const float*)nxt();
+    return MTP_OK;
+}
+
+void release_slot_pages(mtp_ctx* c, int slot) {
+    for (int p : c->slot_pages[slot]) c->free_pages.push_back(p);
+    c->slot_pages[slot].clear();
+    std::fill(c->h_block_table.begin() + (size_t)slot * c->pages_per_seq,
+              c->h_block_table.begin() + (size_t)(slot + 1) * c->pages_per_seq, -1);
+}
+
+int check_ctx(mtp_ctx* c) {
+    if (!c) return fail(MTP_ERR_INVALID, "null context");
+    return MTP_OK;
+}
+
+int check_slot(mtp_ctx* c, int slot) {
+    MTP_TRY(check_ctx(c));
+    if (slot < 0 || slot >= c->cfg.max_batch) return fail(MTP_ERR_INVALID, "slot %d out of range", slot);
+    return MTP_OK;
+}
+
+int check_nk(mtp_ctx* c, int n, int k) {
+    if (n < 1 || n > c->cfg.n_heads_max) return fail(MTP_ERR_INVALID, "n_heads %d: need 1..%d", n, c->cfg.n_heads_max);
+    if (k < 1 || k > c->cfg.top_k_max) return fail(MTP_ERR_INVALID, "top_k %d: need 1..%d", k, c->cfg.top_k_max);
+    return MTP_OK;
+}
+
+void destroy(mtp_ctx* c) {
+    if (!c) return;
+    for (auto& g : c->graphs) cudaGraphExecDestroy(g.second);
+    for (void* p : c->allocs) cudaFree(p);
+    if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+    delete c;
+}
+
+}  // namespace
+
+// ================================================================ C ABI ====
+
+extern "C" {
+
+MTP_API const char* mtp_last_error(void) { return g_err.c_str(); }
+
+MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_t blob_bytes, void* cuda_stream,
+                       mtp_ctx** out) {
+    g_err.clear();
+    if (!config || !out) return fail(MTP_ERR_INVALID, "null config or output handle");
+    *out = nullptr;
+    MTP_TRY(validate_config(*config));
+    mtp_ctx* c = new mtp_ctx();
+    c->cfg = *config;
+    c->stream = static_cast<cudaStream_t>(cuda_stream);
+    c->wbytes = config->weight_dtype == MTP_BF16 ? 2 : 4;
+    auto bail = [&](int r) {
+        destroy(c);
+        return r;
+    };
+    int r;
+    if (cudaGetDevice(&c->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess) {
+        cudaGetLastError();
+        return bail(fail(MTP_ERR_CUDA, "no usable CUDA device"));
+    }
+    if (cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+        return bail(fail(MTP_ERR_CUDA, "cudaStreamCreateWithFlags failed"));
+    const mtp_config& cf = c->cfg;
+    if ((r = upload_weights(c, weights_blob, blob_bytes)) != MTP_OK) return bail(r);
+
+    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size, B = cf.max_batch;
+    const int V = cf.codec_vocab, nm = cf.n_heads_max;
+    c->pages_per_seq = (cf.max_ctx + P - 1) / P;
+    c->n_pages = cf.n_pages > 0 ? cf.n_pages : B * c->pages_per_seq;
+    c->page_elems = (long long)cf.layers * 2 * H * P * HEAD_DIM;
+    // projection slices must fit shared memory
+    for (int K : {d, F}) {
+        int rpc;
+        gemv_grid(c, 3 * d, K, MAX_ROWS, &rpc);
+        if (gemv_smem_bytes(rpc, K, c->wbytes, MAX_ROWS) > 200 * 1024)
+            return bail(fail(MTP_ERR_INVALID, "weight rows of width %d do not fit shared memory", K));
+    }
+    const int S_max = std::max(1, c->num_sms / H) + 1;
+    const size_t ws_floats = attn_workspace_floats(MAX_ROWS, H, S_max, MAX_ROWS);
+    const int lb = std::max(B, MAX_ROWS);
+    if ((r = c->alloc(&c->d_pe, (size_t)cf.max_ctx * d)) ||
+        (r = c->alloc(&c->d_kv, (size_t)c->n_pages * c->page_elems)) ||
+        (r = c->alloc(&c->d_block_table, (size_t)B * c->pages_per_seq)) ||
+        (r = c->alloc(&c->d_len, B)) || (r = c->alloc(&c->d_npend, B)) ||
+        (r = c->alloc(&c->d_pending, (size_t)B * nm)) || (r = c->alloc(&c->d_remaining, B)) ||
+        (r = c->alloc(&c->d_done, B)) || (r = c->alloc(&c->d_active, B)) || (r = c->alloc(&c->d_gen_count, B)) ||
+        (r = c->alloc(&c->d_gen_tokens, (size_t)B * cf.max_ctx)) ||
+        (r = c->alloc(&c->d_prompt, (size_t)B * cf.max_ctx)) || (r = c->alloc(&c->d_h_last, (size_t)lb * d)) ||
+        (r = c->alloc(&c->d_x, (size_t)MAX_ROWS * d)) || (r = c->alloc(&c->d_q, (size_t)MAX_ROWS * d)) ||
+        (r = c->alloc(&c->d_attn, (size_t)MAX_ROWS * d)) || (r = c->alloc(&c->d_u, (size_t)MAX_ROWS * F)) ||
+        (r = c->alloc(&c->d_logits, (size_t)lb * nm * V)) || (r = c->alloc(&c->d_lse, (size_t)lb * nm)) ||
+        (r = c->alloc(&c->d_cand_logp, (size_t)lb * nm * MAX_TOPK)) ||
+        (r = c->alloc(&c->d_cand_ids, (size_t)lb * nm * MAX_TOPK)) || (r = c->alloc(&c->d_path, (size_t)lb * nm)) ||
+        (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
+        (r = c->alloc(&c->d_row_seq, MAX_ROWS)) || (r = c->alloc(&c->d_row_pos, MAX_ROWS)) ||
+        (r = c->alloc(&c->d_row_last, MAX_ROWS)) || (r = c->alloc(&c->d_ws, ws_floats)) ||
+        (r = c->alloc(&c->d_ws_count, (size_t)MAX_ROWS * H)) || (r = c->alloc(&c->d_err, 1)))
+        return bail(r);
+    c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
+    if (cudaMemcpy(c->d_block_table, c->h_block_table.data(), c->h_block_table.size() * sizeof(int),
+                   cudaMemcpyHostToDevice) != cudaSuccess)
+        return bail(fail(MTP_ERR_CUDA, "block table upload failed"));
+    c->slot_pages.assign(B, {});
+    for (int p = c->n_pages - 1; p >= 0; --p) c->free_pages.push_back(p);
+    if (launch_pe_table(c->d_pe, cf.max_ctx, d, c->stream) != cudaSuccess ||
+        cudaStreamSynchronize(c->stream) != cudaSuccess)
+        return bail(fail(MTP_ERR_CUDA, "position table: %s", cudaGetErrorString(cudaGetLastError())));
+    *out = c;
+    return MTP_OK;
+}
+
+MTP_API void mtp_destroy(mtp_ctx* ctx) {
+    if (!ctx) return;
+    cudaStreamSynchronize(ctx->stream);
+    destroy(ctx);
+}
+
+MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (option == MTP_OPT_GRAPHS) {
+        c->use_graphs = value != 0;
+    } else if (option == MTP_OPT_PDL) {
+        if (c->use_pdl != (value != 0)) {
+            for (auto& g : c->graphs) cudaGraphExecDestroy(g.second);
+            c->graphs.clear();
+        }
+        c->use_pdl = value != 0;
+    } else {
+        return fail(MTP_ERR_INVALID, "unknown option %d", option);
+    }
+    return MTP_OK;
+}
+
+MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic, int n_ac,
+                        int max_new_tokens) {
+    g_err.clear();
+    MTP_TRY(check_slot(c, slot));
+    const mtp_config& cf = c->cfg;
+    if (n_ph < 0 || n_ac < 0 || n_ph + n_ac < 1) return fail(MTP_ERR_INVALID, "empty prompt");
+    if ((n_ph && !phonemes) || (n_ac && !acoustic)) return fail(MTP_ERR_INVALID, "null prompt pointer");
+    if (max_new_tokens < 1) return fail(MTP_ERR_INVALID, "max_new_tokens %d", max_new_tokens);
+    const long long T = (long long)n_ph + n_ac;
+    const long long need = T + max_new_tokens + cf.n_heads_max;
+    if (need > cf.max_ctx)
+        return fail(MTP_ERR_INVALID, "prompt %lld + max_new %d + n_heads_max %d exceeds max_ctx %d", T,
+                    max_new_tokens, cf.n_heads_max, cf.max_ctx);
+    // host-side id checks (device prompts are checked by the embedding kernel)
+    const bool ph_dev = is_device_ptr(phonemes), ac_dev = is_device_ptr(acoustic);
+    if (!ph_dev)
+        for (int i = 0; i < n_ph; ++i)
+            if (phonemes[i] < 0 || phonemes[i] >= cf.phone_vocab)
+                return fail(MTP_ERR_INVALID, "phoneme id %d at %d out of range", phonemes[i], i);
+    if (!ac_dev)
+        for (int i = 0; i < n_ac; ++i)
+            if (acoustic[i] < 0 || acoustic[i] >= cf.codec_vocab)
+                return fail(MTP_ERR_INVALID, "acoustic id %d at %d out of range", acoustic[i], i);
+    release_slot_pages(c, slot);
+    const int P = cf.page_size;
+    const int n_pages = (int)((need + P - 1) / P);
+    if ((int)c->free_pages.size() < n_pages)
+        return fail(MTP_ERR_NO_PAGES, "slot %d needs %d pages, %zu free", slot, n_pages, c->free_pages.size());
+    for (int i = 0; i < n_pages; ++i) {
+        const int p = c->free_pages.back();
+        c->free_pages.pop_back();
+        c->slot_pages[slot].push_back(p);
+        c->h_block_table[(size_t)slot * c->pages_per_seq + i] = p;
+    }
+    cudaStream_t s = c->stream;
+    CUDA_TRY(cudaMemcpyAsync(c->d_block_table + (size_t)slot * c->pages_per_seq,
+                             c->h_block_table.data() + (size_t)slot * c->pages_per_seq,
+                             c->pages_per_seq * sizeof(int), cudaMemcpyHostToDevice, s));
+    int* prompt = c->d_prompt + (size_t)slot * cf.max_ctx;
+    if (n_ph) CUDA_TRY(cudaMemcpyAsync(prompt, phonemes, n_ph * sizeof(int), cudaMemcpyDefault, s));
+    if (n_ac) CUDA_TRY(cudaMemcpyAsync(prompt + n_ph, acoustic, n_ac * sizeof(int), cudaMemcpyDefault, s));
+    MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0));
+    Prof* prof = nullptr;
+    for (int p0 = 0; p0 < T; p0 += MAX_ROWS) {
+        const int m = (int)std::min<long long>(MAX_ROWS, T - p0);
+        EmbedArgs e = embed_base(c);
+        e.mode = 1; e.rows = m; e.slot = slot; e.p0 = p0; e.n_ph = n_ph; e.total = (int)T;
+        LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
+        MTP_TRY(run_layers(c, m, 1, m, PLAN_VALUE, 0, slot, p0, m, p0 + m, s, c->use_pdl, prof));
+    }
+    MTP_TRY(slot_set(c, slot, (int)T, -1, -1, -1, -1, -1));
+    // pageable host prompts: copies above are complete when the call returns
+    return MTP_OK;
+}
+
+MTP_API int mtp_release(mtp_ctx* c, int slot) {
+    g_err.clear();
+    MTP_TRY(check_slot(c, slot));
+    release_slot_pages(c, slot);
+    CUDA_TRY(cudaMemcpyAsync(c->d_block_table + (size_t)slot * c->pages_per_seq,
+                             c->h_block_table.data() + (size_t)slot * c->pages_per_seq,
+                             c->pages_per_seq * sizeof(int), cudaMemcpyHostToDevice, c->stream));
+    MTP_TRY(slot_set(c, slot, 0, 0, 0, 0, 0, 0));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_decode_step(mtp_ctx* c, int n, int k, int32_t* out_tokens, int32_t* out_accepted,
+                            int32_t* out_done) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    MTP_TRY(check_nk(c, n, k));
+    MTP_TRY(run_step(c, n, k));
+    const int B = c->cfg.max_batch, nm = c->cfg.n_heads_max;
+    if (out_tokens)
+        CUDA_TRY(cudaMemcpy2DAsync(out_tokens, n * sizeof(int), c->d_out_tokens, nm * sizeof(int), n * sizeof(int), B,
+                                   cudaMemcpyDefault, c->stream));
+    MTP_TRY(copy_out(out_accepted, c->d_out_accepted, B * sizeof(int), c->stream));
+    MTP_TRY(copy_out(out_done, c->d_done, B * sizeof(int), c->stream));
+    const bool host_io = (out_tokens && !is_device_ptr(out_tokens)) || (out_accepted && !is_device_ptr(out_accepted)) ||
+                         (out_done && !is_device_ptr(out_done));
+    if (host_io) MTP_TRY(check_device_error(c));
+    return MTP_OK;
+}
+
+MTP_API int mtp_generate(mtp_ctx* c, int n, int k, int32_t* out_tokens, int out_stride, int32_t* out_lens) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    MTP_TRY(check_nk(c, n, k));
+    if (out_tokens && out_stride < 1) return fail(MTP_ERR_INVALID, "out_stride %d", out_stride);
+    std::vector<int> rem, done, active;
+    MTP_TRY(read_slot_ints(c, c->d_remaining, rem));
+    MTP_TRY(read_slot_ints(c, c->d_done, done));
+    MTP_TRY(read_slot_ints(c, c->d_active, active));
+    int steps = 0;
+    for (int b = 0; b < c->cfg.max_batch; ++b)
+        if (active[b] && !done[b]) steps = std::max(steps, (rem[b] + n - 1) / n);
+    for (int i = 0; i < steps; ++i) MTP_TRY(run_step(c, n, k));
+    MTP_TRY(check_device_error(c));
+    const int B = c->cfg.max_batch, gs = c->cfg.max_ctx;
+    if (out_tokens) {
+        const int w = std::min(out_stride, gs);
+        CUDA_TRY(cudaMemcpy2DAsync(out_tokens, out_stride * sizeof(int), c->d_gen_tokens, gs * sizeof(int),
+                                   w * sizeof(int), B, cudaMemcpyDefault, c->stream));
+    }
+    MTP_TRY(copy_out(out_lens, c->d_gen_count, B * sizeof(int), c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return steps;
+}
+
+MTP_API int mtp_rollback(mtp_ctx* c, int slot, int n_tokens) {
+    g_err.clear();
+    MTP_TRY(check_slot(c, slot));
+    std::vector<int> len;
+    MTP_TRY(read_slot_ints(c, c->d_len, len));
+    if (n_tokens < 0 || n_tokens > len[slot])
+        return fail(MTP_ERR_INVALID, "cannot roll back %d of %d cached tokens", n_tokens, len[slot]);
+    MTP_TRY(slot_set(c, slot, len[slot] - n_tokens, -1, -1, -1, -1, -1));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_set_teacher_tokens(mtp_ctx* c, int slot, const int32_t* tokens, int n) {
+    g_err.clear();
+    MTP_TRY(check_slot(c, slot));
+    if (!tokens || n < 1 || n > c->cfg.n_heads_max)
+        return fail(MTP_ERR_INVALID, "teacher tokens: need 1..%d host ids", c->cfg.n_heads_max);
+    for (int i = 0; i < n; ++i)
+        if (tokens[i] < 0 || tokens[i] >= c->cfg.codec_vocab)
+            return fail(MTP_ERR_INVALID, "teacher token %d out of range", tokens[i]);
+    CUDA_TRY(cudaMemcpyAsync(c->d_pending + (size_t)slot * c->cfg.n_heads_max, tokens, n * sizeof(int),
+                             cudaMemcpyHostToDevice, c->stream));
+    MTP_TRY(slot_set(c, slot, -1, n, -1, -1, -1, -1));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_seq_state(mtp_ctx* c, int slot, int32_t* out6) {
+    g_err.clear();
+    MTP_TRY(check_slot(c, slot));
+    if (!out6) return fail(MTP_ERR_INVALID, "null output");
+    const int* src[6] = {c->d_len, c->d_npend, c->d_remaining, c->d_done, c->d_active, c->d_gen_count};
+    for (int i = 0; i < 6; ++i)
+        CUDA_TRY(cudaMemcpyAsync(out6 + i, src[i] + slot, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_debug_logits(mtp_ctx* c, float* out_logits, float* out_lse) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (c->last_n == 0) return fail(MTP_ERR_INVALID, "no decode step has run");
+    const size_t B = c->cfg.max_batch, n = c->last_n, V = c->cfg.codec_vocab;
+    MTP_TRY(copy_out(out_logits, c->d_logits, B * n * V * sizeof(float), c->stream));
+    MTP_TRY(copy_out(out_lse, c->d_lse, B * n * sizeof(float), c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_debug_lattice(mtp_ctx* c, int32_t* out_ids, float* out_logp, int32_t* out_path) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (c->last_n == 0) return fail(MTP_ERR_INVALID, "no decode step has run");
+    const size_t B = c->cfg.max_batch, n = c->last_n, k = c->last_k;
+    MTP_TRY(copy_out(out_ids, c->d_cand_ids, B * n * k * sizeof(int), c->stream));
+    MTP_TRY(copy_out(out_logp, c->d_cand_logp, B * n * k * sizeof(float), c->stream));
+    MTP_TRY(copy_out(out_path, c->d_path, B * n * sizeof(int), c->stream));
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    return MTP_OK;
+}
+
+MTP_API int mtp_profile_step(mtp_ctx* c, int n, int k, float* out_ms, int32_t* out_launches) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    MTP_TRY(check_nk(c, n, k));
+    Prof prof;
+    c->last_n = n;
+    c->last_k = k;
+    const int r = enqueue_step(c, n, k, c->stream, false, &prof);
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    for (int i = 0; i < MTP_K_COUNT; ++i) {
+        if (out_ms) out_ms[i] = 0.f;
+        if (out_launches) out_launches[i] = 0;
+    }
+    for (auto& ev : prof.ev) {
+        float ms = 0.f;
+        if (r == MTP_OK && e == cudaSuccess) e = cudaEventElapsedTime(&ms, ev.second.first, ev.second.second);
+        if (out_ms) out_ms[ev.first] += ms;
+        if (out_launches) out_launches[ev.first] += 1;
+        cudaEventDestroy(ev.second.first);
+        cudaEventDestroy(ev.second.second);
+    }
+    if (r != MTP_OK) return r;
+    CUDA_TRY(e);
+    return check_device_error(c);
+}
+
+MTP_API int mtp_step_bytes(mtp_ctx* c, int n, uint64_t* out_bytes) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (n < 1 || n > c->cfg.n_heads_max || !out_bytes) return fail(MTP_ERR_INVALID, "bad arguments");
+    const mtp_config& cf = c->cfg;
+    const uint64_t d = cf.d_model, F = cf.d_ffn, V = cf.codec_vocab, wb = c->wbytes;
+    uint64_t bytes = (uint64_t)cf.layers * ((3 * d * d + d * d + 2 * d * F) * wb + (3 * d + d + F + d + 4 * d) * 4);
+    bytes += (uint64_t)n * V * d * wb + (uint64_t)n * V * 4 + 2 * d * 4;
+    std::vector<int> len, npend, active, done;
+    MTP_TRY(read_slot_ints(c, c->d_len, len));
+    MTP_TRY(read_slot_ints(c, c->d_npend, npend));
+    MTP_TRY(read_slot_ints(c, c->d_active, active));
+    MTP_TRY(read_slot_ints(c, c->d_done, done));
+    for (int b = 0; b < cf.max_batch; ++b) {
+        if (!active[b] || done[b] || npend[b] == 0) continue;
+        // keys and values (bf16) read over the visible context, and written for the fed rows
+        bytes += (uint64_t)cf.layers * (uint64_t)(len[b] + npend[b]) * d * 2 * 2;
+        bytes += (uint64_t)cf.layers * (uint64_t)npend[b] * d * 2 * 2;
+    }
+    *out_bytes = bytes;
+    return MTP_OK;
+}
+
+MTP_API int mtp_viterbi(int batch, int n, int k, int vocab, int eos_id, const int32_t* cand_ids,
+                        const float* cand_logp, const float* log_q, const int32_t* remaining, int32_t* out_path,
+                        float* out_score, int32_t* out_accepted, int32_t* out_rollback, void* cuda_stream) {
+    g_err.clear();
+    if (batch < 0 || n < 1 || n > MAX_NHEADS || k < 1 || k > MAX_TOPK || vocab < 1 || k > vocab)
+        return fail(MTP_ERR_INVALID, "viterbi: batch %d, n %d (1..%d), k %d (1..%d), vocab %d", batch, n,
+                    MAX_NHEADS, k, MAX_TOPK, vocab);
+    if (batch > 0 && (!cand_ids || !cand_logp || !log_q || !out_path || !out_accepted))
+        return fail(MTP_ERR_INVALID, "viterbi: null pointer");
+    ViterbiArgs a;
+    a.batch = batch; a.n = n; a.k = k; a.vocab = vocab; a.eos_id = eos_id;
+    a.cand_ids = cand_ids; a.cand_logp = cand_logp; a.log_q = log_q; a.remaining = remaining;
+    a.path = out_path; a.score = out_score; a.accepted = out_accepted; a.rollback = out_rollback;
+    CUDA_TRY(launch_viterbi(a, static_cast<cudaStream_t>(cuda_stream)));
+    return MTP_OK;
+}
+
+MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden_dtype, int n, int k,
+                           int32_t* out_ids, float* out_logp, float* out_logits, float* out_lse) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    MTP_TRY(check_nk(c, n, k));
+    if (batch < 0 || (batch > 0 && (!hidden || !out_ids || !out_logp)))
+        return fail(MTP_ERR_INVALID, "heads_topk: bad batch or null pointer");
+    if (hidden_dtype != MTP_F32 && hidden_dtype != MTP_BF16) return fail(MTP_ERR_INVALID, "hidden dtype");
+    const int d = c->cfg.d_model, V = c->cfg.codec_vocab;
+    cudaStream_t s = c->stream;
+    Prof* prof = nullptr;
+    for (int b0 = 0; b0 < batch; b0 += MAX_ROWS) {
+        const int m = std::min(MAX_ROWS, batch - b0);
+        const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
+        CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,
+                                     hidden_dtype == MTP_BF16, c->d_x, m, d, s));
+        float* logits = out_logits ? out_logits + (size_t)b0 * n * V : c->d_logits;
+        MTP_TRY(launch_heads(c, c->d_x, m, n, logits, s, false, prof));
+        SelectArgs sa = select_base(c, n, k);
+        sa.logits = logits;
+        sa.lse = out_lse ? out_lse + (size_t)b0 * n : c->d_lse;
+        sa.cand_ids = out_ids + (size_t)b0 * n * k;
+        sa.cand_logp = out_logp + (size_t)b0 * n * k;
+        CUDA_TRY(launch_select(sa, m, false, s, false));
+    }
+    return MTP_OK;
+}
+
+MTP_API size_t mtp_attention_workspace_bytes(const mtp_attention_args* a) {
+    if (!a || a->rows < 1 || a->rows_per_group < 1 || a->n_heads < 1 || a->page_size < 1) return 0;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) {
+        cudaGetLastError();
+        return 0;
+    }
+    const int groups = (a->rows + a->rows_per_group - 1) / a->rows_per_group;
+    const int S = attn_splits_for(groups, a->n_heads, a->page_size, a->max_keys, sms);
+    return align256(attn_workspace_floats(groups, a->n_heads, S, a->rows_per_group) * sizeof(float)) +
+           align256((size_t)groups * a->n_heads * sizeof(int));
+}
+
+MTP_API int mtp_attention(const mtp_attention_args* a, void* workspace, size_t workspace_bytes, void* cuda_stream) {
+    g_err.clear();
+    if (!a || a->rows < 1 || a->rows_per_group < 1 || a->rows_per_group > MAX_ROWS || a->n_heads < 1 ||
+        (a->page_size != 16 && a->page_size != 32 && a->page_size != 64 && a->page_size != 128) || a->layers < 1 ||
+        a->layer < 0 || a->layer >= a->layers || a->bt_stride < 1 || a->max_keys < 1)
+        return fail(MTP_ERR_INVALID, "attention: invalid sizes");
+    if (!a->q || !a->kv_pool || !a->block_table || !a->row_seq || !a->row_pos || !a->out || !workspace)
+        return fail(MTP_ERR_INVALID, "attention: null pointer");
+    const size_t need = mtp_attention_workspace_bytes(a);
+    if (need == 0 || workspace_bytes < need)
+        return fail(MTP_ERR_INVALID, "attention: workspace %zu bytes, need %zu", workspace_bytes, need);
+    int dev = 0, sms = 0;
+    CUDA_TRY(cudaGetDevice(&dev));
+    CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int groups = (a->rows + a->rows_per_group - 1) / a->rows_per_group;
+    const int S = attn_splits_for(groups, a->n_heads, a->page_size, a->max_keys, sms);
+    AttnArgs at;
+    std::memset(&at, 0, sizeof(at));
+    const int d = a->n_heads * HEAD_DIM;
+    at.q = a->q; at.ldq = d;
+    at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(a->kv_pool);
+    at.page_elems = (long long)a->layers * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.layer_off = (long long)a->layer * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.block_table = a->block_table; at.bt_stride = a->bt_stride;
+    at.row_seq = a->row_seq; at.row_pos = a->row_pos;
+    at.out = a->out; at.ldo = d;
+    at.ws_part = static_cast<float*>(workspace);
+    at.ws_count = reinterpret_cast<int*>(static_cast<char*>(workspace) +
+                                         align256(attn_workspace_floats(groups, a->n_heads, S, a->rows_per_group) *
+                                                  sizeof(float)));
+    at.rows_per_group = a->rows_per_group; at.n_heads = a->n_heads; at.page_size = a->page_size;
+    at.n_splits = S; at.plan = PLAN_ROWS;
+    at.err = nullptr;
+    CUDA_TRY(launch_attention(at, groups, static_cast<cudaStream_t>(cuda_stream), false));
+    return MTP_OK;
+}
+
+}  // extern "C"

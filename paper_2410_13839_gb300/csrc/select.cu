@@ -1,0 +1,250 @@
+// select.cu -- log-softmax + top-k of each head, Viterbi over the candidate
+// lattice, and acceptance (Sec. III-B, III-C).
+//
+// Top-k (one warp per head): each lane holds 33 of the V <= 1056 logits;
+// lse = m + log(sum exp(l - m)) with a fixed reduction order; the ranking
+// score is logp = l - lse rounded to fp32; k rounds of a warp arg-max with
+// the key (score descending, id ascending) pick the candidates.
+//
+// Viterbi (one warp per sequence, lane j = candidate j, k <= 32): max-plus
+// recursion over the n positions,
+//   delta_t(j) = (max_i delta_{t-1}(i) + log_q[c_{t-1,i}][c_{t,j}]) + s_t(j),
+// every add a single fp32 add (no contraction), the lowest i on ties, the
+// backpointers in registers; the final state is the lowest j of the max.
+// Acceptance (ACCEPT_ALL): the path is cut after its first EOS and at the
+// remaining budget; the slot's state (cached length, fed tokens, output
+// buffer, done flag) is updated on the device, so steps need no host sync.
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace mtp {
+namespace {
+
+constexpr int VPL = MAX_VOCAB / 32;  // logits per lane
+
+// (value desc, index asc) arg-max across the warp; every lane returns the winner.
+__device__ __forceinline__ void warp_argmax(float& v, int& i) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(FULL_MASK, v, o);
+        const int oi = __shfl_xor_sync(FULL_MASK, i, o);
+        if (ov > v || (ov == v && oi < i)) {
+            v = ov;
+            i = oi;
+        }
+    }
+}
+
+// One head: lse and the top-k (ids, scores) of a logit row.  Lanes 0..k-1 of
+// out_ids/out_lp receive candidates 0..k-1 (written by lane 0).
+__device__ void head_topk_warp(const float* row, int V, int k, int* out_ids, float* out_lp, float* out_lse) {
+    const int lane = threadIdx.x & 31;
+    float v[VPL];
+    float m = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < VPL; ++c) {
+        const int idx = lane + 32 * c;
+        v[c] = idx < V ? row[idx] : -INFINITY;
+        m = fmaxf(m, v[c]);
+    }
+    m = warp_max(m);
+    float sum = 0.f;
+#pragma unroll
+    for (int c = 0; c < VPL; ++c)
+        if (lane + 32 * c < V) sum += expf(v[c] - m);
+    sum = warp_sum(sum);
+    const float lse = m + logf(sum);
+#pragma unroll
+    for (int c = 0; c < VPL; ++c) v[c] = __fsub_rn(v[c], lse);  // -inf stays -inf
+    uint64_t taken = 0;
+    for (int r = 0; r < k; ++r) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+#pragma unroll
+        for (int c = 0; c < VPL; ++c) {
+            const int idx = lane + 32 * c;
+            if (idx < V && !((taken >> c) & 1ull) && (v[c] > bv || bi == 0x7fffffff)) {
+                bv = v[c];
+                bi = idx;
+            }
+        }
+        warp_argmax(bv, bi);
+        if ((bi & 31) == lane) taken |= 1ull << (bi >> 5);
+        if (lane == 0) {
+            out_ids[r] = bi;
+            out_lp[r] = bv;
+        }
+    }
+    if (lane == 0 && out_lse) *out_lse = lse;
+}
+
+// Viterbi over ids/lp [n][k] (shared memory); lane 0 receives the results.
+__device__ void viterbi_warp(const int* ids, const float* lp, int n, int k, const float* log_q, int V,
+                             int* path, float* score) {
+    const int lane = threadIdx.x & 31;
+    const bool on = lane < k;
+    float delta = on ? lp[lane] : -INFINITY;
+    int bp[MAX_NHEADS];
+#pragma unroll
+    for (int t = 1; t < MAX_NHEADS; ++t) {
+        bp[t] = 0;
+        if (t < n) {
+            const int cj = on ? ids[t * k + lane] : 0;
+            const bool cj_ok = cj >= 0 && cj < V;
+            const int* prev = ids + (t - 1) * k;
+            float best = 0.f;
+            int arg = 0;
+            for (int i = 0; i < k; ++i) {
+                const float di = __shfl_sync(FULL_MASK, delta, i);
+                const int ci = prev[i];
+                // ids outside [0, V) have no transition: -inf (never read out of range)
+                const float lq = (cj_ok && ci >= 0 && ci < V) ? __ldg(log_q + (size_t)ci * V + cj) : -INFINITY;
+                const float val = __fadd_rn(di, lq);
+                if (i == 0 || val > best) {
+                    best = val;
+                    arg = i;
+                }
+            }
+            delta = on ? __fadd_rn(best, lp[t * k + lane]) : -INFINITY;
+            bp[t] = arg;
+        }
+    }
+    float bv = delta;
+    int bj = on ? lane : 0x7fffffff;
+    warp_argmax(bv, bj);
+    int state = bj;
+    int st[MAX_NHEADS];
+#pragma unroll
+    for (int t = MAX_NHEADS - 1; t >= 0; --t) {
+        st[t] = 0;
+        if (t < n) {
+            st[t] = state;
+            if (t > 0) state = __shfl_sync(FULL_MASK, bp[t], state);
+        }
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int t = 0; t < MAX_NHEADS; ++t)
+            if (t < n) path[t] = ids[t * k + st[t]];
+        *score = bv;
+    }
+}
+
+// ACCEPT_ALL: cut after the first EOS and at the budget.
+__device__ __forceinline__ void accept_all(const int* path, int n, int eos, int remaining, int& a, int& done) {
+    a = n;
+    bool eos_in = false;
+    for (int t = 0; t < n; ++t)
+        if (path[t] == eos) {
+            a = t + 1;
+            eos_in = true;
+            break;
+        }
+    a = min(a, max(remaining, 0));
+    done = (eos_in && a >= 1 && path[a - 1] == eos) || remaining - a <= 0;
+}
+
+__global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_accept) {
+    __shared__ int s_ids[MAX_NHEADS * MAX_TOPK];
+    __shared__ float s_lp[MAX_NHEADS * MAX_TOPK];
+    __shared__ int s_path[MAX_NHEADS];
+    __shared__ float s_score;
+    const int bl = blockIdx.x, b = a.seq_base + bl;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n = a.n, k = a.k;
+    pdl_launch_dependents();
+    pdl_wait();
+    if (do_accept && (!a.active[b] || a.done[b])) {
+        if (threadIdx.x < a.n_max) a.out_tokens[(size_t)b * a.n_max + threadIdx.x] = -1;
+        if (threadIdx.x == 0) a.out_accepted[b] = 0;
+        return;
+    }
+    if (warp < n) {
+        const size_t row = (size_t)bl * n + warp;
+        head_topk_warp(a.logits + row * a.V, a.V, k, s_ids + warp * k, s_lp + warp * k, a.lse + row);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < n * k; i += blockDim.x) {
+        a.cand_ids[(size_t)bl * n * k + i] = s_ids[i];
+        a.cand_logp[(size_t)bl * n * k + i] = s_lp[i];
+    }
+    if (!do_accept) return;
+    if (warp == 0) viterbi_warp(s_ids, s_lp, n, k, a.log_q, a.V, s_path, &s_score);
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+
+    int acc, done;
+    const int rem = a.remaining[b];
+    accept_all(s_path, n, a.eos_id, rem, acc, done);
+    a.seq_len[b] += a.n_pending[b];  // the tokens fed this step are now cached
+    const int gc = a.gen_count[b];
+    if (gc + acc > a.gen_stride) {
+        atomicOr(a.err, ERR_BOUNDS);
+        acc = max(0, a.gen_stride - gc);
+    }
+    for (int t = 0; t < a.n_max; ++t) a.out_tokens[(size_t)b * a.n_max + t] = t < acc ? s_path[t] : -1;
+    for (int t = 0; t < n; ++t) a.path[(size_t)b * n + t] = s_path[t];
+    for (int t = 0; t < acc; ++t) {
+        a.pending[(size_t)b * a.n_max + t] = s_path[t];
+        a.gen_tokens[(size_t)b * a.gen_stride + gc + t] = s_path[t];
+    }
+    a.gen_count[b] = gc + acc;
+    a.remaining[b] = rem - acc;
+    a.n_pending[b] = done ? 0 : acc;
+    a.done[b] = done;
+    a.out_accepted[b] = acc;
+}
+
+__global__ void __launch_bounds__(128) viterbi_kernel(const ViterbiArgs a) {
+    __shared__ int s_ids[4][MAX_NHEADS * MAX_TOPK];
+    __shared__ float s_lp[4][MAX_NHEADS * MAX_TOPK];
+    __shared__ int s_path[4][MAX_NHEADS];
+    __shared__ float s_score[4];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.x * 4 + warp;
+    if (b >= a.batch) return;  // whole warp leaves together
+    const int nk = a.n * a.k;
+    for (int i = lane; i < nk; i += 32) {
+        s_ids[warp][i] = a.cand_ids[(size_t)b * nk + i];
+        s_lp[warp][i] = a.cand_logp[(size_t)b * nk + i];
+    }
+    __syncwarp();
+    viterbi_warp(s_ids[warp], s_lp[warp], a.n, a.k, a.log_q, a.vocab, s_path[warp], &s_score[warp]);
+    __syncwarp();
+    if (lane != 0) return;
+    int acc, done;
+    const int rem = a.remaining ? a.remaining[b] : a.n;
+    accept_all(s_path[warp], a.n, a.eos_id, rem, acc, done);
+    for (int t = 0; t < a.n; ++t) a.path[(size_t)b * a.n + t] = s_path[warp][t];
+    if (a.score) a.score[b] = s_score[warp];
+    a.accepted[b] = acc;
+    if (a.rollback) a.rollback[b] = 0;
+}
+
+}  // namespace
+
+cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl) {
+    if (a.n < 1 || a.n > MAX_NHEADS || a.k < 1 || a.k > MAX_TOPK || a.V > MAX_VOCAB || a.k > a.V)
+        return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(batch);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, select_kernel, a, do_accept ? 1 : 0);
+}
+
+cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s) {
+    if (a.n < 1 || a.n > MAX_NHEADS || a.k < 1 || a.k > MAX_TOPK || a.batch < 0) return cudaErrorInvalidValue;
+    if (a.batch == 0) return cudaSuccess;
+    viterbi_kernel<<<(a.batch + 3) / 4, 128, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace mtp
