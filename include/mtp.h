@@ -193,6 +193,14 @@ typedef enum mtp_kernel_kind {
 MTP_API int mtp_profile_step(mtp_ctx* ctx, int n_heads, int top_k, float* out_ms,
                              int32_t* out_launches);
 
+/* Run one decode step (graph and PDL as the options say) with a timeline
+ * record per kernel launch: out int64 [cap][4] rows of {mtp_kernel_kind,
+ * earliest CTA start, latest CTA past its dependency wait, latest CTA end},
+ * times in ns of the GPU's global timer.  Returns the number of launches
+ * recorded (<= cap).  The step's effect on the slots is that of
+ * mtp_decode_step. */
+MTP_API int mtp_trace_step(mtp_ctx* ctx, int n_heads, int top_k, int64_t* out, int cap);
+
 /* Algorithmic bytes of one decode step: weights read (all blocks and the
  * first n_heads heads) plus keys/values read and written for every active
  * slot, from the current slot state (host uint64 out). */

@@ -66,6 +66,7 @@ def _load() -> ctypes.CDLL:
         "mtp_set_option": (i32, [vp, i32, i32]),
         "mtp_profile_step": (i32, [vp, i32, i32, vp, vp]),
         "mtp_step_bytes": (i32, [vp, i32, vp]),
+        "mtp_trace_step": (i32, [vp, i32, i32, vp, i32]),
         "mtp_viterbi": (i32, [i32, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
         "mtp_heads_topk": (i32, [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]),
         "mtp_attention_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),

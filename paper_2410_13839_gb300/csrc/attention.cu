@@ -24,6 +24,7 @@ constexpr int ATT_THREADS = 256;
 constexpr int ATT_KEYS = 256;    // keys staged per batch: 32 KB of keys + 32 KB of values
 constexpr int RPG = MAX_ROWS;    // rows per group, upper bound
 constexpr int PART = 2 + HEAD_DIM;  // (max, sum, out[64]) per row and split
+constexpr int MAX_SPLITS = 32;     // one warp lane per split in the merge
 static_assert(HEAD_DIM == 64, "score scale 0.125 assumes 64-wide heads");
 
 __device__ __forceinline__ void load_page_block(__nv_bfloat16* dst, const __nv_bfloat16* src, int elems) {
@@ -32,14 +33,16 @@ __device__ __forceinline__ void load_page_block(__nv_bfloat16* dst, const __nv_b
     for (int i = threadIdx.x; i < elems / 8; i += ATT_THREADS) d[i] = s[i];
 }
 
-__global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     __shared__ int s_pos[RPG];
     __shared__ int s_act[RPG];
+    __shared__ int s_rseq[RPG];
     __shared__ int s_seq, s_ktot, s_pre, s_last;
 
     const int sp = blockIdx.x, h = blockIdx.y, g = blockIdx.z;
+    TraceEnd trace_guard(a.trace);
     const int H = a.n_heads, P = a.page_size, S = a.n_splits;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem);
@@ -92,21 +95,24 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const AttnArgs a) {
 
     pdl_launch_dependents();
     pdl_wait();
+    trace_wait(a.trace);
 
     // ---- rows of this group (written by this step's embedding) ----
     const int rpg = a.rows_per_group;
     if (tid < RPG) {
         const int r = g * rpg + tid;
-        const bool act = tid < rpg && a.row_seq[r] >= 0;
-        s_act[tid] = act;
-        s_pos[tid] = act ? a.row_pos[r] : -1;
+        const int rs = tid < rpg ? a.row_seq[r] : -1;
+        const int rp = tid < rpg ? a.row_pos[r] : -1;
+        s_act[tid] = rs >= 0;
+        s_rseq[tid] = rs;
+        s_pos[tid] = rs >= 0 ? rp : -1;
     }
     __syncthreads();
     if (tid == 0) {
         int seq = -1, kmax = 0;
         for (int j = 0; j < RPG; ++j)
             if (s_act[j]) {
-                seq = a.row_seq[g * rpg + j];
+                seq = s_rseq[j];
                 kmax = max(kmax, s_pos[j] + 1);
             }
         s_seq = seq;
@@ -208,12 +214,25 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const AttnArgs a) {
                 m_run = m_new;
                 __syncwarp();
                 const int kend = min(nk, pos_j - bp * P + 1);  // keys past the row's position weigh 0
-                for (int t = 0; t < kend; ++t) {
+                float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+                int t = 0;
+                for (; t + 4 <= kend; t += 4) {  // four independent chains
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float p = pr[t + u];
+                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + (t + u) * HEAD_DIM + 2 * lane);
+                        a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
+                        a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
+                    }
+                }
+                for (; t < kend; ++t) {
                     const float p = pr[t];
                     const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + t * HEAD_DIM + 2 * lane);
-                    acc0 = fmaf(p, bf16_lo(v2), acc0);
-                    acc1 = fmaf(p, bf16_hi(v2), acc1);
+                    a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
+                    a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
                 }
+                acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
+                acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
             }
         }
         __syncthreads();
@@ -246,21 +265,33 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const AttnArgs a) {
     __threadfence();
 
     if (row_on) {
+        // lane s holds split s's (max, sum); every split's output pair is
+        // loaded before any is used, so the merge costs one L2 round trip
         const float* base = a.ws_part + ((size_t)(g * H + h) * S * RPG) * PART + row_j * PART;
-        float M = -INFINITY;
-        for (int s = 0; s < S; ++s) M = fmaxf(M, __ldcg(base + (size_t)s * RPG * PART));
-        float L = 0.f, o0 = 0.f, o1 = 0.f;
-        for (int s = 0; s < S; ++s) {
-            const float* pj = base + (size_t)s * RPG * PART;
-            const float ms = __ldcg(pj);
-            if (ms == -INFINITY) continue;
-            const float w = expf(ms - M);
-            L = fmaf(w, __ldcg(pj + 1), L);
-            o0 = fmaf(w, __ldcg(pj + 2 + 2 * lane), o0);
-            o1 = fmaf(w, __ldcg(pj + 3 + 2 * lane), o1);
+        const size_t sstride = (size_t)RPG * PART;
+        float ms = -INFINITY, ls = 0.f;
+        if (lane < S) {
+            ms = __ldcg(base + lane * sstride);
+            ls = __ldcg(base + lane * sstride + 1);
         }
-        out_row[0] = o0 / L;
-        out_row[1] = o1 / L;
+        float o0[MAX_SPLITS], o1[MAX_SPLITS];
+#pragma unroll
+        for (int s = 0; s < MAX_SPLITS; ++s) {
+            o0[s] = s < S ? __ldcg(base + s * sstride + 2 + 2 * lane) : 0.f;
+            o1[s] = s < S ? __ldcg(base + s * sstride + 3 + 2 * lane) : 0.f;
+        }
+        const float M = warp_max(ms);
+        const float w = (ms == -INFINITY) ? 0.f : expf(ms - M);
+        const float L = warp_sum(w * ls);
+        float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+        for (int s = 0; s < MAX_SPLITS; ++s) {
+            const float ws = __shfl_sync(FULL_MASK, w, s);
+            r0 = fmaf(ws, o0[s], r0);
+            r1 = fmaf(ws, o1[s], r1);
+        }
+        out_row[0] = r0 / L;
+        out_row[1] = r1 / L;
     }
     if (tid == 0) a.ws_count[g * H + h] = 0;
 }
@@ -278,7 +309,7 @@ size_t attn_smem_bytes(int /*page_size*/) {
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms) {
     const int max_pages = (max_keys + page_size - 1) / page_size;
     int s = num_sms / max(1, groups * n_heads);
-    s = max(1, min(s, max_pages));
+    s = max(1, min(min(s, max_pages), MAX_SPLITS));
     return s;
 }
 

@@ -108,6 +108,29 @@ __device__ __forceinline__ void load4(const float* p, float (&w)[4]) {
     w[0] = u.x; w[1] = u.y; w[2] = u.z; w[3] = u.w;
 }
 
+// ---- launch timeline (tracing option) --------------------------------------
+// A traced launch owns 3 u64 words: earliest CTA start, latest CTA past the
+// dependency wait, latest CTA end, all from %globaltimer (ns).
+
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void trace_start(unsigned long long* tr) {
+    if (tr && threadIdx.x == 0) atomicMin(tr, globaltimer());
+}
+__device__ __forceinline__ void trace_wait(unsigned long long* tr) {
+    if (tr && threadIdx.x == 0) atomicMax(tr + 1, globaltimer());
+}
+struct TraceEnd {
+    unsigned long long* tr;
+    __device__ explicit TraceEnd(unsigned long long* t) : tr(t) { trace_start(t); }
+    __device__ ~TraceEnd() {
+        if (tr && threadIdx.x == 0) atomicMax(tr + 2, globaltimer());
+    }
+};
+
 // Exact GELU, x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2)), with CUDA's erff.
 __device__ __forceinline__ float gelu_erf(float x) { return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f)); }
 

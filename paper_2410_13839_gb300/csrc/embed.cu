@@ -10,8 +10,10 @@ namespace {
 __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
     __shared__ int s_tok, s_pos, s_act, s_phone;
     const int r = blockIdx.x, tid = threadIdx.x;
+    TraceEnd trace_guard(a.trace);
     pdl_launch_dependents();
     pdl_wait();
+    trace_wait(a.trace);
     if (tid == 0) {
         int seq = -1, pos = 0, tok = 0, phone = 0, last = 0;
         if (a.mode == 0) {  // decode: row r is fed token j of slot seq_base + r / n
@@ -117,6 +119,19 @@ cudaError_t launch_pe_table(float* pe, int max_ctx, int d, cudaStream_t s) {
 cudaError_t launch_convert_rows(const void* src, int src_bf16, float* dst, int rows, int d, cudaStream_t s) {
     const long long n = (long long)rows * d;
     convert_rows_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(src, src_bf16, dst, n);
+    return cudaGetLastError();
+}
+
+__global__ void trace_reset_kernel(unsigned long long* tr, int records) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= records) return;
+    tr[3 * i] = ~0ull;
+    tr[3 * i + 1] = 0;
+    tr[3 * i + 2] = 0;
+}
+
+cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s) {
+    trace_reset_kernel<<<(records + 255) / 256, 256, 0, s>>>(trace, records);
     return cudaGetLastError();
 }
 

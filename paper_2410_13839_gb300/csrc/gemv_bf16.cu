@@ -7,10 +7,11 @@ cudaError_t launch_gemv_f32(const GemvArgs& a, int epi, int grid, size_t smem, c
 
 size_t gemv_smem_bytes(int rows_per_cta, int K, int wbytes, int M) {
     const int mt = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : 8;
-    const int warps = K <= 1024 ? 8 : 16;
+    const int warps = 8;
     const int groups = (rows_per_cta + 32 / mt - 1) / (32 / mt);
     const size_t wpad = ((size_t)rows_per_cta * K * wbytes + 127) & ~(size_t)127;
-    return wpad + (size_t)warps * groups * 32 * sizeof(float);
+    const size_t xs = K > 1024 ? (size_t)mt * K * sizeof(float) : 0;  // staged wide inputs
+    return wpad + (size_t)warps * groups * 32 * sizeof(float) + xs;
 }
 
 cudaError_t launch_gemv(const GemvArgs& a, int epi, bool ln, bool w_bf16, int grid, cudaStream_t s, bool pdl) {

@@ -41,12 +41,16 @@ __device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
 }
 
 template <typename WT, int MT, int WARPS, int NSUB, int EPI, bool LN>
-__global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
+__global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     __shared__ float ln_part[WARPS][MT];
     __shared__ float ln_stat[2][MT];
-    constexpr int G = 32 / MT;  // weight rows per reduce-scatter group
+    __shared__ int s_seq[MT], s_pos[MT], s_last[MT], s_page[MT];
+    constexpr int G = 32 / MT;           // weight rows per reduce-scatter group
+    constexpr int NT = WARPS * 32;
+    constexpr bool XSMEM = NSUB > 1;     // wide inputs are staged in shared memory
+    TraceEnd trace_guard(a.trace);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int r0 = blockIdx.x * a.rows_per_cta;
@@ -56,7 +60,8 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
     const size_t wpad = ((size_t)a.rows_per_cta * K * sizeof(WT) + 127) & ~(size_t)127;
     const WT* wsm = reinterpret_cast<const WT*>(smem);
     const int ngroups = (max(R, 0) + G - 1) / G;
-    float* red = reinterpret_cast<float*>(smem + wpad);  // [WARPS][ngroups * 32]
+    float* red = reinterpret_cast<float*>(smem + wpad);                   // [WARPS][ngroups * 32]
+    float* xs = red + (size_t)WARPS * ((a.rows_per_cta + G - 1) / G) * 32;  // [MT][K] when XSMEM
 
     if (tid == 0) {
         mbar_init(&bar, 1);
@@ -70,9 +75,10 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
             bulk_copy_g2s(smem + off, src + off, (uint32_t)min((size_t)BULK_CHUNK, wbytes - off), &bar);
     }
 
+    // ---- parameters (weights): read before the wait ----
     const int Kw = K / WARPS;  // columns of this warp
-    float gam[NSUB][4], bet[NSUB][4];
-    if (LN) {  // LayerNorm parameters are weights: read them before the wait
+    float gam[XSMEM ? 1 : NSUB][4], bet[XSMEM ? 1 : NSUB][4];
+    if (LN && !XSMEM) {
 #pragma unroll
         for (int s = 0; s < NSUB; ++s) {
             const int c = s * 32 + lane;
@@ -85,43 +91,92 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
             }
         }
     }
+    float bias_r[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+        const int o = tid + u * NT;
+        bias_r[u] = (o < R * MT) ? __ldg(a.bias + r0 + o / MT) : 0.f;
+    }
 
     pdl_launch_dependents();
     pdl_wait();
+    trace_wait(a.trace);
 
     // ---- inputs of this launch (written by the previous kernel) ----
-    float xv[MT][NSUB][4];
-#pragma unroll
-    for (int m = 0; m < MT; ++m)
-#pragma unroll
-        for (int s = 0; s < NSUB; ++s) {
-            const int c = s * 32 + lane;
-            if (m < a.M && c * 4 < Kw) {
-                load4(a.A + (size_t)m * a.lda + warp * Kw + c * 4, xv[m][s]);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) xv[m][s][i] = 0.f;
-            }
+    if (tid < MT) {
+        const bool in = tid < a.M;
+        s_seq[tid] = (in && a.row_seq) ? a.row_seq[tid] : (in ? 0 : -1);
+        if (EPI == EPI_QKV || EPI == EPI_RESID) {
+            s_pos[tid] = (in && a.row_pos) ? a.row_pos[tid] : -1;
+            s_last[tid] = (in && a.row_last) ? a.row_last[tid] : 0;
         }
+    }
+    float xv[MT][XSMEM ? 1 : NSUB][4];
+    if (!XSMEM) {
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+#pragma unroll
+            for (int s = 0; s < (XSMEM ? 1 : NSUB); ++s) {
+                const int c = s * 32 + lane;
+                if (m < a.M && c * 4 < Kw) {
+                    load4(a.A + (size_t)m * a.lda + warp * Kw + c * 4, xv[m][s]);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) xv[m][s][i] = 0.f;
+                }
+            }
+    } else {
+        for (int i = tid; i < MT * (K / 4); i += NT) {
+            const int m = i / (K / 4), c = i % (K / 4);
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (m < a.M) v = *reinterpret_cast<const float4*>(a.A + (size_t)m * a.lda + c * 4);
+            *reinterpret_cast<float4*>(xs + (size_t)m * K + c * 4) = v;
+        }
+    }
+    __syncthreads();
+    if (EPI == EPI_QKV && tid < MT) {  // page of each row's key/value slot; used in the epilogue
+        const int seq = s_seq[tid], pos = s_pos[tid];
+        s_page[tid] = (seq >= 0 && pos >= 0) ? a.block_table[(size_t)seq * a.bt_stride + pos / a.page_size] : -1;
+    }
 
     if (LN) {
-        // mean, then variance of (x - mean), each a block reduction in fixed order
+        // mean, then variance of (x - mean), each a reduction in fixed order
 #pragma unroll
         for (int pass = 0; pass < 2; ++pass) {
+            if (!XSMEM) {
 #pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                float part = 0.f;
+                for (int m = 0; m < MT; ++m) {
+                    float part = 0.f;
 #pragma unroll
-                for (int s = 0; s < NSUB; ++s) {
-                    const bool valid = (s * 32 + lane) * 4 < Kw;
+                    for (int s = 0; s < (XSMEM ? 1 : NSUB); ++s) {
+                        const bool valid = (s * 32 + lane) * 4 < Kw;
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float t = pass == 0 ? xv[m][s][i] : xv[m][s][i] - ln_stat[0][m];
-                        part += valid ? (pass == 0 ? t : t * t) : 0.f;
+                        for (int i = 0; i < 4; ++i) {
+                            const float t = pass == 0 ? xv[m][s][i] : xv[m][s][i] - ln_stat[0][m];
+                            part += valid ? (pass == 0 ? t : t * t) : 0.f;
+                        }
                     }
+                    part = warp_sum(part);
+                    if (lane == 0) ln_part[warp][m] = part;
                 }
-                part = warp_sum(part);
-                if (lane == 0) ln_part[warp][m] = part;
+            } else {
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+                    float part = 0.f;
+                    for (int e = 0; e < Kw; e += 128) {
+                        const int kk = warp * Kw + e + lane * 4;
+                        if (e + lane * 4 < Kw) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float t = pass == 0 ? xs[(size_t)m * K + kk + i]
+                                                          : xs[(size_t)m * K + kk + i] - ln_stat[0][m];
+                                part += pass == 0 ? t : t * t;
+                            }
+                        }
+                    }
+                    part = warp_sum(part);
+                    if (lane == 0) ln_part[warp][m] = part;
+                }
             }
             __syncthreads();
             if (tid < MT) {
@@ -133,13 +188,21 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
             }
             __syncthreads();
         }
+        if (!XSMEM) {
 #pragma unroll
-        for (int m = 0; m < MT; ++m)
+            for (int m = 0; m < MT; ++m)
 #pragma unroll
-            for (int s = 0; s < NSUB; ++s)
+                for (int s = 0; s < (XSMEM ? 1 : NSUB); ++s)
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    xv[m][s][i] = (xv[m][s][i] - ln_stat[0][m]) * ln_stat[1][m] * gam[s][i] + bet[s][i];
+                    for (int i = 0; i < 4; ++i)
+                        xv[m][s][i] = (xv[m][s][i] - ln_stat[0][m]) * ln_stat[1][m] * gam[s][i] + bet[s][i];
+        } else {
+            for (int i = tid; i < MT * K; i += NT) {
+                const int m = i / K, k = i % K;
+                xs[i] = (xs[i] - ln_stat[0][m]) * ln_stat[1][m] * a.ln_g[k] + a.ln_b[k];
+            }
+            __syncthreads();
+        }
     }
 
     if (wbytes == 0) return;
@@ -160,6 +223,17 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
             const int c = s * 32 + lane;
             if (c * 4 < Kw) {
                 const int k = warp * Kw + c * 4;
+                float xr[MT][4];
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+                    if (XSMEM) {
+                        const float4 v = *reinterpret_cast<const float4*>(xs + (size_t)m * K + k);
+                        xr[m][0] = v.x; xr[m][1] = v.y; xr[m][2] = v.z; xr[m][3] = v.w;
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) xr[m][i] = xv[m][XSMEM ? 0 : s][i];
+                    }
+                }
 #pragma unroll
                 for (int r = 0; r < G; ++r) {
                     const int row = g * G + r;
@@ -169,10 +243,10 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
 #pragma unroll
                         for (int m = 0; m < MT; ++m) {
                             float t = acc[r * MT + m];
-                            t = fmaf(w[0], xv[m][s][0], t);
-                            t = fmaf(w[1], xv[m][s][1], t);
-                            t = fmaf(w[2], xv[m][s][2], t);
-                            t = fmaf(w[3], xv[m][s][3], t);
+                            t = fmaf(w[0], xr[m][0], t);
+                            t = fmaf(w[1], xr[m][1], t);
+                            t = fmaf(w[2], xr[m][2], t);
+                            t = fmaf(w[3], xr[m][3], t);
                             acc[r * MT + m] = t;
                         }
                     }
@@ -185,15 +259,15 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
     __syncthreads();
 
     // ---- epilogue: output o = row * MT + m ----
-    for (int o = tid; o < R * MT; o += WARPS * 32) {
+    for (int o = tid; o < R * MT; o += NT) {
         const int row = o / MT, m = o - row * MT;
         if (m >= a.M) continue;
         float y = 0.f;
 #pragma unroll
         for (int w = 0; w < WARPS; ++w) y += red[w * (ngroups * 32) + o];
         const int f = r0 + row;
-        y += a.bias[f];
-        const bool active = a.row_seq == nullptr || a.row_seq[m] >= 0;
+        y += o < NT ? bias_r[0] : o < 2 * NT ? bias_r[1] : __ldg(a.bias + f);
+        const bool active = s_seq[m] >= 0;
         if (EPI == EPI_QKV) {
             const int d = a.d_model;
             if (f < d) {
@@ -202,8 +276,7 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
                 const int sec = f / d;  // 1 = key, 2 = value
                 const int within = f - sec * d;
                 const int head = within / HEAD_DIM, dd = within % HEAD_DIM;
-                const int seq = a.row_seq[m], pos = a.row_pos[m];
-                const int page = a.block_table[(size_t)seq * a.bt_stride + pos / a.page_size];
+                const int pos = s_pos[m], page = s_page[m];
                 if (page < 0) {
                     atomicOr(a.err, ERR_BOUNDS);
                     continue;
@@ -217,8 +290,7 @@ __global__ void __launch_bounds__(WARPS * 32) gemv_kernel(const GemvArgs a) {
             if (active) {
                 const float x = a.out[(size_t)m * a.ldo + f] + y;
                 a.out[(size_t)m * a.ldo + f] = x;
-                if (a.h_last != nullptr && a.row_last[m])
-                    a.h_last[(size_t)a.row_seq[m] * a.ld_h + f] = x;
+                if (a.h_last != nullptr && s_last[m]) a.h_last[(size_t)s_seq[m] * a.ld_h + f] = x;
             }
         } else if (EPI == EPI_GELU) {
             a.out[(size_t)m * a.ldo + f] = gelu_erf(y);
@@ -264,7 +336,7 @@ cudaError_t dispatch_epi(const GemvArgs& a, int epi, int grid, size_t smem, cuda
 template <typename WT, int MT>
 cudaError_t dispatch_k(const GemvArgs& a, int epi, int grid, size_t smem, cudaStream_t s, bool pdl) {
     if (a.K <= 1024) return dispatch_epi<WT, MT, 8, 1>(a, epi, grid, smem, s, pdl);
-    return dispatch_epi<WT, MT, 16, 2>(a, epi, grid, smem, s, pdl);
+    return dispatch_epi<WT, MT, 8, 4>(a, epi, grid, smem, s, pdl);
 }
 
 template <typename WT>

@@ -43,6 +43,7 @@ struct GemvArgs {
     uint16_t* kv_pool; long long page_elems; long long layer_off; int n_heads, page_size, d_model;
     const int* block_table; int bt_stride;
     int* err;
+    unsigned long long* trace;           // timeline record of this launch (may be null)
 };
 
 size_t gemv_smem_bytes(int rows_per_cta, int K, int wbytes, int M);
@@ -67,6 +68,7 @@ struct AttnArgs {
     const int* seq_len; const int* seq_new; int seq_base;   // PLAN_DEVICE
     int val_seq, val_old, val_new;                           // PLAN_VALUE
     int* err;
+    unsigned long long* trace;
 };
 
 size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
@@ -89,6 +91,7 @@ struct EmbedArgs {
     // prefill
     int slot, p0, n_ph, total, prompt_stride; const int* prompt;
     int* err;
+    unsigned long long* trace;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_pe_table(float* pe, int max_ctx, int d, cudaStream_t s);
@@ -106,6 +109,7 @@ struct SelectArgs {
     int* gen_count; int* gen_tokens; int gen_stride;
     int* out_tokens; int* out_accepted;   // [B][n_max], [B]
     int* err;
+    unsigned long long* trace;
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
 
@@ -126,5 +130,6 @@ struct SlotSet {
     int set_len, set_pending, set_remaining, set_done, set_active, set_gen;
 };
 cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s);
+cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s);
 
 }  // namespace mtp

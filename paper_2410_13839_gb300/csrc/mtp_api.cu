@@ -17,6 +17,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <tuple>
 #include <string>
 #include <utility>
 #include <vector>
@@ -109,8 +110,14 @@ struct mtp_ctx {
     float* d_ws = nullptr;
     int* d_ws_count = nullptr;
     int* d_err = nullptr;
-    std::map<std::pair<int, int>, cudaGraphExec_t> graphs;
+    std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;  // (n_heads, top_k, traced)
+    std::map<std::tuple<int, int, int>, std::vector<int>> graph_kinds;
     int last_n = 0, last_k = 0;
+    // launch timeline (mtp_trace_step)
+    unsigned long long* d_trace = nullptr;
+    int trace_cap = 0;
+    bool tracing = false;
+    std::vector<int> trace_kinds;
 
     template <typename T>
     int alloc(T** p, size_t count) {
@@ -156,10 +163,17 @@ int gemv_grid(const mtp_ctx* c, int N, int K, int M, int* rpc) {
     int ctas = c->num_sms;
     for (;;) {
         *rpc = (N + ctas - 1) / ctas;
-        if (gemv_smem_bytes(*rpc, K, c->wbytes, M) <= 112 * 1024 || *rpc == 1) break;
+        if ((size_t)*rpc * K * c->wbytes <= 112 * 1024 || *rpc == 1) break;
         ctas *= 2;
     }
     return (N + *rpc - 1) / *rpc;
+}
+
+// Timeline record of the next launch (null unless a traced step is being enqueued).
+unsigned long long* tslot(mtp_ctx* c, int kind) {
+    if (!c->tracing || (int)c->trace_kinds.size() >= c->trace_cap) return nullptr;
+    c->trace_kinds.push_back(kind);
+    return c->d_trace + 3 * (c->trace_kinds.size() - 1);
 }
 
 GemvArgs gemv_base(mtp_ctx* c) {
@@ -193,6 +207,7 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
         q.kv_pool = c->d_kv; q.page_elems = c->page_elems; q.layer_off = layer_off;
         q.n_heads = H; q.page_size = P; q.d_model = d;
         q.block_table = c->d_block_table; q.bt_stride = c->pages_per_seq;
+        q.trace = tslot(c, MTP_K_QKV);
         LAUNCH(MTP_K_QKV, launch_gemv(q, EPI_QKV, true, bf, grid, s, pdl));
 
         AttnArgs at;
@@ -208,12 +223,14 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
         at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = seq_base;
         at.val_seq = val_seq; at.val_old = val_old; at.val_new = val_new;
         at.err = c->d_err;
+        at.trace = tslot(c, MTP_K_ATTN);
         LAUNCH(MTP_K_ATTN, launch_attention(at, G, s, pdl));
 
         GemvArgs o = gemv_base(c);
         o.A = c->d_attn; o.lda = d; o.W = L.wo; o.bias = L.bo; o.N = d; o.K = d; o.M = M;
         grid = gemv_grid(c, o.N, o.K, M, &rpc); o.rows_per_cta = rpc;
         o.out = c->d_x; o.ldo = d;
+        o.trace = tslot(c, MTP_K_OPROJ);
         LAUNCH(MTP_K_OPROJ, launch_gemv(o, EPI_RESID, false, bf, grid, s, pdl));
 
         GemvArgs f1 = gemv_base(c);
@@ -221,6 +238,7 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
         f1.W = L.w1; f1.bias = L.b1; f1.N = F; f1.K = d; f1.M = M;
         grid = gemv_grid(c, f1.N, f1.K, M, &rpc); f1.rows_per_cta = rpc;
         f1.out = c->d_u; f1.ldo = F;
+        f1.trace = tslot(c, MTP_K_FFN1);
         LAUNCH(MTP_K_FFN1, launch_gemv(f1, EPI_GELU, true, bf, grid, s, pdl));
 
         GemvArgs f2 = gemv_base(c);
@@ -231,6 +249,7 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
             f2.h_last = c->d_h_last;
             f2.ld_h = d;
         }
+        f2.trace = tslot(c, MTP_K_FFN2);
         LAUNCH(MTP_K_FFN2, launch_gemv(f2, EPI_RESID, false, bf, grid, s, pdl));
     }
     return MTP_OK;
@@ -262,6 +281,7 @@ int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, cudaSt
     h.rows_per_cta = rpc;
     h.row_seq = nullptr;
     h.out = logits; h.ldo = n * V;
+    h.trace = tslot(c, MTP_K_HEADS);
     LAUNCH(MTP_K_HEADS, launch_gemv(h, EPI_LOGITS, true, c->cfg.weight_dtype == MTP_BF16, grid, s, pdl));
     return MTP_OK;
 }
@@ -287,6 +307,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         const int G = std::min(spc, B - b0), M = G * n;
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
+        e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));  // full dependency on the previous pass
         MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, c->cfg.max_ctx, s, pdl, prof));
     }
@@ -295,6 +316,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, s, pdl, prof));
     }
     SelectArgs sa = select_base(c, n, k);
+    sa.trace = tslot(c, MTP_K_SELECT);
     LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
     return MTP_OK;
 }
@@ -302,12 +324,16 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
 int run_step(mtp_ctx* c, int n, int k) {
     c->last_n = n;
     c->last_k = k;
-    if (!c->use_graphs) return enqueue_step(c, n, k, c->stream, c->use_pdl, nullptr);
-    auto key = std::make_pair(n, k);
+    if (!c->use_graphs) {
+        c->trace_kinds.clear();
+        return enqueue_step(c, n, k, c->stream, c->use_pdl, nullptr);
+    }
+    const auto key = std::make_tuple(n, k, c->tracing ? 1 : 0);
     auto it = c->graphs.find(key);
     if (it == c->graphs.end()) {
         cudaGraph_t graph = nullptr;
         cudaGraphExec_t exec = nullptr;
+        c->trace_kinds.clear();
         CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
         const int r = enqueue_step(c, n, k, c->cap_stream, c->use_pdl, nullptr);
         const cudaError_t ec = cudaStreamEndCapture(c->cap_stream, &graph);
@@ -320,7 +346,9 @@ int run_step(mtp_ctx* c, int n, int k) {
         cudaGraphDestroy(graph);
         CUDA_TRY(ei);
         it = c->graphs.emplace(key, exec).first;
+        c->graph_kinds[key] = c->trace_kinds;
     }
+    c->trace_kinds = c->graph_kinds[key];
     CUDA_TRY(cudaGraphLaunch(it->second, c->stream));
     return MTP_OK;
 }
@@ -538,11 +566,12 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
     c->n_pages = cf.n_pages > 0 ? cf.n_pages : B * c->pages_per_seq;
     c->page_elems = (long long)cf.layers * 2 * H * P * HEAD_DIM;
     // projection slices must fit shared memory
-    for (int K : {d, F}) {
+    const int proj[5][2] = {{3 * d, d}, {d, d}, {F, d}, {d, F}, {nm * V, d}};
+    for (const auto& pk : proj) {
         int rpc;
-        gemv_grid(c, 3 * d, K, MAX_ROWS, &rpc);
-        if (gemv_smem_bytes(rpc, K, c->wbytes, MAX_ROWS) > 200 * 1024)
-            return bail(fail(MTP_ERR_INVALID, "weight rows of width %d do not fit shared memory", K));
+        gemv_grid(c, pk[0], pk[1], MAX_ROWS, &rpc);
+        if (gemv_smem_bytes(rpc, pk[1], c->wbytes, MAX_ROWS) > 200 * 1024)
+            return bail(fail(MTP_ERR_INVALID, "projection %d x %d does not fit shared memory", pk[0], pk[1]));
     }
     const int S_max = std::max(1, c->num_sms / H) + 1;
     const size_t ws_floats = attn_workspace_floats(MAX_ROWS, H, S_max, MAX_ROWS);
@@ -796,6 +825,32 @@ MTP_API int mtp_profile_step(mtp_ctx* c, int n, int k, float* out_ms, int32_t* o
     if (r != MTP_OK) return r;
     CUDA_TRY(e);
     return check_device_error(c);
+}
+
+MTP_API int mtp_trace_step(mtp_ctx* c, int n, int k, int64_t* out, int cap) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    MTP_TRY(check_nk(c, n, k));
+    if (!out || cap < 1) return fail(MTP_ERR_INVALID, "trace: null output or capacity < 1");
+    if (!c->d_trace) {
+        c->trace_cap = 4096;
+        MTP_TRY(c->alloc(&c->d_trace, (size_t)3 * c->trace_cap));
+    }
+    CUDA_TRY(launch_trace_reset(c->d_trace, c->trace_cap, c->stream));
+    c->tracing = true;
+    const int r = run_step(c, n, k);
+    c->tracing = false;
+    MTP_TRY(r);
+    std::vector<unsigned long long> h(3 * (size_t)c->trace_cap);
+    CUDA_TRY(cudaMemcpyAsync(h.data(), c->d_trace, h.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost,
+                             c->stream));
+    MTP_TRY(check_device_error(c));
+    const int count = std::min<int>((int)c->trace_kinds.size(), cap);
+    for (int i = 0; i < count; ++i) {
+        out[4 * i] = c->trace_kinds[i];
+        for (int j = 0; j < 3; ++j) out[4 * i + 1 + j] = (int64_t)h[3 * i + j];
+    }
+    return count;
 }
 
 MTP_API int mtp_step_bytes(mtp_ctx* c, int n, uint64_t* out_bytes) {

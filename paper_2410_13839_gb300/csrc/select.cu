@@ -80,9 +80,24 @@ __device__ void head_topk_warp(const float* row, int V, int k, int* out_ids, flo
     if (lane == 0 && out_lse) *out_lse = lse;
 }
 
-// Viterbi over ids/lp [n][k] (shared memory); lane 0 receives the results.
-__device__ void viterbi_warp(const int* ids, const float* lp, int n, int k, const float* log_q, int V,
-                             int* path, float* score) {
+// Gather the transition scores the lattice uses, lq[t-1][i][j] = log_q[c_{t-1,i}][c_{t,j}]
+// for t = 1..n-1, into shared memory with all threads of the group at once
+// (one memory latency instead of one per recursion step).  Ids outside
+// [0, V) get -inf (never read out of range).
+__device__ __forceinline__ void gather_transitions(const int* ids, int n, int k, const float* log_q, int V,
+                                                   float* lq, int tid, int nthreads) {
+    const int kk = k * k;
+    for (int e = tid; e < (n - 1) * kk; e += nthreads) {
+        const int t = e / kk + 1, i = (e % kk) / k, j = e % k;
+        const int ci = ids[(t - 1) * k + i], cj = ids[t * k + j];
+        lq[e] = (ci >= 0 && ci < V && cj >= 0 && cj < V) ? __ldg(log_q + (size_t)ci * V + cj) : -INFINITY;
+    }
+}
+
+// Viterbi over ids/lp [n][k] with transitions lq [n-1][k][k] (all shared
+// memory); lane 0 receives the results.
+__device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, int n, int k, int* path,
+                             float* score) {
     const int lane = threadIdx.x & 31;
     const bool on = lane < k;
     float delta = on ? lp[lane] : -INFINITY;
@@ -91,17 +106,12 @@ __device__ void viterbi_warp(const int* ids, const float* lp, int n, int k, cons
     for (int t = 1; t < MAX_NHEADS; ++t) {
         bp[t] = 0;
         if (t < n) {
-            const int cj = on ? ids[t * k + lane] : 0;
-            const bool cj_ok = cj >= 0 && cj < V;
-            const int* prev = ids + (t - 1) * k;
+            const float* lqt = lq + (size_t)(t - 1) * k * k + (on ? lane : 0);
             float best = 0.f;
             int arg = 0;
             for (int i = 0; i < k; ++i) {
                 const float di = __shfl_sync(FULL_MASK, delta, i);
-                const int ci = prev[i];
-                // ids outside [0, V) have no transition: -inf (never read out of range)
-                const float lq = (cj_ok && ci >= 0 && ci < V) ? __ldg(log_q + (size_t)ci * V + cj) : -INFINITY;
-                const float val = __fadd_rn(di, lq);
+                const float val = __fadd_rn(di, lqt[i * k]);
                 if (i == 0 || val > best) {
                     best = val;
                     arg = i;
@@ -149,13 +159,16 @@ __device__ __forceinline__ void accept_all(const int* path, int n, int eos, int 
 __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_accept) {
     __shared__ int s_ids[MAX_NHEADS * MAX_TOPK];
     __shared__ float s_lp[MAX_NHEADS * MAX_TOPK];
+    __shared__ float s_lq[(MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK];
     __shared__ int s_path[MAX_NHEADS];
     __shared__ float s_score;
     const int bl = blockIdx.x, b = a.seq_base + bl;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
     const int n = a.n, k = a.k;
+    TraceEnd trace_guard(a.trace);
     pdl_launch_dependents();
     pdl_wait();
+    trace_wait(a.trace);
     if (do_accept && (!a.active[b] || a.done[b])) {
         if (threadIdx.x < a.n_max) a.out_tokens[(size_t)b * a.n_max + threadIdx.x] = -1;
         if (threadIdx.x == 0) a.out_accepted[b] = 0;
@@ -171,7 +184,9 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         a.cand_logp[(size_t)bl * n * k + i] = s_lp[i];
     }
     if (!do_accept) return;
-    if (warp == 0) viterbi_warp(s_ids, s_lp, n, k, a.log_q, a.V, s_path, &s_score);
+    gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
+    __syncthreads();
+    if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_path, &s_score);
     __syncthreads();
     if (threadIdx.x != 0) return;
 
@@ -197,13 +212,18 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     a.out_accepted[b] = acc;
 }
 
-__global__ void __launch_bounds__(128) viterbi_kernel(const ViterbiArgs a) {
-    __shared__ int s_ids[4][MAX_NHEADS * MAX_TOPK];
-    __shared__ float s_lp[4][MAX_NHEADS * MAX_TOPK];
-    __shared__ int s_path[4][MAX_NHEADS];
-    __shared__ float s_score[4];
+// Stand-alone Viterbi: one warp per lattice, VIT_WARPS lattices per block;
+// dynamic shared memory holds each warp's transition table.
+constexpr int VIT_WARPS = 4;
+
+__global__ void __launch_bounds__(VIT_WARPS * 32) viterbi_kernel(const ViterbiArgs a) {
+    extern __shared__ float vit_lq[];
+    __shared__ int s_ids[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
+    __shared__ float s_lp[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
+    __shared__ int s_path[VIT_WARPS][MAX_NHEADS];
+    __shared__ float s_score[VIT_WARPS];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.x * 4 + warp;
+    const int b = blockIdx.x * VIT_WARPS + warp;
     if (b >= a.batch) return;  // whole warp leaves together
     const int nk = a.n * a.k;
     for (int i = lane; i < nk; i += 32) {
@@ -211,7 +231,10 @@ __global__ void __launch_bounds__(128) viterbi_kernel(const ViterbiArgs a) {
         s_lp[warp][i] = a.cand_logp[(size_t)b * nk + i];
     }
     __syncwarp();
-    viterbi_warp(s_ids[warp], s_lp[warp], a.n, a.k, a.log_q, a.vocab, s_path[warp], &s_score[warp]);
+    float* lq = vit_lq + (size_t)warp * (a.n - 1) * a.k * a.k;
+    gather_transitions(s_ids[warp], a.n, a.k, a.log_q, a.vocab, lq, lane, 32);
+    __syncwarp();
+    viterbi_warp(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_path[warp], &s_score[warp]);
     __syncwarp();
     if (lane != 0) return;
     int acc, done;
@@ -243,7 +266,15 @@ cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaSt
 cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s) {
     if (a.n < 1 || a.n > MAX_NHEADS || a.k < 1 || a.k > MAX_TOPK || a.batch < 0) return cudaErrorInvalidValue;
     if (a.batch == 0) return cudaSuccess;
-    viterbi_kernel<<<(a.batch + 3) / 4, 128, 0, s>>>(a);
+    const size_t smem = (size_t)VIT_WARPS * (a.n - 1) * a.k * a.k * sizeof(float);
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(viterbi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             VIT_WARPS * (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK * (int)sizeof(float));
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    viterbi_kernel<<<(a.batch + VIT_WARPS - 1) / VIT_WARPS, VIT_WARPS * 32, smem, s>>>(a);
     return cudaGetLastError();
 }
 

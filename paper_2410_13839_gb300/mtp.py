@@ -153,6 +153,13 @@ def mtp_profile_step(ctx: int, n_heads: int, top_k: int) -> dict:
     return {k: (float(ms[i]), int(launches[i])) for i, k in enumerate(_lib.KERNEL_KINDS)}
 
 
+def mtp_trace_step(ctx: int, n_heads: int, top_k: int, cap: int = 4096) -> np.ndarray:
+    """Timeline of one decode step: rows (kind, start_ns, wait_ns, end_ns)."""
+    out = np.zeros((cap, 4), np.int64)
+    count = check(lib.mtp_trace_step(ctx, n_heads, top_k, _ptr(out), cap))
+    return out[:count]
+
+
 def mtp_step_bytes(ctx: int, n_heads: int) -> int:
     out = ctypes.c_uint64()
     check(lib.mtp_step_bytes(ctx, n_heads, ctypes.byref(out)))
