@@ -59,7 +59,7 @@ typedef enum mtp_accept { MTP_ACCEPT_ALL = 0 } mtp_accept;
  * ahead (Sec. III-B). */
 typedef struct mtp_config {
     int32_t layers;        /* transformer blocks                                   */
-    int32_t d_model;       /* multiple of 256                                      */
+    int32_t d_model;       /* multiple of 256, at most 1024                         */
     int32_t n_attn_heads;  /* d_model / n_attn_heads must be 64                    */
     int32_t d_ffn;         /* multiple of 256                                      */
     int32_t phone_vocab;   /* phoneme table rows                                   */
@@ -173,16 +173,28 @@ MTP_API int mtp_debug_logits(mtp_ctx* ctx, float* out_logits, float* out_lse);
  * out_path int32 [max_batch][n]. */
 MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, int32_t* out_path);
 
-/* Options: MTP_OPT_GRAPHS (1 = capture each (n_heads, top_k) step into a
- * CUDA graph, default) and MTP_OPT_PDL (1 = programmatic dependent launch
- * between the step's kernels, default). */
-typedef enum mtp_option { MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1 } mtp_option;
+/* Options:
+ *   MTP_OPT_GRAPHS       1 = capture each (n_heads, top_k) step into a CUDA graph (default)
+ *   MTP_OPT_PDL          1 = programmatic dependent launch between kernels (default)
+ *   MTP_OPT_L2_PREFETCH  1 = each block kernel prefetches the next layer's weights into L2 (default)
+ *   MTP_OPT_MLP_CLUSTERS thread-block clusters of the MLP kernel (>= 1; default: as many as
+ *                        the GPU holds at once) */
+typedef enum mtp_option {
+    MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3
+} mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
+MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
 
 /* Kernel classes reported by mtp_profile_step. */
+/*   EMBED       token embedding + position of the fed rows
+ *   ATTN_BLOCK  LN1, q|k|v projection, key/value append, attention, W_o
+ *   MLP         LN2, W1, GELU, W2
+ *   HEADS       LN_f and the n heads' logits
+ *   SELECT      log-softmax, top-k, Viterbi, acceptance
+ *   SAVE        copy of each slot's last hidden state (multi-pass steps, prefill) */
 typedef enum mtp_kernel_kind {
-    MTP_K_EMBED = 0, MTP_K_QKV = 1, MTP_K_ATTN = 2, MTP_K_OPROJ = 3, MTP_K_FFN1 = 4,
-    MTP_K_FFN2 = 5, MTP_K_HEADS = 6, MTP_K_SELECT = 7, MTP_K_COUNT = 8
+    MTP_K_EMBED = 0, MTP_K_ATTN_BLOCK = 1, MTP_K_MLP = 2, MTP_K_HEADS = 3, MTP_K_SELECT = 4,
+    MTP_K_SAVE = 5, MTP_K_COUNT = 6
 } mtp_kernel_kind;
 
 /* Run one decode step with each kernel launched alone (no graph, no PDL)
@@ -194,11 +206,13 @@ MTP_API int mtp_profile_step(mtp_ctx* ctx, int n_heads, int top_k, float* out_ms
                              int32_t* out_launches);
 
 /* Run one decode step (graph and PDL as the options say) with a timeline
- * record per kernel launch: out int64 [cap][4] rows of {mtp_kernel_kind,
- * earliest CTA start, latest CTA past its dependency wait, latest CTA end},
+ * record per kernel launch: out int64 [cap][MTP_TRACE_COLS] rows of
+ * {mtp_kernel_kind, earliest CTA start, latest CTA past its dependency wait,
+ * latest CTA end, then 8 phase marks (latest CTA past each, 0 if unused)},
  * times in ns of the GPU's global timer.  Returns the number of launches
  * recorded (<= cap).  The step's effect on the slots is that of
  * mtp_decode_step. */
+#define MTP_TRACE_COLS 12
 MTP_API int mtp_trace_step(mtp_ctx* ctx, int n_heads, int top_k, int64_t* out, int cap);
 
 /* Algorithmic bytes of one decode step: weights read (all blocks and the

@@ -21,7 +21,9 @@ MTP_F32 = 0
 MTP_BF16 = 1
 MTP_OPT_GRAPHS = 0
 MTP_OPT_PDL = 1
-KERNEL_KINDS = ("embed", "qkv", "attn", "oproj", "ffn1", "ffn2", "heads", "select")
+MTP_OPT_L2_PREFETCH = 2
+MTP_OPT_MLP_CLUSTERS = 3
+KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save")
 
 
 class MtpConfig(ctypes.Structure):
@@ -64,6 +66,7 @@ def _load() -> ctypes.CDLL:
         "mtp_debug_logits": (i32, [vp, vp, vp]),
         "mtp_debug_lattice": (i32, [vp, vp, vp, vp]),
         "mtp_set_option": (i32, [vp, i32, i32]),
+        "mtp_get_option": (i32, [vp, i32, vp]),
         "mtp_profile_step": (i32, [vp, i32, i32, vp, vp]),
         "mtp_step_bytes": (i32, [vp, i32, vp]),
         "mtp_trace_step": (i32, [vp, i32, i32, vp, i32]),

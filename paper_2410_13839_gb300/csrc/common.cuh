@@ -71,6 +71,11 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
         : "memory");
 }
 
+// Bulk prefetch of a global range into L2 (no destination, no completion).
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Programmatic dependent launch: wait until the preceding kernel in the stream
 // has completed and its writes are visible (a no-op without the attribute).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
@@ -109,8 +114,11 @@ __device__ __forceinline__ void load4(const float* p, float (&w)[4]) {
 }
 
 // ---- launch timeline (tracing option) --------------------------------------
-// A traced launch owns 3 u64 words: earliest CTA start, latest CTA past the
-// dependency wait, latest CTA end, all from %globaltimer (ns).
+// A traced launch owns TRACE_WORDS u64 words: earliest CTA start, latest CTA
+// past the dependency wait, latest CTA end, then TRACE_MARKS phase marks
+// (latest CTA past each mark), all from %globaltimer (ns).
+constexpr int TRACE_MARKS = 8;
+constexpr int TRACE_WORDS = 3 + TRACE_MARKS;
 
 __device__ __forceinline__ unsigned long long globaltimer() {
     unsigned long long t;
@@ -122,6 +130,9 @@ __device__ __forceinline__ void trace_start(unsigned long long* tr) {
 }
 __device__ __forceinline__ void trace_wait(unsigned long long* tr) {
     if (tr && threadIdx.x == 0) atomicMax(tr + 1, globaltimer());
+}
+__device__ __forceinline__ void trace_mark(unsigned long long* tr, int i) {
+    if (tr && threadIdx.x == 0) atomicMax(tr + 3 + i, globaltimer());
 }
 struct TraceEnd {
     unsigned long long* tr;

@@ -46,6 +46,8 @@ __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
         s_phone = phone;
     }
     __syncthreads();
+    if (a.zero_buf)
+        for (int i = tid; i < a.d; i += blockDim.x) a.zero_buf[(size_t)r * a.d + i] = 0.f;
     float* x = a.x + (size_t)r * a.d;
     if (!s_act) {
         for (int i = tid; i < a.d; i += blockDim.x) x[i] = 0.f;
@@ -122,12 +124,36 @@ cudaError_t launch_convert_rows(const void* src, int src_bf16, float* dst, int r
     return cudaGetLastError();
 }
 
+__global__ void __launch_bounds__(256) save_last_kernel(const float* x, const int* row_seq, const int* row_last,
+                                                        float* h_last, int d, unsigned long long* trace) {
+    TraceEnd trace_guard(trace);
+    pdl_launch_dependents();
+    pdl_wait();
+    trace_wait(trace);
+    const int r = blockIdx.x;
+    if (row_seq[r] < 0 || !row_last[r]) return;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) h_last[(size_t)row_seq[r] * d + i] = x[(size_t)r * d + i];
+}
+
+cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
+                             unsigned long long* trace, cudaStream_t s, bool pdl) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(MAX_ROWS);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, save_last_kernel, x, row_seq, row_last, h_last, d, trace);
+}
+
 __global__ void trace_reset_kernel(unsigned long long* tr, int records) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= records) return;
-    tr[3 * i] = ~0ull;
-    tr[3 * i + 1] = 0;
-    tr[3 * i + 2] = 0;
+    tr[TRACE_WORDS * i] = ~0ull;
+    for (int j = 1; j < TRACE_WORDS; ++j) tr[TRACE_WORDS * i + j] = 0;
 }
 
 cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s) {

@@ -112,6 +112,15 @@ __global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
         }
     }
     float xv[MT][XSMEM ? 1 : NSUB][4];
+    const float* xrow[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {  // input row m, or the slot's last fed row of this step
+        xrow[m] = a.A + (size_t)m * a.lda;
+        if (a.gather_x != nullptr && m < a.M) {
+            const int np = a.gather_npend[a.gather_base + m];
+            if (np > 0) xrow[m] = a.gather_x + (size_t)(m * a.gather_n + np - 1) * a.lda;
+        }
+    }
     if (!XSMEM) {
 #pragma unroll
         for (int m = 0; m < MT; ++m)
@@ -119,7 +128,7 @@ __global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
             for (int s = 0; s < (XSMEM ? 1 : NSUB); ++s) {
                 const int c = s * 32 + lane;
                 if (m < a.M && c * 4 < Kw) {
-                    load4(a.A + (size_t)m * a.lda + warp * Kw + c * 4, xv[m][s]);
+                    load4(xrow[m] + warp * Kw + c * 4, xv[m][s]);
                 } else {
 #pragma unroll
                     for (int i = 0; i < 4; ++i) xv[m][s][i] = 0.f;
@@ -129,7 +138,7 @@ __global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
         for (int i = tid; i < MT * (K / 4); i += NT) {
             const int m = i / (K / 4), c = i % (K / 4);
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (m < a.M) v = *reinterpret_cast<const float4*>(a.A + (size_t)m * a.lda + c * 4);
+            if (m < a.M) v = *reinterpret_cast<const float4*>(xrow[m] + c * 4);
             *reinterpret_cast<float4*>(xs + (size_t)m * K + c * 4) = v;
         }
     }

@@ -42,6 +42,9 @@ struct GemvArgs {
     // EPI_QKV key/value placement
     uint16_t* kv_pool; long long page_elems; long long layer_off; int n_heads, page_size, d_model;
     const int* block_table; int bt_stride;
+    // optional row gather: row m is gather_x row (m * gather_n + npend - 1) when
+    // npend = gather_npend[gather_base + m] > 0, else A row m
+    const float* gather_x; const int* gather_npend; int gather_n, gather_base;
     int* err;
     unsigned long long* trace;           // timeline record of this launch (may be null)
 };
@@ -76,6 +79,46 @@ size_t attn_smem_bytes(int page_size);
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms);
 cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl);
 
+// ------------------------------------------------------- fused block ----
+// One transformer block over <= MAX_ROWS fed rows: attn_block (LN1, q|k|v,
+// key/value append, attention, W_o) and mlp (LN2, W1, GELU, W2), each
+// accumulating into a zeroed residual buffer.
+constexpr int MLP_CLUSTER = 8;   // CTAs per cluster of the MLP kernel
+
+struct LayerArgs {
+    const float* x_in;        // [M][d] input rows of the kernel
+    float* x_out;             // [MAX_ROWS][d] accumulation target (zero on entry)
+    float* x_zero;            // [MAX_ROWS][d] buffer the next kernel accumulates into
+    int M, d, d_ffn, n_heads, rows_per_group;
+    const int* row_seq; const int* row_pos;
+    const float* ln_g; const float* ln_b; float ln_eps;
+    // attention half (weights head-major: q|k|v rows of head h, W_o columns of head h)
+    const void* wqkv;         // [H][3*64][d]
+    const float* bqkv;        // [H][3*64]
+    const void* wo;           // [H][d][64]
+    const float* bo;          // [d]
+    __nv_bfloat16* kv_pool; long long page_elems; long long layer_off; int page_size;
+    const int* block_table; int bt_stride;
+    int plan; const int* seq_len; const int* seq_new; int seq_base; int val_seq, val_old, val_new;
+    const int* active; const int* done; int slots;          // PLAN_DEVICE row rule (as the embedding)
+    // next layer's weights of the same kernel, prefetched into L2 (null: none)
+    const void* next_w_a; const void* next_w_b;
+    // MLP half
+    const void* w1;           // [d_ffn][d]
+    const void* w2t;          // [d_ffn][d]  (W2 transposed)
+    const float* b1; const float* b2;
+    int ffn_rows_per_cta;
+    int* err;
+    unsigned long long* trace;
+};
+
+size_t attn_block_smem_bytes(int d, int wbytes, int page_size);
+size_t mlp_smem_bytes(int d, int rows_per_cta, int wbytes);
+cudaError_t launch_attn_block(const LayerArgs& a, bool w_bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_mlp(const LayerArgs& a, bool w_bf16, int grid, cudaStream_t s, bool pdl);
+// clusters of the MLP kernel that can be resident at once (rows per CTA chosen for that count)
+cudaError_t mlp_max_clusters(int d, int num_sms, int wbytes, int d_ffn, int* clusters);
+
 // --------------------------------------------------------------- embed ----
 struct EmbedArgs {
     int mode;                  // 0 = decode rows from slot state, 1 = prefill chunk
@@ -90,6 +133,7 @@ struct EmbedArgs {
     const int* active; const int* done; const int* n_pending; const int* pending; const int* seq_len;
     // prefill
     int slot, p0, n_ph, total, prompt_stride; const int* prompt;
+    float* zero_buf;           // [MAX_ROWS][d] zeroed (first residual accumulation target)
     int* err;
     unsigned long long* trace;
 };
@@ -131,5 +175,8 @@ struct SlotSet {
 };
 cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s);
 cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s);
+// copy each slot's last fed row (row_last) of x [MAX_ROWS][d] into h_last [slot][d]
+cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
+                             unsigned long long* trace, cudaStream_t s, bool pdl);
 
 }  // namespace mtp

@@ -1,0 +1,933 @@
+// layer_fused.cu -- one pre-LN transformer block (Sec. III-A) over <= 8 fed
+// rows as two thread-block-cluster kernels.
+//
+// Kernel A (attention half), grid (CA, H): the CA = 8 CTAs of a cluster serve
+// one attention head.
+//   1. before the dependency wait: cp.async.bulk of the CTA's 24 of the
+//      head's 192 q|k|v weight rows, its d/CA rows of the head's W_o column
+//      block, and the cached key/value pages of its key split;
+//   2. LN1 + its 24 projection rows -> shared memory; key/value rows are
+//      appended to the paged cache (bf16);
+//   3. cluster barrier; every CTA gathers the head's q, k, v of the fed rows
+//      from its peers' shared memory (DSMEM);
+//   4. attention of the fed rows over its split of the keys (online softmax);
+//      the keys fed this step come from the gathered rows, the older ones
+//      from the cache;
+//   5. cluster barrier; the CA partial (max, sum, output) triples are merged
+//      (log-sum-exp) from DSMEM, and the CTA applies its rows of W_o to the
+//      head's output, adding the result (plus residual and bias, head 0) into
+//      the next residual buffer with float atomics.
+// Kernel B (MLP), grid = clusters of CB CTAs over the FFN width: each CTA
+// takes a slice of FFN rows, computes u = GELU(LN2(x) W1^T + b1) for them and
+// the partial u W2^T over all d outputs; the cluster sums its partials in
+// DSMEM and adds them (plus residual and bias, cluster 0) into the layer's
+// output buffer with float atomics.
+//
+// Residual buffers rotate in threes so that every atomic target was zeroed
+// by the previous kernel: A(l) zeroes B(l)'s target and B(l) zeroes the
+// target of A(l + 1).
+#include <cooperative_groups.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace mtp {
+namespace {
+
+constexpr int CA = 8;                    // CTAs per head (cluster of kernel A)
+constexpr int QROWS = 3 * HEAD_DIM / CA;  // projection rows per CTA (24)
+constexpr int MIN_TILE = 64;              // keys staged per batch: at least this many, whole pages
+constexpr int PARTW = 2 + HEAD_DIM;       // (max, sum, out[64])
+constexpr int NTHREADS = 256;
+constexpr int NWARPS = NTHREADS / 32;
+
+__host__ __device__ inline size_t al128(size_t x) { return (x + 127) & ~(size_t)127; }
+
+// ---- shared-memory layouts (host and device compute the same offsets) ----
+struct ALayout {
+    size_t wqkv, wo, ks, vs, qkvp, qkvf, qs, sc, part, attn, red, res, total;
+    int tile;       // keys of the dedicated staging slots
+    int sc_stride;  // keys per batch (dedicated and reused slots)
+    __host__ __device__ ALayout(int d, int wbytes, int mt, int page) {
+        const int groups = (QROWS * mt + 31) / 32;
+        tile = (MIN_TILE + page - 1) / page * page;  // whole pages, at least MIN_TILE keys
+        const int ATT_TILE = tile;
+        wqkv = 0;
+        wo = al128(wqkv + (size_t)QROWS * d * wbytes);
+        ks = al128(wo + (size_t)(d / CA) * HEAD_DIM * wbytes);  // page slots: [keys | values] each
+        vs = ks;
+        qkvp = al128(ks + (size_t)2 * ATT_TILE * HEAD_DIM * 2);
+        qkvf = al128(qkvp + (size_t)QROWS * mt * 4);
+        qs = al128(qkvf + (size_t)3 * HEAD_DIM * mt * 4);
+        sc = al128(qs + (size_t)mt * HEAD_DIM * 4);
+        sc_stride = (ATT_TILE / page + (QROWS * d * wbytes) / (4 * page * HEAD_DIM)) * page;  // keys per batch
+        part = al128(sc + (size_t)mt * sc_stride * 4);
+        attn = al128(part + (size_t)mt * PARTW * 4);
+        red = al128(attn + (size_t)mt * HEAD_DIM * 4);
+        res = al128(red + (size_t)NWARPS * groups * 32 * 4);
+        total = al128(res + (size_t)mt * (d / CA) * 4);
+    }
+};
+
+struct BLayout {
+    size_t w1, w2, u, ypart, red, total;
+    __host__ __device__ BLayout(int d, int rows, int wbytes, int mt, int cb) {
+        (void)cb;
+        const int groups = (rows * mt + 31) / 32;
+        w1 = 0;
+        w2 = al128(w1 + (size_t)rows * d * wbytes);
+        u = al128(w2 + (size_t)rows * d * wbytes);
+        const size_t ybytes = (size_t)mt * d * 4;
+        // the partial outputs reuse W1's space once u is known, when it fits
+        ypart = ((size_t)rows * d * wbytes >= ybytes) ? w1 : al128(u + (size_t)rows * mt * 4);
+        red = al128((ypart == w1 ? u + (size_t)rows * mt * 4 : ypart + ybytes));
+        total = al128(red + (size_t)NWARPS * groups * 32 * 4);
+    }
+};
+
+// Sum v[i] over the 32 lanes for every i; lane l returns the total of v[l].
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int width = 16; width >= 1; width >>= 1) {
+        const bool upper = (lane & width) != 0;
+#pragma unroll
+        for (int i = 0; i < width; ++i) {
+            const float send = upper ? v[i] : v[i + width];
+            const float keep = upper ? v[i + width] : v[i];
+            v[i] = keep + __shfl_xor_sync(FULL_MASK, send, width);
+        }
+    }
+    return v[0];
+}
+
+// Input rows for a projection: lane holds columns warp*Kw + lane*4 .. +3 of
+// each of the MT rows (K <= 1024, one 4-column chunk per lane), LayerNorm'd.
+template <int MT>
+struct RowRegs {
+    float v[MT][4];
+};
+
+template <int MT>
+__device__ __forceinline__ void load_rows(const float* x, int ld, int M, int K, RowRegs<MT>& r) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int Kw = K / NWARPS;
+    const bool valid = lane * 4 < Kw;
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+        if (m < M && valid) {
+            load4(x + (size_t)m * ld + warp * Kw + lane * 4, r.v[m]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) r.v[m][i] = 0.f;
+        }
+    }
+}
+
+// LayerNorm of the register rows in place.  Each warp takes the mean and the
+// sum of squared deviations of its K/NWARPS columns (two passes over
+// registers), and one block reduction merges the warps' equal-sized slices:
+// mean = average of the warp means, M2 = sum of warp M2 + Kw * sum (mean_w - mean)^2.
+template <int MT>
+__device__ __forceinline__ void layer_norm_rows(RowRegs<MT>& r, int K, const float (&gam)[4], const float (&bet)[4],
+                                                float eps, float (*part)[MT], float (*stat)[MT]) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int Kw = K / NWARPS;
+    const bool valid = lane * 4 < Kw;
+    float (*pm2)[MT] = part + NWARPS;  // second half of the scratch
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+        float s1 = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s1 += valid ? r.v[m][i] : 0.f;
+        const float mw = warp_sum(s1) / (float)Kw;
+        float s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float t = r.v[m][i] - mw;
+            s2 += valid ? t * t : 0.f;
+        }
+        const float m2 = warp_sum(s2);
+        if (lane == 0) {
+            part[warp][m] = mw;
+            pm2[warp][m] = m2;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x < MT) {
+        const int m = threadIdx.x;
+        float mean = 0.f;
+#pragma unroll
+        for (int w = 0; w < NWARPS; ++w) mean += part[w][m];
+        mean /= (float)NWARPS;
+        float m2 = 0.f;
+#pragma unroll
+        for (int w = 0; w < NWARPS; ++w) {
+            const float dm = part[w][m] - mean;
+            m2 += pm2[w][m] + (float)Kw * dm * dm;
+        }
+        stat[0][m] = mean;
+        stat[1][m] = 1.0f / sqrtf(m2 / (float)K + eps);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int m = 0; m < MT; ++m)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) r.v[m][i] = (r.v[m][i] - stat[0][m]) * stat[1][m] * gam[i] + bet[i];
+}
+
+// out[row * MT + m] = sum_k W[row, k] x[m, k] for rows < R of the weight
+// slice in shared memory (row-major, K columns); red = NWARPS x groups x 32.
+template <typename WT, int MT>
+__device__ __forceinline__ void project_rows(const WT* wsm, int R, int K, const RowRegs<MT>& x, float* red,
+                                             float* out) {
+    constexpr int G = 32 / MT;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int Kw = K / NWARPS;
+    const int ngroups = (R + G - 1) / G;
+    const bool valid = lane * 4 < Kw;
+    const int k = warp * Kw + lane * 4;
+    for (int g = 0; g < ngroups; ++g) {
+        float acc[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+        if (valid) {
+#pragma unroll
+            for (int r = 0; r < G; ++r) {
+                const int row = g * G + r;
+                if (row < R) {
+                    float w[4];
+                    load4(wsm + (size_t)row * K + k, w);
+#pragma unroll
+                    for (int m = 0; m < MT; ++m) {
+                        float t = acc[r * MT + m];
+                        t = fmaf(w[0], x.v[m][0], t);
+                        t = fmaf(w[1], x.v[m][1], t);
+                        t = fmaf(w[2], x.v[m][2], t);
+                        t = fmaf(w[3], x.v[m][3], t);
+                        acc[r * MT + m] = t;
+                    }
+                }
+            }
+        }
+        red[(warp * ngroups + g) * 32 + lane] = reduce_scatter32(acc, lane);
+    }
+    __syncthreads();
+    for (int o = threadIdx.x; o < R * MT; o += NTHREADS) {
+        const int g = o / 32, l = o % 32;
+        float y = 0.f;
+#pragma unroll
+        for (int w = 0; w < NWARPS; ++w) y += red[(w * ngroups + g) * 32 + l];
+        out[o] = y;
+    }
+    __syncthreads();
+}
+
+__device__ __forceinline__ void zero_slice(float* buf, size_t n, int part, int parts) {
+    if (!buf) return;
+    const size_t per = (n + parts - 1) / parts;
+    const size_t b = (size_t)part * per, e = min(n, b + per);
+    for (size_t i = b + threadIdx.x; i < e; i += NTHREADS) buf[i] = 0.f;
+}
+
+// Slot and position of fed row r of this pass, from state left by earlier
+// steps only (the same rule the embedding applies), so it is known before
+// the dependency wait.
+__device__ __forceinline__ void plan_row(const LayerArgs& a, int r, int& seq, int& pos) {
+    seq = -1;
+    pos = -1;
+    if (r >= a.M) return;
+    if (a.plan == PLAN_DEVICE) {
+        const int g = r / a.rows_per_group, j = r % a.rows_per_group;
+        const int b = a.seq_base + g;
+        if (b < a.slots && a.active[b] && !a.done[b] && j < a.seq_new[b]) {
+            seq = b;
+            pos = a.seq_len[b] + j;
+        }
+    } else if (r < a.val_new) {
+        seq = a.val_seq;
+        pos = a.val_old + r;
+    }
+}
+
+// ============================================================ kernel A ====
+
+template <typename WT, int MT>
+__global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_block_kernel(const LayerArgs a) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ uint64_t bar;
+    __shared__ float ln_part[2 * NWARPS][MT];
+    __shared__ float ln_stat[2][MT];
+    __shared__ int s_seq[MT], s_pos[MT], s_page[MT];
+    __shared__ int s_gseq[MT], s_gold[MT], s_gktot[MT];
+    __shared__ int s_pre, s_armed;
+    TraceEnd trace_guard(a.trace);
+    cg::cluster_group cluster = cg::this_cluster();
+
+    const int s = blockIdx.x, h = blockIdx.y;  // split (cluster rank) and head
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int d = a.d, H = a.n_heads, P = a.page_size;
+    const int orows = d / CA;  // W_o rows of this CTA
+    const ALayout L(d, sizeof(WT), MT, P);
+    const int ATT_TILE = L.tile;
+    const int SC_STRIDE = L.sc_stride;
+    WT* wqkv = reinterpret_cast<WT*>(smem + L.wqkv);
+    WT* wo = reinterpret_cast<WT*>(smem + L.wo);
+    __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem + L.ks);
+    float* qkvp = reinterpret_cast<float*>(smem + L.qkvp);  // [QROWS][MT]
+    float* qkvf = reinterpret_cast<float*>(smem + L.qkvf);  // [192][MT]
+    float* qs = reinterpret_cast<float*>(smem + L.qs);      // [MT][64]
+    float* sc = reinterpret_cast<float*>(smem + L.sc);      // [MT][SC_STRIDE]
+    float* part = reinterpret_cast<float*>(smem + L.part);  // [MT][PARTW]
+    float* attn = reinterpret_cast<float*>(smem + L.attn);  // [MT][64]
+    float* red = reinterpret_cast<float*>(smem + L.red);
+    float* res = reinterpret_cast<float*>(smem + L.res);    // [MT][orows]
+    const long long kv_head = (long long)h * P * HEAD_DIM;
+    const long long v_off = (long long)H * P * HEAD_DIM;
+    const int rpg = a.rows_per_group;
+
+    // ---- 1. before the wait: fed rows, weights, cached keys/values ----
+    if (tid < MT) {
+        int seq, pos;
+        plan_row(a, tid, seq, pos);
+        s_seq[tid] = seq;
+        s_pos[tid] = pos;
+        s_page[tid] = seq >= 0 ? a.block_table[(size_t)seq * a.bt_stride + pos / P] : -1;
+    }
+    if (tid == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+        s_pre = 0;
+    }
+    __syncthreads();
+    if (tid < MT) {  // per group: slot, first fed position (= cached length) and key count
+        const int g = tid;
+        int seq = -1, kmin = 1 << 30, kmax = 0;
+        for (int j = 0; j < rpg && g * rpg + j < MT; ++j) {
+            const int r = g * rpg + j;
+            if (s_seq[r] >= 0) {
+                seq = s_seq[r];
+                kmin = min(kmin, s_pos[r]);
+                kmax = max(kmax, s_pos[r] + 1);
+            }
+        }
+        s_gseq[g] = seq;
+        s_gold[g] = seq >= 0 ? kmin : 0;
+        s_gktot[g] = kmax;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        const uint32_t wq = (uint32_t)QROWS * d * sizeof(WT);
+        const uint32_t wob = (uint32_t)orows * HEAD_DIM * sizeof(WT);
+        uint32_t kvb = 0;
+        int n_pre = 0, pg0 = 0;
+        const int seq = s_gseq[0];
+        if (seq >= 0) {  // group 0: pages of this split holding only keys of earlier steps
+            const int old_len = s_gold[0];
+            const int n_pg = (s_gktot[0] + P - 1) / P;
+            const int pps = (n_pg + CA - 1) / CA;
+            pg0 = s * pps;
+            const int pg1 = min(n_pg, pg0 + pps);
+            int pre_end = min(min(pg1, pg0 + ATT_TILE / P), old_len / P);
+            for (int p = pg0; p < pre_end; ++p)
+                if (a.block_table[(size_t)seq * a.bt_stride + p] < 0) pre_end = p;
+            n_pre = max(0, pre_end - pg0);
+            kvb = 2u * (uint32_t)n_pre * P * HEAD_DIM * 2;
+        }
+        mbar_arrive_expect_tx(&bar, wq + wob + kvb);
+        const char* srcq = reinterpret_cast<const char*>(a.wqkv) + ((size_t)h * 3 * HEAD_DIM + s * QROWS) * d * sizeof(WT);
+        for (uint32_t off = 0; off < wq; off += 32768)
+            bulk_copy_g2s(smem + L.wqkv + off, srcq + off, min(32768u, wq - off), &bar);
+        const char* srco = reinterpret_cast<const char*>(a.wo) + ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT);
+        bulk_copy_g2s(smem + L.wo, srco, wob, &bar);
+        for (int i = 0; i < n_pre; ++i) {
+            const int phys = a.block_table[(size_t)seq * a.bt_stride + pg0 + i];
+            const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
+            bulk_copy_g2s(Ks + (size_t)i * 2 * P * HEAD_DIM, base, (uint32_t)P * HEAD_DIM * 2, &bar);
+            bulk_copy_g2s(Ks + (size_t)i * 2 * P * HEAD_DIM + P * HEAD_DIM, base + v_off, (uint32_t)P * HEAD_DIM * 2,
+                          &bar);
+        }
+        s_pre = n_pre;
+        if (a.next_w_a) {  // the next layer's slices of the same weights, into L2
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + (srcq - reinterpret_cast<const char*>(a.wqkv)), wq);
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + (srco - reinterpret_cast<const char*>(a.wo)), wob);
+        }
+    }
+    float gam[4], bet[4], bq[2] = {0.f, 0.f};
+    {
+        const int Kw = d / NWARPS;
+        if (lane * 4 < Kw) {
+            load4(a.ln_g + warp * Kw + lane * 4, gam);
+            load4(a.ln_b + warp * Kw + lane * 4, bet);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) gam[i] = bet[i] = 0.f;
+        }
+        for (int u = 0; u < 2; ++u) {
+            const int o = tid + u * NTHREADS;
+            if (o < QROWS * MT) bq[u] = __ldg(a.bqkv + h * 3 * HEAD_DIM + s * QROWS + o / MT);
+        }
+    }
+
+    pdl_launch_dependents();
+    pdl_wait();
+    trace_wait(a.trace);
+
+    // ---- 2. inputs: LN1, projection ----
+    RowRegs<MT> xr;
+    load_rows<MT>(a.x_in, d, a.M, d, xr);
+    if (h == 0) {  // residual slice for the W_o rows of this CTA
+        for (int i = tid; i < MT * orows; i += NTHREADS) {
+            const int m = i / orows, f = s * orows + i % orows;
+            res[i] = m < a.M ? a.x_in[(size_t)m * d + f] + a.bo[f] : 0.f;
+        }
+    }
+    zero_slice(a.x_zero, (size_t)MAX_ROWS * d, h * CA + s, H * CA);
+    layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
+    trace_mark(a.trace, 0);  // inputs loaded, LN1 done
+    bool ok = mbar_wait(&bar, 0, a.err);
+    ok = __syncthreads_and(ok) != 0;
+    if (!ok) {
+        mbar_wait(&bar, 0, nullptr);
+        cluster.sync();
+        cluster.sync();
+        cluster.sync();
+        return;
+    }
+    trace_mark(a.trace, 1);  // weights and cached keys in shared memory
+    project_rows<WT, MT>(wqkv, QROWS, d, xr, red, qkvp);
+    for (int o = tid; o < QROWS * MT; o += NTHREADS) {
+        const float y = qkvp[o] + (o < NTHREADS ? bq[0] : bq[1]);
+        qkvp[o] = y;
+        const int row = s * QROWS + o / MT, m = o % MT;  // row within the head's q|k|v
+        if (row >= HEAD_DIM && s_seq[m] >= 0) {             // key or value: append to the cache
+            const int sec = row / HEAD_DIM, dd = row % HEAD_DIM;
+            const int page = s_page[m];
+            if (page < 0) {
+                atomicOr(a.err, ERR_BOUNDS);
+                continue;
+            }
+            const long long idx = (long long)page * a.page_elems + a.layer_off + (sec - 1) * v_off + kv_head +
+                                  (long long)(s_pos[m] % P) * HEAD_DIM + dd;
+            reinterpret_cast<uint16_t*>(a.kv_pool)[idx] = f32_to_bf16_bits(y);
+        }
+    }
+
+    trace_mark(a.trace, 2);  // projection rows done
+    // ---- 3. gather the head's q, k, v of the fed rows from the cluster ----
+    cluster.sync();
+    trace_mark(a.trace, 3);
+    {
+        constexpr int PER = (3 * HEAD_DIM * MT + NTHREADS - 1) / NTHREADS;
+        float v[PER];
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {  // issue every remote load before using any
+            const int i = tid + u * NTHREADS;
+            v[u] = 0.f;
+            if (i < 3 * HEAD_DIM * MT) {
+                const int row = i / MT;
+                v[u] = cluster.map_shared_rank(qkvp, row / QROWS)[(row % QROWS) * MT + i % MT];
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int i = tid + u * NTHREADS;
+            if (i < 3 * HEAD_DIM * MT)
+                qkvf[i] = i / MT >= HEAD_DIM ? __bfloat162float(__float2bfloat16_rn(v[u])) : v[u];  // keys/values as cached
+        }
+    }
+    __syncthreads();
+    for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS) {
+        const int m = i / HEAD_DIM, dd = i % HEAD_DIM;
+        qs[i] = s_seq[m] >= 0 ? qkvf[dd * MT + m] * 0.125f : 0.f;  // 1/sqrt(64)
+    }
+
+    trace_mark(a.trace, 4);  // gathered
+    // ---- 4. attention over this CTA's split of each group's keys ----
+    const int row_j = warp;  // warp j owns fed row j (MT <= 8 warps)
+    const bool row_on = row_j < MT && row_j < a.M && s_seq[min(row_j, MT - 1)] >= 0;
+    const int pos_j = row_on ? s_pos[row_j] : -1;
+    const int grp_j = row_j / rpg;
+    float m_run = -INFINITY, l_run = 0.f, acc0 = 0.f, acc1 = 0.f;
+    const int G = (a.M + rpg - 1) / rpg;
+    // page slots: the dedicated staging area, then the q|k|v weight area, free after the projection
+    const int slot_elems = 2 * P * HEAD_DIM;  // keys then values of one page
+    const int n_ded = ATT_TILE / P;
+    const int n_slots = n_ded + (int)((size_t)QROWS * d * sizeof(WT) / ((size_t)slot_elems * 2));
+    __nv_bfloat16* const wq_slots = reinterpret_cast<__nv_bfloat16*>(smem + L.wqkv);
+    auto slot_keys = [&](int i) -> __nv_bfloat16* {
+        return i < n_ded ? Ks + (size_t)i * slot_elems : wq_slots + (size_t)(i - n_ded) * slot_elems;
+    };
+    uint32_t phase = 1;  // phase 0 of the barrier brought the weights
+    for (int g = 0; g < G; ++g) {
+        const int seq = s_gseq[g], old_len = s_gold[g], K_tot = s_gktot[g];
+        if (seq < 0) continue;
+        const int n_pg = (K_tot + P - 1) / P;
+        const int pps = (n_pg + CA - 1) / CA;
+        const int pg0 = s * pps, pg1 = min(n_pg, pg0 + pps);
+        for (int bp = pg0; bp < pg1; bp += n_slots) {
+            const int nb = min(n_slots, pg1 - bp);
+            const int nk = nb * P;
+            const int first = (g == 0 && bp == pg0) ? s_pre : 0;  // slots already filled before the wait
+            __syncthreads();  // every reader of the slots is done with the previous batch
+            if (tid == 0) {
+                uint32_t bytes = 0;
+                for (int p = first; p < nb; ++p)
+                    if (a.block_table[(size_t)seq * a.bt_stride + bp + p] >= 0) bytes += (uint32_t)slot_elems * 2;
+                if (bytes) {
+                    mbar_arrive_expect_tx(&bar, bytes);
+                    for (int p = first; p < nb; ++p) {
+                        const int phys = a.block_table[(size_t)seq * a.bt_stride + bp + p];
+                        if (phys < 0) {
+                            atomicOr(a.err, ERR_BOUNDS);
+                            continue;
+                        }
+                        const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
+                        bulk_copy_g2s(slot_keys(p), base, (uint32_t)P * HEAD_DIM * 2, &bar);
+                        bulk_copy_g2s(slot_keys(p) + P * HEAD_DIM, base + v_off, (uint32_t)P * HEAD_DIM * 2, &bar);
+                    }
+                }
+                s_armed = bytes > 0;
+            }
+            __syncthreads();
+            if (s_armed) {
+                if (!mbar_wait(&bar, phase & 1, a.err)) mbar_wait(&bar, phase & 1, nullptr);
+                ++phase;
+            }
+            for (int i = tid; i < nk * HEAD_DIM; i += NTHREADS) {  // keys fed this step, from the gather
+                const int key = bp * P + i / HEAD_DIM, dd = i % HEAD_DIM;
+                if (key >= old_len && key < K_tot) {
+                    const int m = g * rpg + (key - old_len);
+                    __nv_bfloat16* kp = slot_keys((key - bp * P) / P) + ((key - bp * P) % P) * HEAD_DIM + dd;
+                    kp[0] = __float2bfloat16_rn(qkvf[(HEAD_DIM + dd) * MT + m]);
+                    kp[P * HEAD_DIM] = __float2bfloat16_rn(qkvf[(2 * HEAD_DIM + dd) * MT + m]);
+                }
+            }
+            __syncthreads();
+            // scores: thread t = key t of the batch, rows of this group
+            for (int t = tid; t < nk; t += NTHREADS) {
+                const __nv_bfloat16* krow = slot_keys(t / P) + (t % P) * HEAD_DIM;
+                float scv[MT];
+#pragma unroll
+                for (int j = 0; j < MT; ++j) scv[j] = 0.f;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const int cc = (c + t) & 7;
+                    const uint4 kr = *reinterpret_cast<const uint4*>(krow + cc * 8);
+                    const float kf[8] = {bf16_lo(kr.x), bf16_hi(kr.x), bf16_lo(kr.y), bf16_hi(kr.y),
+                                         bf16_lo(kr.z), bf16_hi(kr.z), bf16_lo(kr.w), bf16_hi(kr.w)};
+#pragma unroll
+                    for (int j = 0; j < MT; ++j) {
+                        const float4 q0 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8);
+                        const float4 q1 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8 + 4);
+                        float v = scv[j];
+                        v = fmaf(q0.x, kf[0], v); v = fmaf(q0.y, kf[1], v);
+                        v = fmaf(q0.z, kf[2], v); v = fmaf(q0.w, kf[3], v);
+                        v = fmaf(q1.x, kf[4], v); v = fmaf(q1.y, kf[5], v);
+                        v = fmaf(q1.z, kf[6], v); v = fmaf(q1.w, kf[7], v);
+                        scv[j] = v;
+                    }
+                }
+                const int kp = bp * P + t;
+#pragma unroll
+                for (int j = 0; j < MT; ++j) {
+                    const bool vis = j < a.M && s_seq[j] >= 0 && j / rpg == g && kp <= s_pos[j] && kp < K_tot;
+                    sc[j * SC_STRIDE + t] = vis ? scv[j] : -INFINITY;
+                }
+            }
+            __syncthreads();
+            if (row_on && grp_j == g) {
+                float* pr = sc + row_j * SC_STRIDE;
+                float bmax = -INFINITY;
+                for (int t = lane; t < nk; t += 32) bmax = fmaxf(bmax, pr[t]);
+                bmax = warp_max(bmax);
+                const float m_new = fmaxf(m_run, bmax);
+                if (m_new != -INFINITY) {
+                    const float corr = expf(m_run - m_new);
+                    float lsum = 0.f;
+                    for (int t = lane; t < nk; t += 32) {
+                        const float p = expf(pr[t] - m_new);
+                        pr[t] = p;
+                        lsum += p;
+                    }
+                    lsum = warp_sum(lsum);
+                    l_run = l_run * corr + lsum;
+                    acc0 *= corr;
+                    acc1 *= corr;
+                    m_run = m_new;
+                    __syncwarp();
+                    const int kend = min(nk, pos_j - bp * P + 1);
+                    float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+                    for (int p0 = 0; p0 < kend; p0 += P) {  // page by page
+                        const __nv_bfloat16* vpage = slot_keys(p0 / P) + P * HEAD_DIM + 2 * lane;
+                        const int pend = min(P, kend - p0);
+                        int t = 0;
+                        for (; t + 4 <= pend; t += 4) {
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                const float p = pr[p0 + t + u];
+                                const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t + u) * HEAD_DIM);
+                                a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
+                                a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
+                            }
+                        }
+                        for (; t < pend; ++t) {
+                            const float p = pr[p0 + t];
+                            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + t * HEAD_DIM);
+                            a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
+                            a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
+                        }
+                    }
+                    acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
+                    acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (row_j < MT) {
+        float* pj = part + row_j * PARTW;
+        if (lane == 0) {
+            pj[0] = m_run;
+            pj[1] = l_run;
+        }
+        pj[2 + 2 * lane] = acc0;
+        pj[3 + 2 * lane] = acc1;
+    }
+
+    trace_mark(a.trace, 5);  // attention partials done
+    // ---- 5. merge the splits (DSMEM) and apply this CTA's W_o rows ----
+    cluster.sync();
+    trace_mark(a.trace, 6);
+    if (row_on) {
+        float ms = -INFINITY, ls = 0.f, o0[CA], o1[CA];
+#pragma unroll
+        for (int r = 0; r < CA; ++r) {
+            const float* peer = cluster.map_shared_rank(part, r) + row_j * PARTW;
+            if (lane == r) {
+                ms = peer[0];
+                ls = peer[1];
+            }
+            o0[r] = peer[2 + 2 * lane];
+            o1[r] = peer[3 + 2 * lane];
+        }
+        const float M = warp_max(ms);
+        const float w = (ms == -INFINITY) ? 0.f : expf(ms - M);
+        const float Lsum = warp_sum(lane < CA ? w * ls : 0.f);
+        float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+        for (int r = 0; r < CA; ++r) {
+            const float wr = __shfl_sync(FULL_MASK, w, r);
+            r0 = fmaf(wr, o0[r], r0);
+            r1 = fmaf(wr, o1[r], r1);
+        }
+        attn[row_j * HEAD_DIM + 2 * lane] = r0 / Lsum;
+        attn[row_j * HEAD_DIM + 2 * lane + 1] = r1 / Lsum;
+    } else if (row_j < MT) {
+        attn[row_j * HEAD_DIM + 2 * lane] = 0.f;
+        attn[row_j * HEAD_DIM + 2 * lane + 1] = 0.f;
+    }
+    __syncthreads();
+    for (int o = tid; o < orows * MT; o += NTHREADS) {
+        const int m = o / orows, t = o % orows;  // fed row m, W_o row t: a warp adds 32 consecutive floats
+        if (m >= a.M || s_seq[m] < 0) continue;
+        const WT* wr = wo + (size_t)t * HEAD_DIM;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};  // four independent chains
+#pragma unroll
+        for (int c = 0; c < HEAD_DIM / 4; ++c) {
+            const int cc = (c + t) & (HEAD_DIM / 4 - 1);  // rotate to spread banks
+            float w4[4];
+            load4(wr + cc * 4, w4);
+            const float4 av = *reinterpret_cast<const float4*>(attn + m * HEAD_DIM + cc * 4);
+            float v = acc[c & 3];
+            v = fmaf(w4[0], av.x, v);
+            v = fmaf(w4[1], av.y, v);
+            v = fmaf(w4[2], av.z, v);
+            v = fmaf(w4[3], av.w, v);
+            acc[c & 3] = v;
+        }
+        float y = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+        if (h == 0) y += res[m * orows + t];
+        atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
+    }
+    trace_mark(a.trace, 7);  // output projection added
+    cluster.sync();  // peers may still read this CTA's shared memory
+}
+
+// ============================================================ kernel B ====
+
+template <typename WT, int MT, int CB>
+__global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ uint64_t bar;
+    __shared__ float ln_part[2 * NWARPS][MT];
+    __shared__ float ln_stat[2][MT];
+    __shared__ int s_act[MT];
+    TraceEnd trace_guard(a.trace);
+    cg::cluster_group cluster = cg::this_cluster();
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int d = a.d, F = a.d_ffn;
+    const int rpc = a.ffn_rows_per_cta;
+    const int f0 = blockIdx.x * rpc;
+    const int R = max(0, min(rpc, F - f0));
+    const int rank = (int)cluster.block_rank();
+    const int cols = d / CB;  // output columns this CTA reduces
+    const BLayout L(d, rpc, sizeof(WT), MT, CB);
+    WT* w1 = reinterpret_cast<WT*>(smem + L.w1);
+    WT* w2 = reinterpret_cast<WT*>(smem + L.w2);
+    float* u = reinterpret_cast<float*>(smem + L.u);          // [R][MT]
+    float* ypart = reinterpret_cast<float*>(smem + L.ypart);  // [MT][d]
+    float* red = reinterpret_cast<float*>(smem + L.red);
+    const bool first_cluster = blockIdx.x < CB;
+
+    if (tid < MT) {
+        int seq, pos;
+        plan_row(a, tid, seq, pos);
+        s_act[tid] = seq >= 0;
+    }
+    if (tid == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (tid == 0 && R > 0) {
+        const uint32_t wb = (uint32_t)R * d * sizeof(WT);
+        mbar_arrive_expect_tx(&bar, 2 * wb);
+        const size_t off0 = (size_t)f0 * d * sizeof(WT);
+        const char* s1 = reinterpret_cast<const char*>(a.w1) + off0;
+        const char* s2 = reinterpret_cast<const char*>(a.w2t) + off0;
+        for (uint32_t off = 0; off < wb; off += 32768) {
+            bulk_copy_g2s(smem + L.w1 + off, s1 + off, min(32768u, wb - off), &bar);
+            bulk_copy_g2s(smem + L.w2 + off, s2 + off, min(32768u, wb - off), &bar);
+        }
+        if (a.next_w_a) {  // the next layer's slices, into L2
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + off0, wb);
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + off0, wb);
+        }
+    }
+    float gam[4], bet[4], b1v[2] = {0.f, 0.f};
+    {
+        const int Kw = d / NWARPS;
+        if (lane * 4 < Kw) {
+            load4(a.ln_g + warp * Kw + lane * 4, gam);
+            load4(a.ln_b + warp * Kw + lane * 4, bet);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) gam[i] = bet[i] = 0.f;
+        }
+        for (int k = 0; k < 2; ++k) {
+            const int o = tid + k * NTHREADS;
+            if (o < R * MT) b1v[k] = __ldg(a.b1 + f0 + o / MT);
+        }
+    }
+
+    pdl_launch_dependents();
+    pdl_wait();
+    trace_wait(a.trace);
+
+    RowRegs<MT> xr;
+    load_rows<MT>(a.x_in, d, a.M, d, xr);
+    constexpr int RES_PER = 2;  // residual items per thread kept in registers (MT * cols / 4 <= 512)
+    float4 resv[RES_PER];
+#pragma unroll
+    for (int k = 0; k < RES_PER; ++k) {  // residual and bias of the columns this CTA reduces
+        const int i = tid + k * NTHREADS;
+        resv[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (first_cluster && i < MT * cols / 4) {
+            const int m = i / (cols / 4), c = rank * cols + (i % (cols / 4)) * 4;
+            if (m < a.M) {
+                const float4 xv = *reinterpret_cast<const float4*>(a.x_in + (size_t)m * d + c);
+                const float4 bv = *reinterpret_cast<const float4*>(a.b2 + c);
+                resv[k] = make_float4(xv.x + bv.x, xv.y + bv.y, xv.z + bv.z, xv.w + bv.w);
+            }
+        }
+    }
+    zero_slice(a.x_zero, (size_t)MAX_ROWS * d, blockIdx.x, gridDim.x);
+    layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
+
+    trace_mark(a.trace, 0);  // inputs loaded, LN2 done
+    bool ok = R == 0 || mbar_wait(&bar, 0, a.err);
+    ok = __syncthreads_and(ok) != 0;
+    if (!ok) {
+        if (R > 0) mbar_wait(&bar, 0, nullptr);
+        cluster.sync();
+        cluster.sync();
+        return;
+    }
+    trace_mark(a.trace, 1);  // weights in shared memory
+    // u = GELU(LN2(x) W1^T + b1) for this CTA's FFN rows
+    if (R > 0) project_rows<WT, MT>(w1, R, d, xr, red, u);
+    for (int o = tid; o < R * MT; o += NTHREADS) u[o] = gelu_erf(u[o] + (o < NTHREADS ? b1v[0] : b1v[1]));
+    __syncthreads();
+    trace_mark(a.trace, 2);  // u done
+    // partial u W2^T over all d columns (W2 stored transposed: row f = column f of W2)
+    for (int c = tid * 4; c < d; c += NTHREADS * 4) {
+        float acc[MT][4];
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[m][i] = 0.f;
+        for (int f = 0; f < R; ++f) {
+            float w4[4];
+            load4(w2 + (size_t)f * d + c, w4);
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                const float uf = u[f * MT + m];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[m][i] = fmaf(uf, w4[i], acc[m][i]);
+            }
+        }
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+            *reinterpret_cast<float4*>(ypart + (size_t)m * d + c) =
+                make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]);
+    }
+    trace_mark(a.trace, 3);  // partial outputs done
+    cluster.sync();
+    trace_mark(a.trace, 4);
+    // this CTA sums columns [rank * cols, +cols) over the cluster and adds them to the output
+#pragma unroll
+    for (int k = 0; k < RES_PER; ++k) {
+        const int i = tid + k * NTHREADS;
+        if (i >= MT * cols / 4) continue;
+        const int m = i / (cols / 4), c = rank * cols + (i % (cols / 4)) * 4;
+        if (!s_act[m]) continue;
+        float4 y = resv[k];
+#pragma unroll
+        for (int r = 0; r < CB; ++r) {
+            const float4 p = *reinterpret_cast<const float4*>(cluster.map_shared_rank(ypart, r) + (size_t)m * d + c);
+            y.x += p.x;
+            y.y += p.y;
+            y.z += p.z;
+            y.w += p.w;
+        }
+        atomicAdd(reinterpret_cast<float4*>(a.x_out + (size_t)m * d + c), y);
+    }
+    trace_mark(a.trace, 5);  // cluster sums added
+    cluster.sync();
+}
+
+template <typename T>
+cudaError_t set_smem(T kern, size_t bytes) {
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+template <typename WT, int MT>
+cudaError_t launch_attn_block_t(const LayerArgs& a, cudaStream_t s, bool pdl) {
+    const ALayout L(a.d, sizeof(WT), MT, a.page_size);
+    auto kern = attn_block_kernel<WT, MT>;
+    static size_t configured = 0;
+    if (configured < L.total) {
+        cudaError_t e = set_smem(kern, L.total);
+        if (e != cudaSuccess) return e;
+        configured = L.total;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(CA, a.n_heads);
+    cfg.blockDim = dim3(NTHREADS);
+    cfg.dynamicSmemBytes = L.total;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <typename WT, int MT>
+cudaError_t launch_mlp_t(const LayerArgs& a, int grid, cudaStream_t s, bool pdl) {
+    const BLayout L(a.d, a.ffn_rows_per_cta, sizeof(WT), MT, MLP_CLUSTER);
+    auto kern = mlp_kernel<WT, MT, MLP_CLUSTER>;
+    static size_t configured = 0;
+    if (configured < L.total) {
+        cudaError_t e = set_smem(kern, L.total);
+        if (e != cudaSuccess) return e;
+        configured = L.total;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(NTHREADS);
+    cfg.dynamicSmemBytes = L.total;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = MLP_CLUSTER;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <int MT>
+cudaError_t dispatch_layer(const LayerArgs& a, int which, bool bf, int grid, cudaStream_t s, bool pdl) {
+    if (which == 0) return bf ? launch_attn_block_t<__nv_bfloat16, MT>(a, s, pdl) : launch_attn_block_t<float, MT>(a, s, pdl);
+    return bf ? launch_mlp_t<__nv_bfloat16, MT>(a, grid, s, pdl) : launch_mlp_t<float, MT>(a, grid, s, pdl);
+}
+
+cudaError_t dispatch_rows(const LayerArgs& a, int which, bool bf, int grid, cudaStream_t s, bool pdl) {
+    if (a.M < 1 || a.M > MAX_ROWS) return cudaErrorInvalidValue;
+    if (a.M <= 1) return dispatch_layer<1>(a, which, bf, grid, s, pdl);
+    if (a.M <= 2) return dispatch_layer<2>(a, which, bf, grid, s, pdl);
+    if (a.M <= 4) return dispatch_layer<4>(a, which, bf, grid, s, pdl);
+    return dispatch_layer<8>(a, which, bf, grid, s, pdl);
+}
+
+}  // namespace
+
+size_t attn_block_smem_bytes(int d, int wbytes, int page) { return ALayout(d, wbytes, MAX_ROWS, page).total; }
+
+size_t mlp_smem_bytes(int d, int rows_per_cta, int wbytes) {
+    return BLayout(d, rows_per_cta, wbytes, MAX_ROWS, MLP_CLUSTER).total;
+}
+
+cudaError_t mlp_max_clusters(int d, int num_sms, int wbytes, int d_ffn, int* clusters) {
+    // the most clusters C of MLP_CLUSTER CTAs, each with ceil(d_ffn / (C * MLP_CLUSTER))
+    // FFN rows, that the GPU can hold at once
+    auto kern = wbytes == 2 ? mlp_kernel<__nv_bfloat16, MAX_ROWS, MLP_CLUSTER> : mlp_kernel<float, MAX_ROWS, MLP_CLUSTER>;
+    *clusters = 0;
+    for (int C = num_sms / MLP_CLUSTER; C >= 1; --C) {  // one CTA per SM at most
+        const int rpc = (d_ffn + C * MLP_CLUSTER - 1) / (C * MLP_CLUSTER);
+        const BLayout L(d, rpc, wbytes, MAX_ROWS, MLP_CLUSTER);
+        if (L.total > 200 * 1024) break;  // fewer clusters only need more shared memory
+        cudaError_t e = set_smem(kern, L.total);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(C * MLP_CLUSTER);
+        cfg.blockDim = dim3(NTHREADS);
+        cfg.dynamicSmemBytes = L.total;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = MLP_CLUSTER;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int fit = 0;
+        e = cudaOccupancyMaxActiveClusters(&fit, kern, &cfg);
+        if (e != cudaSuccess) return e;
+        if (fit >= C) {
+            *clusters = C;
+            return cudaSuccess;
+        }
+    }
+    return cudaSuccess;
+}
+
+cudaError_t launch_attn_block(const LayerArgs& a, bool w_bf16, cudaStream_t s, bool pdl) {
+    if (a.d % CA || a.d > 1024 || a.rows_per_group < 1 || a.page_size < 1) return cudaErrorInvalidValue;
+    return dispatch_rows(a, 0, w_bf16, 0, s, pdl);
+}
+
+cudaError_t launch_mlp(const LayerArgs& a, bool w_bf16, int grid, cudaStream_t s, bool pdl) {
+    if (a.d % (4 * MLP_CLUSTER) || a.d > 1024 || grid % MLP_CLUSTER) return cudaErrorInvalidValue;
+    return dispatch_rows(a, 1, w_bf16, grid, s, pdl);
+}
+
+}  // namespace mtp

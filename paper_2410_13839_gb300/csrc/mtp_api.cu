@@ -22,6 +22,7 @@
 #include <utility>
 #include <vector>
 
+#include "common.cuh"
 #include "kernels.cuh"
 #include "mtp.h"
 
@@ -82,7 +83,8 @@ struct mtp_ctx {
     cudaStream_t stream = nullptr;
     cudaStream_t cap_stream = nullptr;
     int device = 0, num_sms = 0, wbytes = 2;
-    bool use_graphs = true, use_pdl = true;
+    int mlp_clusters = 1;  // MLP clusters co-resident in one wave
+    bool use_graphs = true, use_pdl = true, use_l2_prefetch = true;
     std::vector<void*> allocs;
     // weights
     void* d_weights = nullptr;
@@ -103,12 +105,9 @@ struct mtp_ctx {
         *d_active = nullptr, *d_gen_count = nullptr, *d_gen_tokens = nullptr, *d_prompt = nullptr;
     float* d_h_last = nullptr;
     // step buffers
-    float *d_x = nullptr, *d_q = nullptr, *d_attn = nullptr, *d_u = nullptr, *d_logits = nullptr, *d_lse = nullptr,
-          *d_cand_logp = nullptr;
+    float *d_xb = nullptr, *d_logits = nullptr, *d_lse = nullptr, *d_cand_logp = nullptr;  // d_xb: 3 residual buffers
     int *d_row_seq = nullptr, *d_row_pos = nullptr, *d_row_last = nullptr, *d_cand_ids = nullptr, *d_path = nullptr,
         *d_out_tokens = nullptr, *d_out_accepted = nullptr;
-    float* d_ws = nullptr;
-    int* d_ws_count = nullptr;
     int* d_err = nullptr;
     std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;  // (n_heads, top_k, traced)
     std::map<std::tuple<int, int, int>, std::vector<int>> graph_kinds;
@@ -173,7 +172,7 @@ int gemv_grid(const mtp_ctx* c, int N, int K, int M, int* rpc) {
 unsigned long long* tslot(mtp_ctx* c, int kind) {
     if (!c->tracing || (int)c->trace_kinds.size() >= c->trace_cap) return nullptr;
     c->trace_kinds.push_back(kind);
-    return c->d_trace + 3 * (c->trace_kinds.size() - 1);
+    return c->d_trace + TRACE_WORDS * (c->trace_kinds.size() - 1);
 }
 
 GemvArgs gemv_base(mtp_ctx* c) {
@@ -187,71 +186,62 @@ GemvArgs gemv_base(mtp_ctx* c) {
     return a;
 }
 
-// The layer stack over the M rows currently in d_x (G groups of rpg rows).
+// Residual buffer of the rotation: in(l), mid(l) = in(l)+1, out(l) = in(l)+2 (mod 3),
+// with out(l) = in(l + 1).  Layer 0 reads buffer 0 (written by the embedding).
+float* xbuf(mtp_ctx* c, int i) { return c->d_xb + (size_t)(((i % 3) + 3) % 3) * MAX_ROWS * c->cfg.d_model; }
+int x_in_index(int l) { return (3 - l % 3) % 3; }
+
+// CTAs of the MLP kernel (clusters that are co-resident in one wave) and FFN rows per CTA.
+int mlp_grid(const mtp_ctx* c, int* rpc) {
+    const int ctas = std::max(1, c->mlp_clusters) * MLP_CLUSTER;
+    *rpc = (c->cfg.d_ffn + ctas - 1) / ctas;
+    const int used = (c->cfg.d_ffn + *rpc - 1) / *rpc;
+    return (used + MLP_CLUSTER - 1) / MLP_CLUSTER * MLP_CLUSTER;
+}
+
+// The block stack over the M rows the embedding put in buffer 0 (G groups of rpg
+// rows); returns the buffer holding the final hidden states.
 int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int val_seq, int val_old, int val_new,
-               int max_keys, cudaStream_t s, bool pdl, Prof* prof) {
+               cudaStream_t s, bool pdl, Prof* prof, float** final_x) {
+    (void)G;
     const mtp_config& cf = c->cfg;
-    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
+    const int d = cf.d_model, H = cf.n_attn_heads, P = cf.page_size;
     const bool bf = cf.weight_dtype == MTP_BF16;
-    const int S = attn_splits_for(G, H, P, max_keys, c->num_sms);
+    int rpc;
+    const int grid_b = mlp_grid(c, &rpc);
     for (int l = 0; l < cf.layers; ++l) {
         const Layer& L = c->layers[l];
-        const long long layer_off = (long long)l * 2 * H * P * HEAD_DIM;
-        int rpc, grid;
+        const int xi = x_in_index(l);
+        LayerArgs a;
+        std::memset(&a, 0, sizeof(a));
+        a.M = M; a.d = d; a.d_ffn = cf.d_ffn; a.n_heads = H; a.rows_per_group = rpg;
+        a.row_seq = c->d_row_seq; a.row_pos = c->d_row_pos; a.ln_eps = cf.ln_eps;
+        a.kv_pool = reinterpret_cast<__nv_bfloat16*>(c->d_kv); a.page_elems = c->page_elems;
+        a.layer_off = (long long)l * 2 * H * P * HEAD_DIM; a.page_size = P;
+        a.block_table = c->d_block_table; a.bt_stride = c->pages_per_seq;
+        a.plan = plan; a.seq_len = c->d_len; a.seq_new = c->d_npend; a.seq_base = seq_base;
+        a.val_seq = val_seq; a.val_old = val_old; a.val_new = val_new;
+        a.active = c->d_active; a.done = c->d_done; a.slots = cf.max_batch;
+        a.err = c->d_err;
+        const Layer* next = l + 1 < cf.layers && c->use_l2_prefetch ? &c->layers[l + 1] : nullptr;
 
-        GemvArgs q = gemv_base(c);
-        q.A = c->d_x; q.lda = d; q.ln_g = L.ln1_g; q.ln_b = L.ln1_b;
-        q.W = L.wqkv; q.bias = L.bqkv; q.N = 3 * d; q.K = d; q.M = M;
-        grid = gemv_grid(c, q.N, q.K, M, &rpc); q.rows_per_cta = rpc;
-        q.out = c->d_q; q.ldo = d;
-        q.kv_pool = c->d_kv; q.page_elems = c->page_elems; q.layer_off = layer_off;
-        q.n_heads = H; q.page_size = P; q.d_model = d;
-        q.block_table = c->d_block_table; q.bt_stride = c->pages_per_seq;
-        q.trace = tslot(c, MTP_K_QKV);
-        LAUNCH(MTP_K_QKV, launch_gemv(q, EPI_QKV, true, bf, grid, s, pdl));
+        LayerArgs at = a;
+        at.x_in = xbuf(c, xi); at.x_out = xbuf(c, xi + 1); at.x_zero = xbuf(c, xi + 2);
+        at.ln_g = L.ln1_g; at.ln_b = L.ln1_b;
+        at.wqkv = L.wqkv; at.bqkv = L.bqkv; at.wo = L.wo; at.bo = L.bo;
+        at.next_w_a = next ? next->wqkv : nullptr; at.next_w_b = next ? next->wo : nullptr;
+        at.trace = tslot(c, MTP_K_ATTN_BLOCK);
+        LAUNCH(MTP_K_ATTN_BLOCK, launch_attn_block(at, bf, s, pdl));
 
-        AttnArgs at;
-        std::memset(&at, 0, sizeof(at));
-        at.q = c->d_q; at.ldq = d;
-        at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(c->d_kv);
-        at.page_elems = c->page_elems; at.layer_off = layer_off;
-        at.block_table = c->d_block_table; at.bt_stride = c->pages_per_seq;
-        at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
-        at.out = c->d_attn; at.ldo = d;
-        at.ws_part = c->d_ws; at.ws_count = c->d_ws_count;
-        at.rows_per_group = rpg; at.n_heads = H; at.page_size = P; at.n_splits = S;
-        at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = seq_base;
-        at.val_seq = val_seq; at.val_old = val_old; at.val_new = val_new;
-        at.err = c->d_err;
-        at.trace = tslot(c, MTP_K_ATTN);
-        LAUNCH(MTP_K_ATTN, launch_attention(at, G, s, pdl));
-
-        GemvArgs o = gemv_base(c);
-        o.A = c->d_attn; o.lda = d; o.W = L.wo; o.bias = L.bo; o.N = d; o.K = d; o.M = M;
-        grid = gemv_grid(c, o.N, o.K, M, &rpc); o.rows_per_cta = rpc;
-        o.out = c->d_x; o.ldo = d;
-        o.trace = tslot(c, MTP_K_OPROJ);
-        LAUNCH(MTP_K_OPROJ, launch_gemv(o, EPI_RESID, false, bf, grid, s, pdl));
-
-        GemvArgs f1 = gemv_base(c);
-        f1.A = c->d_x; f1.lda = d; f1.ln_g = L.ln2_g; f1.ln_b = L.ln2_b;
-        f1.W = L.w1; f1.bias = L.b1; f1.N = F; f1.K = d; f1.M = M;
-        grid = gemv_grid(c, f1.N, f1.K, M, &rpc); f1.rows_per_cta = rpc;
-        f1.out = c->d_u; f1.ldo = F;
-        f1.trace = tslot(c, MTP_K_FFN1);
-        LAUNCH(MTP_K_FFN1, launch_gemv(f1, EPI_GELU, true, bf, grid, s, pdl));
-
-        GemvArgs f2 = gemv_base(c);
-        f2.A = c->d_u; f2.lda = F; f2.W = L.w2; f2.bias = L.b2; f2.N = d; f2.K = F; f2.M = M;
-        grid = gemv_grid(c, f2.N, f2.K, M, &rpc); f2.rows_per_cta = rpc;
-        f2.out = c->d_x; f2.ldo = d;
-        if (l == cf.layers - 1) {
-            f2.h_last = c->d_h_last;
-            f2.ld_h = d;
-        }
-        f2.trace = tslot(c, MTP_K_FFN2);
-        LAUNCH(MTP_K_FFN2, launch_gemv(f2, EPI_RESID, false, bf, grid, s, pdl));
+        LayerArgs mb = a;
+        mb.x_in = xbuf(c, xi + 1); mb.x_out = xbuf(c, xi + 2); mb.x_zero = xbuf(c, xi);
+        mb.ln_g = L.ln2_g; mb.ln_b = L.ln2_b;
+        mb.w1 = L.w1; mb.w2t = L.w2; mb.b1 = L.b1; mb.b2 = L.b2; mb.ffn_rows_per_cta = rpc;
+        mb.next_w_a = next ? next->w1 : nullptr; mb.next_w_b = next ? next->w2 : nullptr;
+        mb.trace = tslot(c, MTP_K_MLP);
+        LAUNCH(MTP_K_MLP, launch_mlp(mb, bf, grid_b, s, pdl));
     }
+    *final_x = xbuf(c, x_in_index(cf.layers - 1) + 2);
     return MTP_OK;
 }
 
@@ -262,7 +252,7 @@ EmbedArgs embed_base(mtp_ctx* c) {
     e.w_bf16 = c->cfg.weight_dtype == MTP_BF16;
     e.phone_vocab = c->cfg.phone_vocab; e.codec_vocab = c->cfg.codec_vocab;
     e.pe = c->d_pe; e.d = c->cfg.d_model; e.max_pos = c->cfg.max_ctx;
-    e.x = c->d_x; e.row_seq = c->d_row_seq; e.row_pos = c->d_row_pos; e.row_last = c->d_row_last;
+    e.x = xbuf(c, 0); e.zero_buf = xbuf(c, 1); e.row_seq = c->d_row_seq; e.row_pos = c->d_row_pos; e.row_last = c->d_row_last;
     e.n_max = c->cfg.n_heads_max; e.slots = c->cfg.max_batch;
     e.active = c->d_active; e.done = c->d_done; e.n_pending = c->d_npend; e.pending = c->d_pending;
     e.seq_len = c->d_len; e.prompt = c->d_prompt; e.prompt_stride = c->cfg.max_ctx;
@@ -270,8 +260,10 @@ EmbedArgs embed_base(mtp_ctx* c) {
     return e;
 }
 
-// Heads on h_last of slots [b0, b0 + m) -> logits rows of those slots.
-int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, cudaStream_t s, bool pdl, Prof* prof) {
+// Heads on the hidden states of slots [b0, b0 + m): rows of A, or, with
+// `gather`, the slot's last row fed this step in the single pass `gather`.
+int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, const float* gather, int b0,
+                 cudaStream_t s, bool pdl, Prof* prof) {
     const int d = c->cfg.d_model, V = c->cfg.codec_vocab;
     GemvArgs h = gemv_base(c);
     h.A = A; h.lda = d; h.ln_g = c->lnf_g; h.ln_b = c->lnf_b;
@@ -281,6 +273,9 @@ int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, cudaSt
     h.rows_per_cta = rpc;
     h.row_seq = nullptr;
     h.out = logits; h.ldo = n * V;
+    if (gather) {
+        h.gather_x = gather; h.gather_npend = c->d_npend; h.gather_n = n; h.gather_base = b0;
+    }
     h.trace = tslot(c, MTP_K_HEADS);
     LAUNCH(MTP_K_HEADS, launch_gemv(h, EPI_LOGITS, true, c->cfg.weight_dtype == MTP_BF16, grid, s, pdl));
     return MTP_OK;
@@ -303,17 +298,24 @@ SelectArgs select_base(mtp_ctx* c, int n, int k) {
 int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof) {
     const int B = c->cfg.max_batch, d = c->cfg.d_model, V = c->cfg.codec_vocab;
     const int spc = std::max(1, MAX_ROWS / n);
+    const bool single = B <= spc;  // one pass feeds every slot: the heads read its rows directly
+    float* final_x = nullptr;
     for (int b0 = 0; b0 < B; b0 += spc) {
         const int G = std::min(spc, B - b0), M = G * n;
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
         e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));  // full dependency on the previous pass
-        MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, c->cfg.max_ctx, s, pdl, prof));
+        MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
+        if (!single) {
+            unsigned long long* tr = tslot(c, MTP_K_SAVE);
+            LAUNCH(MTP_K_SAVE, launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, d, tr, s, pdl));
+        }
     }
     for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
         const int m = std::min(MAX_ROWS, B - b0);
-        MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, s, pdl, prof));
+        MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V,
+                             single ? final_x : nullptr, b0, s, pdl, prof));
     }
     SelectArgs sa = select_base(c, n, k);
     sa.trace = tslot(c, MTP_K_SELECT);
@@ -387,8 +389,8 @@ int read_slot_ints(mtp_ctx* c, const int* dptr, std::vector<int>& out) {
 
 int validate_config(const mtp_config& c) {
     if (c.layers < 1 || c.layers > 256) return fail(MTP_ERR_INVALID, "layers %d out of range", c.layers);
-    if (c.d_model < 256 || c.d_model % 256 || c.d_model > 4096)
-        return fail(MTP_ERR_INVALID, "d_model %d: need a multiple of 256 up to 4096", c.d_model);
+    if (c.d_model < 256 || c.d_model % 256 || c.d_model > 1024)
+        return fail(MTP_ERR_INVALID, "d_model %d: need a multiple of 256 up to 1024", c.d_model);
     if (c.n_attn_heads * HEAD_DIM != c.d_model)
         return fail(MTP_ERR_INVALID, "d_model / n_attn_heads must be %d", HEAD_DIM);
     if (c.d_ffn < 256 || c.d_ffn % 256 || c.d_ffn > 4096)
@@ -438,6 +440,30 @@ std::vector<TensorSpec> blob_specs(const mtp_config& c) {
     return t;
 }
 
+// Device layouts of a block's matrices (element size es bytes):
+//   j = 2  wqkv [3d][d]  -> head-major [H][q 64 | k 64 | v 64][d]
+//   j = 3  bqkv [3d]     -> head-major [H][192]
+//   j = 4  wo   [d][d]   -> [H][d][64]: head h's input columns of every output row
+//   j = 10 w2   [d][F]   -> transposed [F][d]
+void relayout(const mtp_config& cf, int j, int es, const unsigned char* src, unsigned char* dst) {
+    const size_t d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads;
+    if (j == 2 || j == 3) {
+        const size_t row = (j == 2 ? d : 1) * es;
+        for (size_t h = 0; h < H; ++h)
+            for (size_t r = 0; r < 3 * HEAD_DIM; ++r) {
+                const size_t sec = r / HEAD_DIM, within = r % HEAD_DIM;
+                std::memcpy(dst + (h * 3 * HEAD_DIM + r) * row, src + (sec * d + h * HEAD_DIM + within) * row, row);
+            }
+    } else if (j == 4) {
+        for (size_t h = 0; h < H; ++h)
+            for (size_t f = 0; f < d; ++f)
+                std::memcpy(dst + ((h * d + f) * HEAD_DIM) * es, src + (f * d + h * HEAD_DIM) * es, HEAD_DIM * es);
+    } else {
+        for (size_t c = 0; c < d; ++c)
+            for (size_t f = 0; f < F; ++f) std::memcpy(dst + (f * d + c) * es, src + (c * F + f) * es, es);
+    }
+}
+
 int upload_weights(mtp_ctx* c, const void* blob, size_t bytes) {
     const mtp_config& cf = c->cfg;
     const unsigned char* b = static_cast<const unsigned char*>(blob);
@@ -467,11 +493,19 @@ int upload_weights(mtp_ctx* c, const void* blob, size_t bytes) {
     unsigned char* dw = nullptr;
     MTP_TRY(c->alloc(&dw, total));
     c->d_weights = dw;
+    std::vector<unsigned char> tmp;
     for (uint32_t i = 0; i < n_t; ++i) {
         uint64_t off, nb;
         std::memcpy(&off, b + 24 + 16 * i, 8);
         std::memcpy(&nb, b + 24 + 16 * i + 8, 8);
-        CUDA_TRY(cudaMemcpy(dw + dev_off[i], b + off, nb, cudaMemcpyHostToDevice));
+        const unsigned char* src = b + off;
+        const int j = i >= 2 && i < 2 + 12u * cf.layers ? (int)((i - 2) % 12) : -1;
+        if (j == 2 || j == 3 || j == 4 || j == 10) {  // device layouts of the fused block kernels
+            tmp.resize(nb);
+            relayout(cf, j, j == 3 ? 4 : c->wbytes, src, tmp.data());
+            src = tmp.data();
+        }
+        CUDA_TRY(cudaMemcpy(dw + dev_off[i], src, nb, cudaMemcpyHostToDevice));
     }
     size_t i = 0;
     auto nxt = [&]() { return static_cast<const void*>(dw + dev_off[i++]); };
@@ -565,16 +599,24 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
     c->pages_per_seq = (cf.max_ctx + P - 1) / P;
     c->n_pages = cf.n_pages > 0 ? cf.n_pages : B * c->pages_per_seq;
     c->page_elems = (long long)cf.layers * 2 * H * P * HEAD_DIM;
-    // projection slices must fit shared memory
-    const int proj[5][2] = {{3 * d, d}, {d, d}, {F, d}, {d, F}, {nm * V, d}};
-    for (const auto& pk : proj) {
+    // the fused block kernels' shared memory; MLP clusters that fit one wave
+    {
+        int clusters = 0;
+        if (mlp_max_clusters(d, c->num_sms, c->wbytes, cf.d_ffn, &clusters) != cudaSuccess || clusters < 1) {
+            cudaGetLastError();
+            clusters = std::max(1, c->num_sms / MLP_CLUSTER / 2);
+        }
+        c->mlp_clusters = std::min(clusters, std::max(1, c->num_sms / MLP_CLUSTER));
         int rpc;
-        gemv_grid(c, pk[0], pk[1], MAX_ROWS, &rpc);
-        if (gemv_smem_bytes(rpc, pk[1], c->wbytes, MAX_ROWS) > 200 * 1024)
-            return bail(fail(MTP_ERR_INVALID, "projection %d x %d does not fit shared memory", pk[0], pk[1]));
+        mlp_grid(c, &rpc);
+        const size_t sa = attn_block_smem_bytes(d, c->wbytes, P), sb = mlp_smem_bytes(d, rpc, c->wbytes);
+        int hrpc;
+        gemv_grid(c, nm * V, d, MAX_ROWS, &hrpc);
+        const size_t sh = gemv_smem_bytes(hrpc, d, c->wbytes, MAX_ROWS);
+        if (sa > 200 * 1024 || sb > 200 * 1024 || sh > 200 * 1024)
+            return bail(fail(MTP_ERR_INVALID, "model too wide for the shared-memory plan (%zu, %zu, %zu bytes)", sa,
+                             sb, sh));
     }
-    const int S_max = std::max(1, c->num_sms / H) + 1;
-    const size_t ws_floats = attn_workspace_floats(MAX_ROWS, H, S_max, MAX_ROWS);
     const int lb = std::max(B, MAX_ROWS);
     if ((r = c->alloc(&c->d_pe, (size_t)cf.max_ctx * d)) ||
         (r = c->alloc(&c->d_kv, (size_t)c->n_pages * c->page_elems)) ||
@@ -584,15 +626,13 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_done, B)) || (r = c->alloc(&c->d_active, B)) || (r = c->alloc(&c->d_gen_count, B)) ||
         (r = c->alloc(&c->d_gen_tokens, (size_t)B * cf.max_ctx)) ||
         (r = c->alloc(&c->d_prompt, (size_t)B * cf.max_ctx)) || (r = c->alloc(&c->d_h_last, (size_t)lb * d)) ||
-        (r = c->alloc(&c->d_x, (size_t)MAX_ROWS * d)) || (r = c->alloc(&c->d_q, (size_t)MAX_ROWS * d)) ||
-        (r = c->alloc(&c->d_attn, (size_t)MAX_ROWS * d)) || (r = c->alloc(&c->d_u, (size_t)MAX_ROWS * F)) ||
+        (r = c->alloc(&c->d_xb, (size_t)3 * MAX_ROWS * d)) ||
         (r = c->alloc(&c->d_logits, (size_t)lb * nm * V)) || (r = c->alloc(&c->d_lse, (size_t)lb * nm)) ||
         (r = c->alloc(&c->d_cand_logp, (size_t)lb * nm * MAX_TOPK)) ||
         (r = c->alloc(&c->d_cand_ids, (size_t)lb * nm * MAX_TOPK)) || (r = c->alloc(&c->d_path, (size_t)lb * nm)) ||
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
         (r = c->alloc(&c->d_row_seq, MAX_ROWS)) || (r = c->alloc(&c->d_row_pos, MAX_ROWS)) ||
-        (r = c->alloc(&c->d_row_last, MAX_ROWS)) || (r = c->alloc(&c->d_ws, ws_floats)) ||
-        (r = c->alloc(&c->d_ws_count, (size_t)MAX_ROWS * H)) || (r = c->alloc(&c->d_err, 1)))
+        (r = c->alloc(&c->d_row_last, MAX_ROWS)) || (r = c->alloc(&c->d_err, 1)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
     if (cudaMemcpy(c->d_block_table, c->h_block_table.data(), c->h_block_table.size() * sizeof(int),
@@ -616,16 +656,48 @@ MTP_API void mtp_destroy(mtp_ctx* ctx) {
 MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
     g_err.clear();
     MTP_TRY(check_ctx(c));
+    bool changed = false;
     if (option == MTP_OPT_GRAPHS) {
         c->use_graphs = value != 0;
     } else if (option == MTP_OPT_PDL) {
-        if (c->use_pdl != (value != 0)) {
-            for (auto& g : c->graphs) cudaGraphExecDestroy(g.second);
-            c->graphs.clear();
-        }
+        changed = c->use_pdl != (value != 0);
         c->use_pdl = value != 0;
+    } else if (option == MTP_OPT_L2_PREFETCH) {
+        changed = c->use_l2_prefetch != (value != 0);
+        c->use_l2_prefetch = value != 0;
+    } else if (option == MTP_OPT_MLP_CLUSTERS) {
+        if (value < 1 || value > std::max(1, 2 * c->num_sms / MLP_CLUSTER))
+            return fail(MTP_ERR_INVALID, "MLP clusters %d out of range", value);
+        int rpc;
+        const int keep = c->mlp_clusters;
+        c->mlp_clusters = value;
+        mlp_grid(c, &rpc);
+        if (mlp_smem_bytes(c->cfg.d_model, rpc, c->wbytes) > 200 * 1024) {
+            c->mlp_clusters = keep;
+            return fail(MTP_ERR_INVALID, "%d MLP clusters need too much shared memory", value);
+        }
+        changed = keep != value;
     } else {
         return fail(MTP_ERR_INVALID, "unknown option %d", option);
+    }
+    if (changed) {  // captured steps bake these in
+        for (auto& g : c->graphs) cudaGraphExecDestroy(g.second);
+        c->graphs.clear();
+        c->graph_kinds.clear();
+    }
+    return MTP_OK;
+}
+
+MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (!value) return fail(MTP_ERR_INVALID, "null output");
+    switch (option) {
+        case MTP_OPT_GRAPHS: *value = c->use_graphs; break;
+        case MTP_OPT_PDL: *value = c->use_pdl; break;
+        case MTP_OPT_L2_PREFETCH: *value = c->use_l2_prefetch; break;
+        case MTP_OPT_MLP_CLUSTERS: *value = c->mlp_clusters; break;
+        default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;
 }
@@ -673,13 +745,16 @@ MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph,
     if (n_ac) CUDA_TRY(cudaMemcpyAsync(prompt + n_ph, acoustic, n_ac * sizeof(int), cudaMemcpyDefault, s));
     MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0));
     Prof* prof = nullptr;
+    float* final_x = nullptr;
     for (int p0 = 0; p0 < T; p0 += MAX_ROWS) {
         const int m = (int)std::min<long long>(MAX_ROWS, T - p0);
         EmbedArgs e = embed_base(c);
         e.mode = 1; e.rows = m; e.slot = slot; e.p0 = p0; e.n_ph = n_ph; e.total = (int)T;
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
-        MTP_TRY(run_layers(c, m, 1, m, PLAN_VALUE, 0, slot, p0, m, p0 + m, s, c->use_pdl, prof));
+        MTP_TRY(run_layers(c, m, 1, m, PLAN_VALUE, 0, slot, p0, m, s, c->use_pdl, prof, &final_x));
     }
+    LAUNCH(MTP_K_SAVE, launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, nullptr, s,
+                                        c->use_pdl));
     MTP_TRY(slot_set(c, slot, (int)T, -1, -1, -1, -1, -1));
     // pageable host prompts: copies above are complete when the call returns
     return MTP_OK;
@@ -834,21 +909,21 @@ MTP_API int mtp_trace_step(mtp_ctx* c, int n, int k, int64_t* out, int cap) {
     if (!out || cap < 1) return fail(MTP_ERR_INVALID, "trace: null output or capacity < 1");
     if (!c->d_trace) {
         c->trace_cap = 4096;
-        MTP_TRY(c->alloc(&c->d_trace, (size_t)3 * c->trace_cap));
+        MTP_TRY(c->alloc(&c->d_trace, (size_t)TRACE_WORDS * c->trace_cap));
     }
     CUDA_TRY(launch_trace_reset(c->d_trace, c->trace_cap, c->stream));
     c->tracing = true;
     const int r = run_step(c, n, k);
     c->tracing = false;
     MTP_TRY(r);
-    std::vector<unsigned long long> h(3 * (size_t)c->trace_cap);
+    std::vector<unsigned long long> h(TRACE_WORDS * (size_t)c->trace_cap);
     CUDA_TRY(cudaMemcpyAsync(h.data(), c->d_trace, h.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost,
                              c->stream));
     MTP_TRY(check_device_error(c));
     const int count = std::min<int>((int)c->trace_kinds.size(), cap);
     for (int i = 0; i < count; ++i) {
-        out[4 * i] = c->trace_kinds[i];
-        for (int j = 0; j < 3; ++j) out[4 * i + 1 + j] = (int64_t)h[3 * i + j];
+        out[(TRACE_WORDS + 1) * i] = c->trace_kinds[i];
+        for (int j = 0; j < TRACE_WORDS; ++j) out[(TRACE_WORDS + 1) * i + 1 + j] = (int64_t)h[(size_t)TRACE_WORDS * i + j];
     }
     return count;
 }
@@ -908,9 +983,9 @@ MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden
         const int m = std::min(MAX_ROWS, batch - b0);
         const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
         CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,
-                                     hidden_dtype == MTP_BF16, c->d_x, m, d, s));
+                                     hidden_dtype == MTP_BF16, xbuf(c, 0), m, d, s));
         float* logits = out_logits ? out_logits + (size_t)b0 * n * V : c->d_logits;
-        MTP_TRY(launch_heads(c, c->d_x, m, n, logits, s, false, prof));
+        MTP_TRY(launch_heads(c, xbuf(c, 0), m, n, logits, nullptr, 0, s, false, prof));
         SelectArgs sa = select_base(c, n, k);
         sa.logits = logits;
         sa.lse = out_lse ? out_lse + (size_t)b0 * n : c->d_lse;

@@ -146,6 +146,12 @@ def mtp_set_option(ctx: int, option: int, value: int) -> None:
     check(lib.mtp_set_option(ctx, option, value))
 
 
+def mtp_get_option(ctx: int, option: int) -> int:
+    out = ctypes.c_int32()
+    check(lib.mtp_get_option(ctx, option, ctypes.byref(out)))
+    return int(out.value)
+
+
 def mtp_profile_step(ctx: int, n_heads: int, top_k: int) -> dict:
     ms = np.zeros(len(_lib.KERNEL_KINDS), np.float32)
     launches = np.zeros(len(_lib.KERNEL_KINDS), np.int32)
@@ -154,8 +160,8 @@ def mtp_profile_step(ctx: int, n_heads: int, top_k: int) -> dict:
 
 
 def mtp_trace_step(ctx: int, n_heads: int, top_k: int, cap: int = 4096) -> np.ndarray:
-    """Timeline of one decode step: rows (kind, start_ns, wait_ns, end_ns)."""
-    out = np.zeros((cap, 4), np.int64)
+    """Timeline of one decode step: rows (kind, start_ns, wait_ns, end_ns, 8 phase marks)."""
+    out = np.zeros((cap, 12), np.int64)
     count = check(lib.mtp_trace_step(ctx, n_heads, top_k, _ptr(out), cap))
     return out[:count]
 

@@ -112,7 +112,14 @@ def test_n1_is_greedy_on_gpu_scores():
         dec.close()
 
 
-def test_rollback_then_append_is_bit_exact():
+# The block kernels add residual contributions from many CTAs with float
+# atomics, so two runs of the same step may differ in the last bits; the
+# cache-bookkeeping checks below therefore compare to 1e-5 (a wrong page,
+# position or length moves logits by O(0.1)).
+REPEAT_ATOL = 1e-5
+
+
+def test_rollback_then_append():
     """append(A); rollback(|A|); append(C) gives the logits of append(C) on a fresh cache."""
     mtp = lib_module()
     ph, ac = synth.make_prompt(3, 12, 30, synth.TINY.phone_vocab)
@@ -129,7 +136,7 @@ def test_rollback_then_append_is_bit_exact():
         mtp.mtp_set_teacher_tokens(dec.ctx, 0, a_toks[0])   # A again: same logits
         dec.decode_step(4, 4)
         lg_a2, _ = dec.logits(4)
-        assert np.array_equal(lg_a, lg_a2)
+        assert np.abs(lg_a - lg_a2).max() <= REPEAT_ATOL
         c = np.array([7, 1000, 3, 512], np.int32)
         mtp.mtp_rollback(dec.ctx, 0, 4)
         mtp.mtp_set_teacher_tokens(dec.ctx, 0, c)
@@ -140,13 +147,13 @@ def test_rollback_then_append_is_bit_exact():
         mtp.mtp_set_teacher_tokens(ref.ctx, 0, c)
         ref.decode_step(4, 4)
         lg_ref, _ = ref.logits(4)
-        assert np.array_equal(lg_c, lg_ref)
+        assert np.abs(lg_c - lg_ref).max() <= REPEAT_ATOL
     finally:
         dec.close()
         ref.close()
 
 
-def test_page_placement_is_bit_exact():
+def test_page_placement():
     """The same sequence on other physical pages gives identical logits."""
     ph, ac = synth.make_prompt(4, 12, 40, synth.TINY.phone_vocab)
     other_ph, other_ac = synth.make_prompt(9, 30, 60, synth.TINY.phone_vocab)
@@ -168,7 +175,7 @@ def test_page_placement_is_bit_exact():
         finally:
             dec.close()
     for a, b in zip(out[0], out[1]):
-        assert np.array_equal(a, b)
+        assert np.abs(a - b).max() <= REPEAT_ATOL
 
 
 def test_eos_finishes_a_slot():
