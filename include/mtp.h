@@ -280,6 +280,26 @@ MTP_API size_t mtp_attention_workspace_bytes(const mtp_attention_args* args);
 MTP_API int mtp_attention(const mtp_attention_args* args, void* workspace, size_t workspace_bytes,
                           void* cuda_stream);
 
+/* mtp_attention without a caller workspace and without any allocation.  The
+ * paper has no counterpart: this serves callers that must not allocate GPU
+ * memory while they run -- for instance a real-time audio callback, where
+ * cudaMalloc/cudaFree may block on the driver or synchronise the device and
+ * so stall playback, or a host application that owns every byte of GPU
+ * memory and hands none to the library.
+ * The split-merge scratch lives in one fixed device array of
+ * MTP_ATTENTION_NOALLOC_SCRATCH_BYTES per GPU, held from library load until
+ * process exit and shared by every call on that GPU.  A call whose scratch
+ * need (mtp_attention_workspace_bytes) exceeds it fails with MTP_ERR_INVALID
+ * before launching anything.  The first call on a device looks up the
+ * array's device address; make that first call before any stream capture.
+ * Each call clears the merge counters it uses (an asynchronous memset on the
+ * stream); the partial results keep the last call's contents.  Calls that
+ * overlap on the GPU (other streams or threads) race on the array: order
+ * them on one stream.  Arguments, outputs and errors as mtp_attention.  No
+ * cudaMalloc, cudaFree or allocating library call is made. */
+#define MTP_ATTENTION_NOALLOC_SCRATCH_BYTES (4u << 20)
+MTP_API int mtp_attention_noalloc(const mtp_attention_args* args, void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -74,6 +74,7 @@ def _load() -> ctypes.CDLL:
         "mtp_heads_topk": (i32, [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]),
         "mtp_attention_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),
         "mtp_attention": (i32, [ctypes.POINTER(MtpAttentionArgs), vp, sz, vp]),
+        "mtp_attention_noalloc": (i32, [ctypes.POINTER(MtpAttentionArgs), vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

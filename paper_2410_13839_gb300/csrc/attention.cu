@@ -14,8 +14,12 @@
 // the pages touched by this step's appends are read after it.
 #include <math.h>
 
+#include <cstdio>
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
+#include "mtp.h"
 
 namespace mtp {
 namespace {
@@ -337,3 +341,71 @@ cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool
 }
 
 }  // namespace mtp
+
+// ---- allocation-free attention (mtp_attention_noalloc) ----------------------
+// For callers that may not allocate GPU memory while they run (a real-time
+// audio callback, where cudaMalloc/cudaFree can block or synchronise the
+// device; a host that owns all GPU memory): the split-merge scratch of the
+// attention kernel is this fixed array, one per GPU that loads the library,
+// held until the process exits and shared by every call on that GPU.
+static __device__ __align__(256) unsigned char g_attention_scratch[MTP_ATTENTION_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  The array's
+// name is only a host-side stand-in, so the address is looked up once per
+// device (with that device current) and remembered.
+int scratch_address(void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
+    if (dev < 0 || dev >= kMaxDevices) return mtp::report_error(MTP_ERR_INVALID, "device index out of range");
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    if (!g_scratch_addr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_attention_scratch);
+        if (e != cudaSuccess || !p) {
+            char msg[256];
+            std::snprintf(msg, sizeof(msg), "attention scratch address lookup failed: %s", cudaGetErrorString(e));
+            return mtp::report_error(MTP_ERR_CUDA, msg);
+        }
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return MTP_OK;
+}
+
+}  // namespace
+
+extern "C" MTP_API int mtp_attention_noalloc(const mtp_attention_args* args, void* cuda_stream) {
+    mtp::clear_error();
+    if (!args) return mtp::report_error(MTP_ERR_INVALID, "attention: null arguments");
+    const size_t need = mtp_attention_workspace_bytes(args);
+    if (need == 0) return mtp::report_error(MTP_ERR_INVALID, "attention: invalid sizes");
+    if (need > MTP_ATTENTION_NOALLOC_SCRATCH_BYTES) {
+        char msg[256];
+        std::snprintf(msg, sizeof(msg),
+                      "attention: this call needs %zu bytes of scratch, the fixed scratch array holds %u", need,
+                      (unsigned)MTP_ATTENTION_NOALLOC_SCRATCH_BYTES);
+        return mtp::report_error(MTP_ERR_INVALID, msg);
+    }
+    void* scratch = nullptr;
+    const int r = scratch_address(&scratch);
+    if (r != MTP_OK) return r;
+    // the merge counters follow the 256-byte-aligned partials and must start at zero
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
+    const int groups = (args->rows + args->rows_per_group - 1) / args->rows_per_group;
+    const int splits = mtp::attn_splits_for(groups, args->n_heads, args->page_size, args->max_keys, sms);
+    const size_t part = (mtp::attn_workspace_floats(groups, args->n_heads, splits, args->rows_per_group) * 4 + 255) &
+                        ~(size_t)255;
+    e = cudaMemsetAsync(static_cast<char*>(scratch) + part, 0, need - part, static_cast<cudaStream_t>(cuda_stream));
+    if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
+    return mtp_attention(args, scratch, MTP_ATTENTION_NOALLOC_SCRATCH_BYTES, cuda_stream);
+}

@@ -179,4 +179,8 @@ cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStrea
 cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
                              unsigned long long* trace, cudaStream_t s, bool pdl);
 
+// C-ABI error reporting shared by the translation units (message for mtp_last_error)
+int report_error(int code, const char* msg);
+void clear_error();
+
 }  // namespace mtp

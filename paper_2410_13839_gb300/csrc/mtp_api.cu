@@ -42,6 +42,17 @@ int fail(int code, const char* fmt, ...) {
     return code;
 }
 
+}  // namespace
+
+// error reporting for C-ABI functions defined in other translation units
+int mtp::report_error(int code, const char* msg) {
+    g_err = msg;
+    return code;
+}
+void mtp::clear_error() { g_err.clear(); }
+
+namespace {
+
 #define CUDA_TRY(expr)                                                                                  \
     do {                                                                                                \
         cudaError_t e_ = (expr);                                                                        \

@@ -201,6 +201,11 @@ def mtp_attention(args: MtpAttentionArgs, workspace, workspace_bytes: int, strea
     check(lib.mtp_attention(ctypes.byref(args), _ptr(workspace), workspace_bytes, _stream_handle(stream)))
 
 
+def mtp_attention_noalloc(args: MtpAttentionArgs, stream=None) -> None:
+    """mtp_attention with the library's fixed scratch array: no workspace, no allocation."""
+    check(lib.mtp_attention_noalloc(ctypes.byref(args), _stream_handle(stream)))
+
+
 def _as_i32(x):
     if x is None:
         return None
