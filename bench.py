@@ -60,6 +60,21 @@ def _dist():
     return world, rank, local
 
 
+def max_over_ranks(x: float, dist=None, device="cuda") -> float:
+    """The largest x over all ranks (the slowest rank's time); x itself on one rank."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(world: int, steps: int, seconds: float) -> float:
+    """Whole-job throughput: every rank's generated tokens over the slowest rank's time."""
+    return world * steps * GEN * BATCH / seconds
+
+
 def _kernel_bytes(d, F, V, L, n, wb, ctx_keys, fed):
     """Algorithmic bytes per launch of each kernel class (weights + parameters; keys/values)."""
     return {
@@ -252,11 +267,8 @@ def run_ours(args):
     assert tokens_done == GEN, f"generation stopped at {tokens_done} tokens"
     prefill_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     decode_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * args.steps * GEN * BATCH / (ms / 1e3)
+    ms = max_over_ranks(ms, dist)
+    value = job_tokens_per_s(world, args.steps, ms / 1e3)
 
     # end to end through the public API with host buffers (pinned), copies inside the timed region
     ph_h = torch.from_numpy(ph).pin_memory()
@@ -270,11 +282,8 @@ def run_ours(args):
         mtp.mtp_generate(ctx, N_HEADS, TOP_K, out_h, GEN, lens_h)
     barrier()
     e2e_s = time.perf_counter() - t0
-    if dist:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e = {"value": world * args.steps * GEN * BATCH / e2e_s, "unit": "codec tokens/s",
+    e2e_s = max_over_ranks(e2e_s, dist)
+    e2e = {"value": job_tokens_per_s(world, args.steps, e2e_s), "unit": "codec tokens/s",
            "h2d_bytes_per_step": (N_PH + N_AC) * 4, "d2h_bytes_per_step": BATCH * GEN * 4 + BATCH * 4}
 
     # per-kernel durations: one eager step mid-generation, events around every launch

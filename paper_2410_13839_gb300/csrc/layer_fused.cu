@@ -48,45 +48,148 @@ __host__ __device__ inline size_t al128(size_t x) { return (x + 127) & ~(size_t)
 
 // ---- shared-memory layouts (host and device compute the same offsets) ----
 struct ALayout {
-    size_t wqkv, wo, ks, vs, qkvp, qkvf, qs, sc, part, attn, red, res, total;
+    size_t wqkv, wo, ks, qkvp, qkvf, qs, part, attn, res, uni, total;
+    size_t xb, accs, red, sc, pvred, attn_b, ytile;  // inside the union (phases do not overlap)
     int tile;       // keys of the dedicated staging slots
     int sc_stride;  // keys per batch (dedicated and reused slots)
     __host__ __device__ ALayout(int d, int wbytes, int mt, int page) {
         const int groups = (QROWS * mt + 31) / 32;
         tile = (MIN_TILE + page - 1) / page * page;  // whole pages, at least MIN_TILE keys
-        const int ATT_TILE = tile;
         wqkv = 0;
         wo = al128(wqkv + (size_t)QROWS * d * wbytes);
         ks = al128(wo + (size_t)(d / CA) * HEAD_DIM * wbytes);  // page slots: [keys | values] each
-        vs = ks;
-        qkvp = al128(ks + (size_t)2 * ATT_TILE * HEAD_DIM * 2);
-        qkvf = al128(qkvp + (size_t)QROWS * mt * 4);
+        qkvp = al128(ks + (size_t)2 * tile * HEAD_DIM * 2);
+        res = al128(qkvp + (size_t)QROWS * mt * 4);
+        qkvf = al128(res + (size_t)mt * (d / CA) * 4);
         qs = al128(qkvf + (size_t)3 * HEAD_DIM * mt * 4);
-        sc = al128(qs + (size_t)mt * HEAD_DIM * 4);
-        sc_stride = (ATT_TILE / page + (QROWS * d * wbytes) / (4 * page * HEAD_DIM)) * page;  // keys per batch
-        part = al128(sc + (size_t)mt * sc_stride * 4);
+        part = al128(qs + (size_t)mt * HEAD_DIM * 4);
         attn = al128(part + (size_t)mt * PARTW * 4);
-        red = al128(attn + (size_t)mt * HEAD_DIM * 4);
-        res = al128(red + (size_t)NWARPS * groups * 32 * 4);
-        total = al128(res + (size_t)mt * (d / CA) * 4);
+        uni = al128(attn + (size_t)mt * HEAD_DIM * 4);
+        sc_stride = (tile / page + (QROWS * d * wbytes) / (4 * page * HEAD_DIM)) * page;  // keys per batch
+        // projection: bf16 inputs + tile sums (tensor cores) or the reduce-scatter scratch (fp32);
+        // qkvf, qs, part and attn are written only after the projection, so it may start there
+        xb = qkvf;
+        accs = al128(xb + (size_t)mt * (d + 8) * 2);
+        red = al128(accs + (size_t)QROWS * 8 * 4);
+        const size_t p1 = wbytes == 2 ? red : red + (size_t)NWARPS * groups * 32 * 4;
+        // attention: scores, per-warp P.V partials
+        sc = uni;
+        pvred = al128(sc + (size_t)mt * sc_stride * 4);
+        const size_t p2 = pvred + (size_t)NWARPS * HEAD_DIM * 4;
+        // output projection: bf16 head output, projected rows
+        attn_b = uni;
+        ytile = al128(attn_b + (size_t)mt * (HEAD_DIM + 8) * 2);
+        const size_t p3 = ytile + (size_t)mt * (d / CA) * 4;
+        total = al128(p1 > p2 ? (p1 > p3 ? p1 : p3) : (p2 > p3 ? p2 : p3));
     }
 };
 
 struct BLayout {
-    size_t w1, w2, u, ypart, red, total;
+    size_t w1, w2, xb, accs, ub, u, red, ypart, total;
+    int rpad;  // FFN rows rounded up to the 16-row MMA step
     __host__ __device__ BLayout(int d, int rows, int wbytes, int mt, int cb) {
         (void)cb;
         const int groups = (rows * mt + 31) / 32;
+        rpad = (rows + 15) / 16 * 16;
         w1 = 0;
         w2 = al128(w1 + (size_t)rows * d * wbytes);
-        u = al128(w2 + (size_t)rows * d * wbytes);
+        xb = al128(w2 + (size_t)rows * d * wbytes);
+        accs = al128(xb + (size_t)mt * (d + 8) * 2);
+        ub = al128(accs + (size_t)rows * 8 * 4);
+        u = al128(ub + (size_t)mt * (rpad + 8) * 2);
+        red = al128(u + (wbytes == 2 ? 0 : (size_t)rows * mt * 4));
+        size_t end = al128(red + (wbytes == 2 ? 0 : (size_t)NWARPS * groups * 32 * 4));
         const size_t ybytes = (size_t)mt * d * 4;
         // the partial outputs reuse W1's space once u is known, when it fits
-        ypart = ((size_t)rows * d * wbytes >= ybytes) ? w1 : al128(u + (size_t)rows * mt * 4);
-        red = al128((ypart == w1 ? u + (size_t)rows * mt * 4 : ypart + ybytes));
-        total = al128(red + (size_t)NWARPS * groups * 32 * 4);
+        if ((size_t)rows * d * wbytes >= ybytes) {
+            ypart = w1;
+        } else {
+            ypart = end;
+            end = al128(end + ybytes);
+        }
+        total = end;
     }
 };
+
+// ---- tensor-core building blocks (mma.sync m16n8k16, bf16 in, fp32 accumulate) ----
+// Fed rows are at most 8 tokens: they are the N = 8 side of the MMA and the
+// weight rows the M = 16 side, so no token padding beyond 8 is needed.
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t (&r)[2], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// Shared address of 16-byte chunk `chunk` of weight row `row` (row_bytes each):
+// the weights are stored with chunk c of global row g at position c ^ (g & 7)
+// (made at create), which keeps ldmatrix free of bank conflicts.
+__device__ __forceinline__ uint32_t wchunk(uint32_t base, int row, int row_bytes, int chunk, int key) {
+    return base + (uint32_t)row * row_bytes + ((uint32_t)(chunk ^ (key & 7)) << 4);
+}
+
+// accs[row][n] += sum_k W[row][k] x[n][k] for the R (<= 64) rows of a weight
+// slice in shared memory (rows keyed key0 + row), K split across the 8 warps;
+// each warp adds its tile sums into accs (zeroed beforehand) with shared atomics.
+template <int MT>
+__device__ __forceinline__ void mma_rows_ksplit(const void* w, int R, int K, int key0, const __nv_bfloat16* xb,
+                                                float* accs) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int tiles = (R + 15) / 16;
+    const int kslice = K / NWARPS;
+    const uint32_t wb = smem_addr(w), xbase = smem_addr(xb);
+    const int xstride = (K + 8) * 2, row_bytes = K * 2;
+    const int brow = (lane & 7) < MT ? (lane & 7) : 0;  // tokens past MT repeat token 0 (ignored)
+    const int bhalf = (lane >> 3) & 1;
+    const int arow = lane & 15, ahalf = lane >> 4;
+    float acc[4][4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[t][i] = 0.f;
+    for (int k0 = warp * kslice; k0 < (warp + 1) * kslice; k0 += 16) {
+        uint32_t b[2];
+        ldsm_x2(b, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            if (t < tiles) {
+                const int row = min(t * 16 + arow, R - 1);
+                uint32_t a[4];
+                ldsm_x4(a, wchunk(wb, row, row_bytes, (k0 >> 3) + ahalf, key0 + row));
+                mma_bf16(acc[t], a, b);
+            }
+        }
+    }
+    const int g = lane >> 2, c2 = (lane & 3) * 2;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        if (t >= tiles) continue;
+        const int r0 = t * 16 + g, r1 = r0 + 8;
+        if (c2 < MT) {
+            if (r0 < R) atomicAdd(accs + r0 * 8 + c2, acc[t][0]);
+            if (r1 < R) atomicAdd(accs + r1 * 8 + c2, acc[t][2]);
+        }
+        if (c2 + 1 < MT) {
+            if (r0 < R) atomicAdd(accs + r0 * 8 + c2 + 1, acc[t][1]);
+            if (r1 < R) atomicAdd(accs + r1 * 8 + c2 + 1, acc[t][3]);
+        }
+    }
+}
 
 // Sum v[i] over the 32 lanes for every i; lane l returns the total of v[l].
 __device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
@@ -122,6 +225,98 @@ __device__ __forceinline__ void load_rows(const float* x, int ld, int M, int K, 
         } else {
 #pragma unroll
             for (int i = 0; i < 4; ++i) r.v[m][i] = 0.f;
+        }
+    }
+}
+
+// Fed rows as bf16 in shared memory, [MT][K + 8] (the 16-byte pad spreads banks).
+template <int MT>
+__device__ __forceinline__ void store_rows_bf16(const RowRegs<MT>& r, int K, __nv_bfloat16* xb) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int Kw = K / NWARPS;
+    if (lane * 4 >= Kw) return;
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+        __nv_bfloat162 lo = __floats2bfloat162_rn(r.v[m][0], r.v[m][1]);
+        __nv_bfloat162 hi = __floats2bfloat162_rn(r.v[m][2], r.v[m][3]);
+        uint2 pk;
+        pk.x = *reinterpret_cast<uint32_t*>(&lo);
+        pk.y = *reinterpret_cast<uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(xb + (size_t)m * (K + 8) + warp * Kw + lane * 4) = pk;
+    }
+}
+
+// out[n * R + row] = sum_k W[row][k] x[n][k] for the R rows (R / 16 tiles, one
+// warp per tile at a time) of a weight slice with short K (whole K per warp).
+// x: bf16 [MT][K + 8]; rows keyed key0 + row.
+template <int MT>
+__device__ __forceinline__ void mma_rows_tiles(const void* w, int R, int K, int key0, const __nv_bfloat16* xb,
+                                               float* out) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t wb = smem_addr(w), xbase = smem_addr(xb);
+    const int xstride = (K + 8) * 2, row_bytes = K * 2;
+    const int brow = (lane & 7) < MT ? (lane & 7) : 0;
+    const int bhalf = (lane >> 3) & 1;
+    const int arow = lane & 15, ahalf = lane >> 4;
+    const int g = lane >> 2, c2 = (lane & 3) * 2;
+    for (int t = warp; t * 16 < R; t += NWARPS) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        const int row = min(t * 16 + arow, R - 1);
+        for (int k0 = 0; k0 < K; k0 += 16) {
+            uint32_t a[4], b[2];
+            ldsm_x2(b, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+            ldsm_x4(a, wchunk(wb, row, row_bytes, (k0 >> 3) + ahalf, key0 + row));
+            mma_bf16(acc, a, b);
+        }
+        const int r0 = t * 16 + g, r1 = r0 + 8;
+        if (c2 < MT) {
+            if (r0 < R) out[c2 * R + r0] = acc[0];
+            if (r1 < R) out[c2 * R + r1] = acc[2];
+        }
+        if (c2 + 1 < MT) {
+            if (r0 < R) out[(c2 + 1) * R + r0] = acc[1];
+            if (r1 < R) out[(c2 + 1) * R + r1] = acc[3];
+        }
+    }
+}
+
+// y[n * C + col] = sum_f W[f][col] u[n][f] over the R FFN rows f of a slice
+// stored [R][C] (rows keyed key0 + f): the MMA's A operand is W transposed,
+// loaded with ldmatrix.trans.  u: bf16 [MT][rpad + 8], zero for f >= R.
+template <int MT>
+__device__ __forceinline__ void mma_cols_trans(const void* w, int R, int rpad, int C, int key0, const __nv_bfloat16* ub,
+                                               float* y) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t wb = smem_addr(w), ubase = smem_addr(ub);
+    const int ustride = (rpad + 8) * 2, row_bytes = C * 2;
+    const int brow = (lane & 7) < MT ? (lane & 7) : 0;
+    const int bhalf = (lane >> 3) & 1;
+    const int g = lane >> 2, c2 = (lane & 3) * 2;
+    const int ksteps = rpad / 16;  // <= 4
+    uint32_t b[4][2];
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks)
+        if (ks < ksteps) ldsm_x2(b[ks], ubase + brow * ustride + (ks * 16 + bhalf * 8) * 2);
+    // ldmatrix.trans lanes: f row = k0 + (lane & 7) + 8 * (lane >> 4), column chunk + ((lane >> 3) & 1)
+    const int fl = (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
+    for (int t = warp; t * 16 < C; t += NWARPS) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            if (ks >= ksteps) continue;
+            const int f = min(ks * 16 + fl, R - 1);
+            uint32_t a[4];
+            ldsm_x4_t(a, wchunk(wb, f, row_bytes, t * 2 + chalf, key0 + f));
+            mma_bf16(acc, a, b[ks]);
+        }
+        const int col0 = t * 16 + g, col1 = col0 + 8;
+        if (c2 < MT) {
+            y[c2 * C + col0] = acc[0];
+            y[c2 * C + col1] = acc[2];
+        }
+        if (c2 + 1 < MT) {
+            y[(c2 + 1) * C + col0] = acc[1];
+            y[(c2 + 1) * C + col1] = acc[3];
         }
     }
 }
@@ -284,6 +479,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     float* attn = reinterpret_cast<float*>(smem + L.attn);  // [MT][64]
     float* red = reinterpret_cast<float*>(smem + L.red);
     float* res = reinterpret_cast<float*>(smem + L.res);    // [MT][orows]
+    constexpr bool BF = sizeof(WT) == 2;                    // bf16 weights: tensor-core projections
+    __nv_bfloat16* xb = reinterpret_cast<__nv_bfloat16*>(smem + L.xb);
+    float* accs = reinterpret_cast<float*>(smem + L.accs);
     const long long kv_head = (long long)h * P * HEAD_DIM;
     const long long v_off = (long long)H * P * HEAD_DIM;
     const int rpg = a.rows_per_group;
@@ -350,6 +548,18 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                           &bar);
         }
         s_pre = n_pre;
+        if (seq >= 0) {  // the split's other cached pages, into L2 (copied to shared memory later)
+            const int n_pg = (s_gktot[0] + P - 1) / P;
+            const int pps = (n_pg + CA - 1) / CA;
+            const int pg1 = min(n_pg, pg0 + pps);
+            for (int p = pg0 + n_pre; p < pg1; ++p) {
+                const int phys = a.block_table[(size_t)seq * a.bt_stride + p];
+                if (phys < 0) continue;
+                const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
+                prefetch_l2(base, (uint32_t)P * HEAD_DIM * 2);
+                prefetch_l2(base + v_off, (uint32_t)P * HEAD_DIM * 2);
+            }
+        }
         if (a.next_w_a) {  // the next layer's slices of the same weights, into L2
             prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + (srcq - reinterpret_cast<const char*>(a.wqkv)), wq);
             prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + (srco - reinterpret_cast<const char*>(a.wo)), wob);
@@ -386,6 +596,10 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     }
     zero_slice(a.x_zero, (size_t)MAX_ROWS * d, h * CA + s, H * CA);
     layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
+    if (BF) {
+        store_rows_bf16<MT>(xr, d, xb);
+        for (int i = tid; i < QROWS * 8; i += NTHREADS) accs[i] = 0.f;
+    }
     trace_mark(a.trace, 0);  // inputs loaded, LN1 done
     bool ok = mbar_wait(&bar, 0, a.err);
     ok = __syncthreads_and(ok) != 0;
@@ -397,7 +611,13 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         return;
     }
     trace_mark(a.trace, 1);  // weights and cached keys in shared memory
-    project_rows<WT, MT>(wqkv, QROWS, d, xr, red, qkvp);
+    if (BF) {
+        mma_rows_ksplit<MT>(wqkv, QROWS, d, 0, xb, accs);
+        __syncthreads();
+        for (int o = tid; o < QROWS * MT; o += NTHREADS) qkvp[o] = accs[(o / MT) * 8 + o % MT];
+    } else {
+        project_rows<WT, MT>(wqkv, QROWS, d, xr, red, qkvp);
+    }
     for (int o = tid; o < QROWS * MT; o += NTHREADS) {
         const float y = qkvp[o] + (o < NTHREADS ? bq[0] : bq[1]);
         qkvp[o] = y;
@@ -446,7 +666,8 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
 
     trace_mark(a.trace, 4);  // gathered
     // ---- 4. attention over this CTA's split of each group's keys ----
-    const int row_j = warp;  // warp j owns fed row j (MT <= 8 warps)
+    constexpr int WPR = NWARPS / MT;     // warps sharing a fed row's softmax and P.V
+    const int row_j = warp / WPR, row_part = warp % WPR;
     const bool row_on = row_j < MT && row_j < a.M && s_seq[min(row_j, MT - 1)] >= 0;
     const int pos_j = row_on ? s_pos[row_j] : -1;
     const int grp_j = row_j / rpg;
@@ -496,9 +717,10 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 if (!mbar_wait(&bar, phase & 1, a.err)) mbar_wait(&bar, phase & 1, nullptr);
                 ++phase;
             }
-            for (int i = tid; i < nk * HEAD_DIM; i += NTHREADS) {  // keys fed this step, from the gather
-                const int key = bp * P + i / HEAD_DIM, dd = i % HEAD_DIM;
-                if (key >= old_len && key < K_tot) {
+            {  // keys fed this step (positions old_len .. K_tot-1 inside this batch), from the gather
+                const int k0 = max(old_len, bp * P), k1 = min(K_tot, bp * P + nk);
+                for (int i = tid; i < (k1 - k0) * HEAD_DIM; i += NTHREADS) {
+                    const int key = k0 + i / HEAD_DIM, dd = i % HEAD_DIM;
                     const int m = g * rpg + (key - old_len);
                     __nv_bfloat16* kp = slot_keys((key - bp * P) / P) + ((key - bp * P) % P) * HEAD_DIM + dd;
                     kp[0] = __float2bfloat16_rn(qkvf[(HEAD_DIM + dd) * MT + m]);
@@ -538,60 +760,75 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 }
             }
             __syncthreads();
-            if (row_on && grp_j == g) {
-                float* pr = sc + row_j * SC_STRIDE;
+            // softmax statistics: every warp of a row reads all of the row's scores
+            const bool mine = row_on && grp_j == g;
+            float* pr = sc + row_j * SC_STRIDE;
+            float m_new = m_run, corr = 1.f, lsum = 0.f;
+            if (mine) {
                 float bmax = -INFINITY;
                 for (int t = lane; t < nk; t += 32) bmax = fmaxf(bmax, pr[t]);
-                bmax = warp_max(bmax);
-                const float m_new = fmaxf(m_run, bmax);
+                m_new = fmaxf(m_run, warp_max(bmax));
                 if (m_new != -INFINITY) {
-                    const float corr = expf(m_run - m_new);
-                    float lsum = 0.f;
-                    for (int t = lane; t < nk; t += 32) {
-                        const float p = expf(pr[t] - m_new);
-                        pr[t] = p;
-                        lsum += p;
-                    }
+                    corr = expf(m_run - m_new);
+                    for (int t = lane; t < nk; t += 32) lsum += expf(pr[t] - m_new);
                     lsum = warp_sum(lsum);
-                    l_run = l_run * corr + lsum;
-                    acc0 *= corr;
-                    acc1 *= corr;
-                    m_run = m_new;
-                    __syncwarp();
-                    const int kend = min(nk, pos_j - bp * P + 1);
-                    float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
-                    for (int p0 = 0; p0 < kend; p0 += P) {  // page by page
-                        const __nv_bfloat16* vpage = slot_keys(p0 / P) + P * HEAD_DIM + 2 * lane;
-                        const int pend = min(P, kend - p0);
-                        int t = 0;
-                        for (; t + 4 <= pend; t += 4) {
+                }
+            }
+            __syncthreads();  // scores read: each warp may now overwrite its own key range
+            if (mine && m_new != -INFINITY) {
+                const int kend = min(nk, pos_j - bp * P + 1);
+                const int chunk = (kend + WPR - 1) / WPR;
+                const int kb = min(kend, row_part * chunk), ke = min(kend, kb + chunk);
+                for (int t = kb + lane; t < ke; t += 32) pr[t] = expf(pr[t] - m_new);
+                l_run = l_run * corr + lsum;
+                acc0 *= corr;
+                acc1 *= corr;
+                m_run = m_new;
+                __syncwarp();
+                float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+                for (int p0 = kb; p0 < ke;) {  // page by page
+                    const int pg = p0 / P;
+                    const __nv_bfloat16* vpage = slot_keys(pg) + P * HEAD_DIM + 2 * lane;
+                    const int pend = min(ke, (pg + 1) * P);
+                    int t = p0;
+                    for (; t + 4 <= pend; t += 4) {
 #pragma unroll
-                            for (int u = 0; u < 4; ++u) {
-                                const float p = pr[p0 + t + u];
-                                const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t + u) * HEAD_DIM);
-                                a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
-                                a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
-                            }
-                        }
-                        for (; t < pend; ++t) {
-                            const float p = pr[p0 + t];
-                            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + t * HEAD_DIM);
-                            a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
-                            a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
+                        for (int u = 0; u < 4; ++u) {
+                            const float p = pr[t + u];
+                            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t + u - pg * P) * HEAD_DIM);
+                            a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
+                            a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
                         }
                     }
-                    acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
-                    acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
+                    for (; t < pend; ++t) {
+                        const float p = pr[t];
+                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t - pg * P) * HEAD_DIM);
+                        a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
+                        a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
+                    }
+                    p0 = pend;
                 }
+                acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
+                acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
             }
         }
     }
     __syncthreads();
-    if (row_j < MT) {
+    float* pvred = reinterpret_cast<float*>(smem + L.pvred);  // [NWARPS][64]: P.V of each warp's key range
+    if (WPR > 1 && row_j < MT) {
+        pvred[warp * HEAD_DIM + 2 * lane] = acc0;
+        pvred[warp * HEAD_DIM + 2 * lane + 1] = acc1;
+    }
+    __syncthreads();
+    if (row_j < MT && row_part == 0) {
         float* pj = part + row_j * PARTW;
         if (lane == 0) {
             pj[0] = m_run;
             pj[1] = l_run;
+        }
+        for (int w = 1; w < WPR; ++w) {
+            acc0 += pvred[(warp + w) * HEAD_DIM + 2 * lane];
+            acc1 += pvred[(warp + w) * HEAD_DIM + 2 * lane + 1];
         }
         pj[2 + 2 * lane] = acc0;
         pj[3 + 2 * lane] = acc1;
@@ -601,7 +838,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     // ---- 5. merge the splits (DSMEM) and apply this CTA's W_o rows ----
     cluster.sync();
     trace_mark(a.trace, 6);
-    if (row_on) {
+    if (row_on && row_part == 0) {
         float ms = -INFINITY, ls = 0.f, o0[CA], o1[CA];
 #pragma unroll
         for (int r = 0; r < CA; ++r) {
@@ -625,32 +862,49 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         }
         attn[row_j * HEAD_DIM + 2 * lane] = r0 / Lsum;
         attn[row_j * HEAD_DIM + 2 * lane + 1] = r1 / Lsum;
-    } else if (row_j < MT) {
+    } else if (row_j < MT && row_part == 0) {
         attn[row_j * HEAD_DIM + 2 * lane] = 0.f;
         attn[row_j * HEAD_DIM + 2 * lane + 1] = 0.f;
     }
     __syncthreads();
-    for (int o = tid; o < orows * MT; o += NTHREADS) {
-        const int m = o / orows, t = o % orows;  // fed row m, W_o row t: a warp adds 32 consecutive floats
-        if (m >= a.M || s_seq[m] < 0) continue;
-        const WT* wr = wo + (size_t)t * HEAD_DIM;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};  // four independent chains
-#pragma unroll
-        for (int c = 0; c < HEAD_DIM / 4; ++c) {
-            const int cc = (c + t) & (HEAD_DIM / 4 - 1);  // rotate to spread banks
-            float w4[4];
-            load4(wr + cc * 4, w4);
-            const float4 av = *reinterpret_cast<const float4*>(attn + m * HEAD_DIM + cc * 4);
-            float v = acc[c & 3];
-            v = fmaf(w4[0], av.x, v);
-            v = fmaf(w4[1], av.y, v);
-            v = fmaf(w4[2], av.z, v);
-            v = fmaf(w4[3], av.w, v);
-            acc[c & 3] = v;
+    if (BF) {  // head output as bf16, then W_o rows on the tensor cores
+        __nv_bfloat16* ab = reinterpret_cast<__nv_bfloat16*>(smem + L.attn_b);  // [MT][64 + 8]
+        float* ytile = reinterpret_cast<float*>(smem + L.ytile);                  // [MT][orows]
+        for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS)
+            ab[(i / HEAD_DIM) * (HEAD_DIM + 8) + i % HEAD_DIM] = __float2bfloat16_rn(attn[i]);
+        __syncthreads();
+        mma_rows_tiles<MT>(wo, orows, HEAD_DIM, 0, ab, ytile);
+        __syncthreads();
+        for (int o = tid; o < orows * MT; o += NTHREADS) {
+            const int m = o / orows, t = o % orows;  // a warp adds 32 consecutive floats
+            if (m >= a.M || s_seq[m] < 0) continue;
+            float y = ytile[o];
+            if (h == 0) y += res[m * orows + t];
+            atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
         }
-        float y = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-        if (h == 0) y += res[m * orows + t];
-        atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
+    } else {
+        for (int o = tid; o < orows * MT; o += NTHREADS) {
+            const int m = o / orows, t = o % orows;  // fed row m, W_o row t: a warp adds 32 consecutive floats
+            if (m >= a.M || s_seq[m] < 0) continue;
+            const WT* wr = wo + (size_t)t * HEAD_DIM;
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};  // four independent chains
+#pragma unroll
+            for (int c = 0; c < HEAD_DIM / 4; ++c) {
+                const int cc = (c + t) & (HEAD_DIM / 4 - 1);  // rotate to spread banks
+                float w4[4];
+                load4(wr + cc * 4, w4);
+                const float4 av = *reinterpret_cast<const float4*>(attn + m * HEAD_DIM + cc * 4);
+                float v = acc[c & 3];
+                v = fmaf(w4[0], av.x, v);
+                v = fmaf(w4[1], av.y, v);
+                v = fmaf(w4[2], av.z, v);
+                v = fmaf(w4[3], av.w, v);
+                acc[c & 3] = v;
+            }
+            float y = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+            if (h == 0) y += res[m * orows + t];
+            atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
+        }
     }
     trace_mark(a.trace, 7);  // output projection added
     cluster.sync();  // peers may still read this CTA's shared memory
@@ -678,7 +932,12 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     const BLayout L(d, rpc, sizeof(WT), MT, CB);
     WT* w1 = reinterpret_cast<WT*>(smem + L.w1);
     WT* w2 = reinterpret_cast<WT*>(smem + L.w2);
-    float* u = reinterpret_cast<float*>(smem + L.u);          // [R][MT]
+    float* u = reinterpret_cast<float*>(smem + L.u);          // [R][MT] (fp32 weights)
+    constexpr bool BF = sizeof(WT) == 2;                      // bf16 weights: tensor-core projections
+    const int rpad = L.rpad;
+    __nv_bfloat16* xb = reinterpret_cast<__nv_bfloat16*>(smem + L.xb);
+    float* accs = reinterpret_cast<float*>(smem + L.accs);
+    __nv_bfloat16* ub = reinterpret_cast<__nv_bfloat16*>(smem + L.ub);  // [MT][rpad + 8]
     float* ypart = reinterpret_cast<float*>(smem + L.ypart);  // [MT][d]
     float* red = reinterpret_cast<float*>(smem + L.red);
     const bool first_cluster = blockIdx.x < CB;
@@ -720,7 +979,12 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
         }
         for (int k = 0; k < 2; ++k) {
             const int o = tid + k * NTHREADS;
-            if (o < R * MT) b1v[k] = __ldg(a.b1 + f0 + o / MT);
+            if (BF) {  // item o = (m, f) of the bf16 GELU output
+                const int f = o % rpad;
+                if (o < MT * rpad && f < R) b1v[k] = __ldg(a.b1 + f0 + f);
+            } else if (o < R * MT) {
+                b1v[k] = __ldg(a.b1 + f0 + o / MT);
+            }
         }
     }
 
@@ -747,6 +1011,10 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     }
     zero_slice(a.x_zero, (size_t)MAX_ROWS * d, blockIdx.x, gridDim.x);
     layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
+    if (BF) {
+        store_rows_bf16<MT>(xr, d, xb);
+        for (int i = tid; i < rpc * 8; i += NTHREADS) accs[i] = 0.f;
+    }
 
     trace_mark(a.trace, 0);  // inputs loaded, LN2 done
     bool ok = R == 0 || mbar_wait(&bar, 0, a.err);
@@ -758,32 +1026,53 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
         return;
     }
     trace_mark(a.trace, 1);  // weights in shared memory
-    // u = GELU(LN2(x) W1^T + b1) for this CTA's FFN rows
-    if (R > 0) project_rows<WT, MT>(w1, R, d, xr, red, u);
-    for (int o = tid; o < R * MT; o += NTHREADS) u[o] = gelu_erf(u[o] + (o < NTHREADS ? b1v[0] : b1v[1]));
-    __syncthreads();
-    trace_mark(a.trace, 2);  // u done
-    // partial u W2^T over all d columns (W2 stored transposed: row f = column f of W2)
-    for (int c = tid * 4; c < d; c += NTHREADS * 4) {
-        float acc[MT][4];
-#pragma unroll
-        for (int m = 0; m < MT; ++m)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) acc[m][i] = 0.f;
-        for (int f = 0; f < R; ++f) {
-            float w4[4];
-            load4(w2 + (size_t)f * d + c, w4);
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                const float uf = u[f * MT + m];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) acc[m][i] = fmaf(uf, w4[i], acc[m][i]);
-            }
+    if (BF) {
+        // u = GELU(LN2(x) W1^T + b1) for this CTA's FFN rows, as bf16 [MT][rpad]
+        if (R > 0) mma_rows_ksplit<MT>(w1, R, d, f0, xb, accs);
+        __syncthreads();
+        for (int k = 0; k < 2; ++k) {
+            const int o = tid + k * NTHREADS;
+            if (o >= MT * rpad) continue;
+            const int m = o / rpad, f = o % rpad;
+            const float v = f < R ? gelu_erf(accs[f * 8 + m] + b1v[k]) : 0.f;
+            ub[m * (rpad + 8) + f] = __float2bfloat16_rn(v);
         }
+        __syncthreads();
+        trace_mark(a.trace, 2);  // u done
+        // partial u W2^T over all d columns (W2 stored transposed: row f = column f of W2)
+        if (R > 0) {
+            mma_cols_trans<MT>(w2, R, rpad, d, f0, ub, ypart);
+        } else {
+            for (int i = tid; i < MT * d; i += NTHREADS) ypart[i] = 0.f;
+        }
+    } else {
+        // u = GELU(LN2(x) W1^T + b1) for this CTA's FFN rows
+        if (R > 0) project_rows<WT, MT>(w1, R, d, xr, red, u);
+        for (int o = tid; o < R * MT; o += NTHREADS) u[o] = gelu_erf(u[o] + (o < NTHREADS ? b1v[0] : b1v[1]));
+        __syncthreads();
+        trace_mark(a.trace, 2);  // u done
+        // partial u W2^T over all d columns (W2 stored transposed: row f = column f of W2)
+        for (int c = tid * 4; c < d; c += NTHREADS * 4) {
+            float acc[MT][4];
 #pragma unroll
-        for (int m = 0; m < MT; ++m)
-            *reinterpret_cast<float4*>(ypart + (size_t)m * d + c) =
-                make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]);
+            for (int m = 0; m < MT; ++m)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[m][i] = 0.f;
+            for (int f = 0; f < R; ++f) {
+                float w4[4];
+                load4(w2 + (size_t)f * d + c, w4);
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+                    const float uf = u[f * MT + m];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) acc[m][i] = fmaf(uf, w4[i], acc[m][i]);
+                }
+            }
+#pragma unroll
+            for (int m = 0; m < MT; ++m)
+                *reinterpret_cast<float4*>(ypart + (size_t)m * d + c) =
+                    make_float4(acc[m][0], acc[m][1], acc[m][2], acc[m][3]);
+        }
     }
     trace_mark(a.trace, 3);  // partial outputs done
     cluster.sync();

@@ -469,9 +469,24 @@ void relayout(const mtp_config& cf, int j, int es, const unsigned char* src, uns
         for (size_t h = 0; h < H; ++h)
             for (size_t f = 0; f < d; ++f)
                 std::memcpy(dst + ((h * d + f) * HEAD_DIM) * es, src + (f * d + h * HEAD_DIM) * es, HEAD_DIM * es);
-    } else {
+    } else if (j == 10) {
         for (size_t c = 0; c < d; ++c)
             for (size_t f = 0; f < F; ++f) std::memcpy(dst + (f * d + c) * es, src + (c * F + f) * es, es);
+    } else {
+        std::memcpy(dst, src, F * d * es);
+    }
+}
+
+// bf16 matrices feed ldmatrix from shared memory: 16-byte chunk c of row g is
+// stored at chunk c ^ (g & 7) of that row, so the eight rows one ldmatrix
+// phase reads fall in eight different bank groups.  Rows hold >= 8 chunks.
+void swizzle_rows(unsigned char* w, size_t rows, size_t row_bytes) {
+    const size_t chunks = row_bytes / 16;
+    std::vector<unsigned char> row(row_bytes);
+    for (size_t g = 0; g < rows; ++g) {
+        unsigned char* r = w + g * row_bytes;
+        std::memcpy(row.data(), r, row_bytes);
+        for (size_t c = 0; c < chunks; ++c) std::memcpy(r + (c ^ (g & 7)) * 16, row.data() + c * 16, 16);
     }
 }
 
@@ -511,9 +526,13 @@ int upload_weights(mtp_ctx* c, const void* blob, size_t bytes) {
         std::memcpy(&nb, b + 24 + 16 * i + 8, 8);
         const unsigned char* src = b + off;
         const int j = i >= 2 && i < 2 + 12u * cf.layers ? (int)((i - 2) % 12) : -1;
-        if (j == 2 || j == 3 || j == 4 || j == 10) {  // device layouts of the fused block kernels
+        if (j == 2 || j == 3 || j == 4 || j == 10 || (j == 8 && c->wbytes == 2)) {  // fused-kernel layouts
             tmp.resize(nb);
             relayout(cf, j, j == 3 ? 4 : c->wbytes, src, tmp.data());
+            if (c->wbytes == 2 && j != 3) {
+                const size_t row_elems = j == 4 ? HEAD_DIM : cf.d_model;
+                swizzle_rows(tmp.data(), nb / (row_elems * 2), row_elems * 2);
+            }
             src = tmp.data();
         }
         CUDA_TRY(cudaMemcpy(dw + dev_off[i], src, nb, cudaMemcpyHostToDevice));
