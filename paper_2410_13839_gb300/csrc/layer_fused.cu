@@ -48,39 +48,43 @@ __host__ __device__ inline size_t al128(size_t x) { return (x + 127) & ~(size_t)
 
 // ---- shared-memory layouts (host and device compute the same offsets) ----
 struct ALayout {
-    size_t wqkv, wo, ks, qkvp, qkvf, qs, part, attn, res, uni, total;
-    size_t xb, accs, red, sc, pvred, attn_b, ytile;  // inside the union (phases do not overlap)
-    int tile;       // keys of the dedicated staging slots
-    int sc_stride;  // keys per batch (dedicated and reused slots)
+    size_t wqkv, wo, ks, qkvp, qkvf, qs, part, attn, uni, total;
+    size_t xb, red, attn_b, ytile;  // inside the union (phases do not overlap)
+    int tile;  // keys of the dedicated staging slots (filled before the dependency wait)
     __host__ __device__ ALayout(int d, int wbytes, int mt, int page) {
         const int groups = (QROWS * mt + 31) / 32;
-        tile = (MIN_TILE + page - 1) / page * page;  // whole pages, at least MIN_TILE keys
+        const size_t wq_bytes = (size_t)QROWS * d * wbytes, slot_bytes = (size_t)2 * page * HEAD_DIM * 2;
+        // whole pages, at least MIN_TILE keys; none at 8 rows when the weight area holds a page
+        // (the 8-row inputs need the space; every page then arrives after the projection)
+        tile = mt >= 8 && wq_bytes >= slot_bytes ? 0 : (MIN_TILE + page - 1) / page * page;
+        // the q|k|v slice and the dedicated page slots are adjacent: after the
+        // attention they hold the warps' softmax states [NWARPS][mt][PARTW]
+        size_t ks_bytes = (size_t)2 * tile * HEAD_DIM * 2;
+        const size_t merge_bytes = (size_t)NWARPS * mt * PARTW * 4;
+        if (wq_bytes + ks_bytes < merge_bytes) ks_bytes = merge_bytes - wq_bytes;
         wqkv = 0;
-        wo = al128(wqkv + (size_t)QROWS * d * wbytes);
-        ks = al128(wo + (size_t)(d / CA) * HEAD_DIM * wbytes);  // page slots: [keys | values] each
-        qkvp = al128(ks + (size_t)2 * tile * HEAD_DIM * 2);
-        res = al128(qkvp + (size_t)QROWS * mt * 4);
-        qkvf = al128(res + (size_t)mt * (d / CA) * 4);
+        ks = al128(wqkv + wq_bytes);  // page slots: [keys | values] each
+        wo = al128(ks + ks_bytes);
+        qkvp = al128(wo + (size_t)(d / CA) * HEAD_DIM * wbytes);
+        qkvf = al128(qkvp + (size_t)QROWS * mt * 4);
         qs = al128(qkvf + (size_t)3 * HEAD_DIM * mt * 4);
         part = al128(qs + (size_t)mt * HEAD_DIM * 4);
         attn = al128(part + (size_t)mt * PARTW * 4);
         uni = al128(attn + (size_t)mt * HEAD_DIM * 4);
-        sc_stride = (tile / page + (QROWS * d * wbytes) / (4 * page * HEAD_DIM)) * page;  // keys per batch
-        // projection: bf16 inputs + tile sums (tensor cores) or the reduce-scatter scratch (fp32);
-        // qkvf, qs, part and attn are written only after the projection, so it may start there
+        // projection: bf16 hi/lo inputs, then (same space) the warps' tile sums (tensor cores),
+        // or the reduce-scatter scratch (fp32); qkvf, qs, part and attn are written only after
+        // the projection, so it may start there
         xb = qkvf;
-        accs = al128(xb + (size_t)mt * (d + 8) * 2);
-        red = al128(accs + (size_t)QROWS * 8 * 4);
-        const size_t p1 = wbytes == 2 ? red : red + (size_t)NWARPS * groups * 32 * 4;
-        // attention: scores, per-warp P.V partials
-        sc = uni;
-        pvred = al128(sc + (size_t)mt * sc_stride * 4);
-        const size_t p2 = pvred + (size_t)NWARPS * HEAD_DIM * 4;
-        // output projection: bf16 head output, projected rows
+        red = xb;  // the tile sums are reduced into qkvp, outside this space
+        size_t xbytes = (size_t)2 * mt * (d + 8) * 2;
+        const size_t rbytes = wbytes == 2 ? (size_t)NWARPS * QROWS * 8 * 4 : (size_t)NWARPS * groups * 32 * 4;
+        if (rbytes > xbytes) xbytes = rbytes;
+        const size_t p1 = xb + xbytes;
+        // output projection: bf16 hi/lo head output, projected rows
         attn_b = uni;
-        ytile = al128(attn_b + (size_t)mt * (HEAD_DIM + 8) * 2);
+        ytile = al128(attn_b + (size_t)2 * mt * (HEAD_DIM + 8) * 2);
         const size_t p3 = ytile + (size_t)mt * (d / CA) * 4;
-        total = al128(p1 > p2 ? (p1 > p3 ? p1 : p3) : (p2 > p3 ? p2 : p3));
+        total = al128(p1 > p3 ? p1 : p3);
     }
 };
 
@@ -94,11 +98,11 @@ struct BLayout {
         w1 = 0;
         w2 = al128(w1 + (size_t)rows * d * wbytes);
         xb = al128(w2 + (size_t)rows * d * wbytes);
-        accs = al128(xb + (size_t)mt * (d + 8) * 2);
+        accs = al128(xb + (size_t)2 * mt * (d + 8) * 2);
         ub = al128(accs + (size_t)rows * 8 * 4);
-        u = al128(ub + (size_t)mt * (rpad + 8) * 2);
+        u = al128(ub + (size_t)2 * mt * (rpad + 8) * 2);
         red = al128(u + (wbytes == 2 ? 0 : (size_t)rows * mt * 4));
-        size_t end = al128(red + (wbytes == 2 ? 0 : (size_t)NWARPS * groups * 32 * 4));
+        size_t end = al128(red + (wbytes == 2 ? (size_t)NWARPS * rows * 8 * 4 : (size_t)NWARPS * groups * 32 * 4));
         const size_t ybytes = (size_t)mt * d * 4;
         // the partial outputs reuse W1's space once u is known, when it fits
         if ((size_t)rows * d * wbytes >= ybytes) {
@@ -136,6 +140,16 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
+// x0, x1 as bf16 pairs hi + lo with hi + lo = x to about 2^-16 relative
+// (low halves hold the first element, as the MMA fragments expect).
+__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+    const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
+    const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+    hi = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    lo = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+}
+
 // Shared address of 16-byte chunk `chunk` of weight row `row` (row_bytes each):
 // the weights are stored with chunk c of global row g at position c ^ (g & 7)
 // (made at create), which keeps ldmatrix free of bank conflicts.
@@ -143,12 +157,15 @@ __device__ __forceinline__ uint32_t wchunk(uint32_t base, int row, int row_bytes
     return base + (uint32_t)row * row_bytes + ((uint32_t)(chunk ^ (key & 7)) << 4);
 }
 
-// accs[row][n] += sum_k W[row][k] x[n][k] for the R (<= 64) rows of a weight
-// slice in shared memory (rows keyed key0 + row), K split across the 8 warps;
-// each warp adds its tile sums into accs (zeroed beforehand) with shared atomics.
+// out[row][n] = sum_k W[row][k] x[n][k] ([R][MT]) for the R (<= 64) rows of a weight
+// slice in shared memory (rows keyed key0 + row), K split across the 8
+// warps.  x is given as bf16 hi and lo parts ([MT][K + 8] each, lo right
+// after hi), one MMA each, so the product keeps x to fp32 accuracy.  Each
+// warp stores its tile sums in wpart [NWARPS][R][8] (which may overlap x)
+// and a second pass adds the warps' partials (no shared-memory atomics).
 template <int MT>
 __device__ __forceinline__ void mma_rows_ksplit(const void* w, int R, int K, int key0, const __nv_bfloat16* xb,
-                                                float* accs) {
+                                                float* wpart, float* out) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int tiles = (R + 15) / 16;
     const int kslice = K / NWARPS;
@@ -162,32 +179,39 @@ __device__ __forceinline__ void mma_rows_ksplit(const void* w, int R, int K, int
     for (int t = 0; t < 4; ++t)
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[t][i] = 0.f;
+    const uint32_t xlo = (uint32_t)MT * xstride;
     for (int k0 = warp * kslice; k0 < (warp + 1) * kslice; k0 += 16) {
-        uint32_t b[2];
-        ldsm_x2(b, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+        uint32_t bh[2], bl[2];
+        ldsm_x2(bh, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+        ldsm_x2(bl, xbase + xlo + brow * xstride + (k0 + bhalf * 8) * 2);
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
             if (t < tiles) {
                 const int row = min(t * 16 + arow, R - 1);
                 uint32_t a[4];
                 ldsm_x4(a, wchunk(wb, row, row_bytes, (k0 >> 3) + ahalf, key0 + row));
-                mma_bf16(acc[t], a, b);
+                mma_bf16(acc[t], a, bh);
+                mma_bf16(acc[t], a, bl);
             }
         }
     }
+    __syncthreads();  // every warp is done with x
     const int g = lane >> 2, c2 = (lane & 3) * 2;
+    float* mine = wpart + (size_t)warp * R * 8;
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
         if (t >= tiles) continue;
         const int r0 = t * 16 + g, r1 = r0 + 8;
-        if (c2 < MT) {
-            if (r0 < R) atomicAdd(accs + r0 * 8 + c2, acc[t][0]);
-            if (r1 < R) atomicAdd(accs + r1 * 8 + c2, acc[t][2]);
-        }
-        if (c2 + 1 < MT) {
-            if (r0 < R) atomicAdd(accs + r0 * 8 + c2 + 1, acc[t][1]);
-            if (r1 < R) atomicAdd(accs + r1 * 8 + c2 + 1, acc[t][3]);
-        }
+        if (r0 < R) *reinterpret_cast<float2*>(mine + r0 * 8 + c2) = make_float2(acc[t][0], acc[t][1]);
+        if (r1 < R) *reinterpret_cast<float2*>(mine + r1 * 8 + c2) = make_float2(acc[t][2], acc[t][3]);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < R * MT; i += NTHREADS) {
+        const int j = (i / MT) * 8 + i % MT;
+        float y = 0.f;
+#pragma unroll
+        for (int w2 = 0; w2 < NWARPS; ++w2) y += wpart[(size_t)w2 * R * 8 + j];
+        out[i] = y;
     }
 }
 
@@ -229,26 +253,27 @@ __device__ __forceinline__ void load_rows(const float* x, int ld, int M, int K, 
     }
 }
 
-// Fed rows as bf16 in shared memory, [MT][K + 8] (the 16-byte pad spreads banks).
+// Fed rows as bf16 hi and lo parts in shared memory, [MT][K + 8] each (lo
+// right after hi; the 16-byte pad spreads banks).
 template <int MT>
-__device__ __forceinline__ void store_rows_bf16(const RowRegs<MT>& r, int K, __nv_bfloat16* xb) {
+__device__ __forceinline__ void store_rows_split(const RowRegs<MT>& r, int K, __nv_bfloat16* xb) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int Kw = K / NWARPS;
     if (lane * 4 >= Kw) return;
 #pragma unroll
     for (int m = 0; m < MT; ++m) {
-        __nv_bfloat162 lo = __floats2bfloat162_rn(r.v[m][0], r.v[m][1]);
-        __nv_bfloat162 hi = __floats2bfloat162_rn(r.v[m][2], r.v[m][3]);
-        uint2 pk;
-        pk.x = *reinterpret_cast<uint32_t*>(&lo);
-        pk.y = *reinterpret_cast<uint32_t*>(&hi);
-        *reinterpret_cast<uint2*>(xb + (size_t)m * (K + 8) + warp * Kw + lane * 4) = pk;
+        uint2 h, l;
+        split_bf16x2(r.v[m][0], r.v[m][1], h.x, l.x);
+        split_bf16x2(r.v[m][2], r.v[m][3], h.y, l.y);
+        const size_t at = (size_t)m * (K + 8) + warp * Kw + lane * 4;
+        *reinterpret_cast<uint2*>(xb + at) = h;
+        *reinterpret_cast<uint2*>(xb + (size_t)MT * (K + 8) + at) = l;
     }
 }
 
 // out[n * R + row] = sum_k W[row][k] x[n][k] for the R rows (R / 16 tiles, one
 // warp per tile at a time) of a weight slice with short K (whole K per warp).
-// x: bf16 [MT][K + 8]; rows keyed key0 + row.
+// x: bf16 hi and lo parts [MT][K + 8] each (lo right after hi); rows keyed key0 + row.
 template <int MT>
 __device__ __forceinline__ void mma_rows_tiles(const void* w, int R, int K, int key0, const __nv_bfloat16* xb,
                                                float* out) {
@@ -263,10 +288,12 @@ __device__ __forceinline__ void mma_rows_tiles(const void* w, int R, int K, int 
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
         const int row = min(t * 16 + arow, R - 1);
         for (int k0 = 0; k0 < K; k0 += 16) {
-            uint32_t a[4], b[2];
-            ldsm_x2(b, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+            uint32_t a[4], bh[2], bl[2];
+            ldsm_x2(bh, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
+            ldsm_x2(bl, xbase + MT * xstride + brow * xstride + (k0 + bhalf * 8) * 2);
             ldsm_x4(a, wchunk(wb, row, row_bytes, (k0 >> 3) + ahalf, key0 + row));
-            mma_bf16(acc, a, b);
+            mma_bf16(acc, a, bh);
+            mma_bf16(acc, a, bl);
         }
         const int r0 = t * 16 + g, r1 = r0 + 8;
         if (c2 < MT) {
@@ -282,7 +309,8 @@ __device__ __forceinline__ void mma_rows_tiles(const void* w, int R, int K, int 
 
 // y[n * C + col] = sum_f W[f][col] u[n][f] over the R FFN rows f of a slice
 // stored [R][C] (rows keyed key0 + f): the MMA's A operand is W transposed,
-// loaded with ldmatrix.trans.  u: bf16 [MT][rpad + 8], zero for f >= R.
+// loaded with ldmatrix.trans.  u: bf16 hi and lo parts [MT][rpad + 8] each
+// (lo right after hi), zero for f >= R.
 template <int MT>
 __device__ __forceinline__ void mma_cols_trans(const void* w, int R, int rpad, int C, int key0, const __nv_bfloat16* ub,
                                                float* y) {
@@ -293,10 +321,13 @@ __device__ __forceinline__ void mma_cols_trans(const void* w, int R, int rpad, i
     const int bhalf = (lane >> 3) & 1;
     const int g = lane >> 2, c2 = (lane & 3) * 2;
     const int ksteps = rpad / 16;  // <= 4
-    uint32_t b[4][2];
+    uint32_t bh[4][2], bl[4][2];
 #pragma unroll
     for (int ks = 0; ks < 4; ++ks)
-        if (ks < ksteps) ldsm_x2(b[ks], ubase + brow * ustride + (ks * 16 + bhalf * 8) * 2);
+        if (ks < ksteps) {
+            ldsm_x2(bh[ks], ubase + brow * ustride + (ks * 16 + bhalf * 8) * 2);
+            ldsm_x2(bl[ks], ubase + MT * ustride + brow * ustride + (ks * 16 + bhalf * 8) * 2);
+        }
     // ldmatrix.trans lanes: f row = k0 + (lane & 7) + 8 * (lane >> 4), column chunk + ((lane >> 3) & 1)
     const int fl = (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
     for (int t = warp; t * 16 < C; t += NWARPS) {
@@ -307,7 +338,8 @@ __device__ __forceinline__ void mma_cols_trans(const void* w, int R, int rpad, i
             const int f = min(ks * 16 + fl, R - 1);
             uint32_t a[4];
             ldsm_x4_t(a, wchunk(wb, f, row_bytes, t * 2 + chalf, key0 + f));
-            mma_bf16(acc, a, b[ks]);
+            mma_bf16(acc, a, bh[ks]);
+            mma_bf16(acc, a, bl[ks]);
         }
         const int col0 = t * 16 + g, col1 = col0 + 8;
         if (c2 < MT) {
@@ -447,6 +479,38 @@ __device__ __forceinline__ void plan_row(const LayerArgs& a, int r, int& seq, in
     }
 }
 
+// Column of element dd of key/value row t inside a cached page: the row's
+// 16-byte chunks are stored in the order chunk ^ (t & 7), which keeps the
+// attention's ldmatrix reads of eight consecutive rows free of bank conflicts.
+__device__ __forceinline__ int kv_col(int t, int dd) { return (((dd >> 3) ^ (t & 7)) << 3) | (dd & 7); }
+
+// Bulk copies of cached pages bp + first .. bp + nb - 1 of sequence seq into
+// slots first .. nb - 1 (the first n_ded slots in the dedicated area, the
+// rest in the free weight area), on barrier `bar`.  One thread calls it;
+// returns whether anything was requested.
+__device__ __forceinline__ int issue_pages(const LayerArgs& a, int seq, int bp, int first, int nb, int slot_elems,
+                                           long long kv_head, long long v_off, __nv_bfloat16* ks,
+                                           __nv_bfloat16* wq_slots, int n_ded, uint64_t* bar) {
+    const int P = a.page_size;
+    uint32_t bytes = 0;
+    for (int p = first; p < nb; ++p)
+        if (a.block_table[(size_t)seq * a.bt_stride + bp + p] >= 0) bytes += (uint32_t)slot_elems * 2;
+    if (!bytes) return 0;
+    mbar_arrive_expect_tx(bar, bytes);
+    for (int p = first; p < nb; ++p) {
+        const int phys = a.block_table[(size_t)seq * a.bt_stride + bp + p];
+        if (phys < 0) {
+            atomicOr(a.err, ERR_BOUNDS);
+            continue;
+        }
+        __nv_bfloat16* dst = p < n_ded ? ks + (size_t)p * slot_elems : wq_slots + (size_t)(p - n_ded) * slot_elems;
+        const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
+        bulk_copy_g2s(dst, base, (uint32_t)P * HEAD_DIM * 2, bar);
+        bulk_copy_g2s(dst + P * HEAD_DIM, base + v_off, (uint32_t)P * HEAD_DIM * 2, bar);
+    }
+    return 1;
+}
+
 // ============================================================ kernel A ====
 
 template <typename WT, int MT>
@@ -467,24 +531,25 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     const int orows = d / CA;  // W_o rows of this CTA
     const ALayout L(d, sizeof(WT), MT, P);
     const int ATT_TILE = L.tile;
-    const int SC_STRIDE = L.sc_stride;
     WT* wqkv = reinterpret_cast<WT*>(smem + L.wqkv);
     WT* wo = reinterpret_cast<WT*>(smem + L.wo);
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem + L.ks);
     float* qkvp = reinterpret_cast<float*>(smem + L.qkvp);  // [QROWS][MT]
     float* qkvf = reinterpret_cast<float*>(smem + L.qkvf);  // [192][MT]
     float* qs = reinterpret_cast<float*>(smem + L.qs);      // [MT][64]
-    float* sc = reinterpret_cast<float*>(smem + L.sc);      // [MT][SC_STRIDE]
     float* part = reinterpret_cast<float*>(smem + L.part);  // [MT][PARTW]
     float* attn = reinterpret_cast<float*>(smem + L.attn);  // [MT][64]
     float* red = reinterpret_cast<float*>(smem + L.red);
-    float* res = reinterpret_cast<float*>(smem + L.res);    // [MT][orows]
     constexpr bool BF = sizeof(WT) == 2;                    // bf16 weights: tensor-core projections
     __nv_bfloat16* xb = reinterpret_cast<__nv_bfloat16*>(smem + L.xb);
-    float* accs = reinterpret_cast<float*>(smem + L.accs);
     const long long kv_head = (long long)h * P * HEAD_DIM;
     const long long v_off = (long long)H * P * HEAD_DIM;
     const int rpg = a.rows_per_group;
+    // page slots: the dedicated staging area, then the q|k|v weight area, free after the projection
+    const int slot_elems = 2 * P * HEAD_DIM;  // keys then values of one page
+    const int n_ded = ATT_TILE / P;
+    const int n_slots = n_ded + (int)((size_t)QROWS * d * sizeof(WT) / ((size_t)slot_elems * 2));
+    __nv_bfloat16* const wq_slots = reinterpret_cast<__nv_bfloat16*>(smem + L.wqkv);
 
     // ---- 1. before the wait: fed rows, weights, cached keys/values ----
     if (tid < MT) {
@@ -588,17 +653,17 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     // ---- 2. inputs: LN1, projection ----
     RowRegs<MT> xr;
     load_rows<MT>(a.x_in, d, a.M, d, xr);
-    if (h == 0) {  // residual slice for the W_o rows of this CTA
-        for (int i = tid; i < MT * orows; i += NTHREADS) {
-            const int m = i / orows, f = s * orows + i % orows;
-            res[i] = m < a.M ? a.x_in[(size_t)m * d + f] + a.bo[f] : 0.f;
-        }
+    constexpr int RES_N = (MT * (1024 / CA) + NTHREADS - 1) / NTHREADS;  // W_o outputs per thread
+    float resr[RES_N];  // residual + bias of this thread's W_o outputs (head 0 adds them)
+#pragma unroll
+    for (int k = 0; k < RES_N; ++k) {
+        const int o = tid + k * NTHREADS, m = o / orows, f = s * orows + o % orows;
+        resr[k] = h == 0 && o < orows * MT && m < a.M ? a.x_in[(size_t)m * d + f] + a.bo[f] : 0.f;
     }
     zero_slice(a.x_zero, (size_t)MAX_ROWS * d, h * CA + s, H * CA);
     layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
     if (BF) {
-        store_rows_bf16<MT>(xr, d, xb);
-        for (int i = tid; i < QROWS * 8; i += NTHREADS) accs[i] = 0.f;
+        store_rows_split<MT>(xr, d, xb);
     }
     trace_mark(a.trace, 0);  // inputs loaded, LN1 done
     bool ok = mbar_wait(&bar, 0, a.err);
@@ -612,11 +677,21 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     }
     trace_mark(a.trace, 1);  // weights and cached keys in shared memory
     if (BF) {
-        mma_rows_ksplit<MT>(wqkv, QROWS, d, 0, xb, accs);
+        mma_rows_ksplit<MT>(wqkv, QROWS, d, 0, xb, red, qkvp);
         __syncthreads();
-        for (int o = tid; o < QROWS * MT; o += NTHREADS) qkvp[o] = accs[(o / MT) * 8 + o % MT];
     } else {
         project_rows<WT, MT>(wqkv, QROWS, d, xr, red, qkvp);
+    }
+    if (tid == 0) {  // group 0's first batch of cached pages into the slots, while the cluster gathers
+        s_armed = 0;
+        const int seq = s_gseq[0];
+        if (seq >= 0) {
+            const int n_pg = (s_gktot[0] + P - 1) / P, pps = (n_pg + CA - 1) / CA;
+            const int pg0 = s * pps, pg1 = min(n_pg, pg0 + pps);
+            if (pg0 < pg1)
+                s_armed = issue_pages(a, seq, pg0, s_pre, min(n_slots, pg1 - pg0), slot_elems, kv_head, v_off, Ks,
+                                      wq_slots, n_ded, &bar);
+        }
     }
     for (int o = tid; o < QROWS * MT; o += NTHREADS) {
         const float y = qkvp[o] + (o < NTHREADS ? bq[0] : bq[1]);
@@ -629,8 +704,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 atomicOr(a.err, ERR_BOUNDS);
                 continue;
             }
+            const int t = s_pos[m] % P;  // key row of the page; its 16-byte chunks are stored swizzled
             const long long idx = (long long)page * a.page_elems + a.layer_off + (sec - 1) * v_off + kv_head +
-                                  (long long)(s_pos[m] % P) * HEAD_DIM + dd;
+                                  (long long)t * HEAD_DIM + kv_col(t, dd);
             reinterpret_cast<uint16_t*>(a.kv_pool)[idx] = f32_to_bf16_bits(y);
         }
     }
@@ -666,22 +742,35 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
 
     trace_mark(a.trace, 4);  // gathered
     // ---- 4. attention over this CTA's split of each group's keys ----
-    constexpr int WPR = NWARPS / MT;     // warps sharing a fed row's softmax and P.V
-    const int row_j = warp / WPR, row_part = warp % WPR;
-    const bool row_on = row_j < MT && row_j < a.M && s_seq[min(row_j, MT - 1)] >= 0;
-    const int pos_j = row_on ? s_pos[row_j] : -1;
-    const int grp_j = row_j / rpg;
-    float m_run = -INFINITY, l_run = 0.f, acc0 = 0.f, acc1 = 0.f;
+    // Flash-attention style on the tensor cores: each warp takes 16-key tiles
+    // of a batch; S = Q K^T (fed rows as the M = 16 side, rows >= MT zero)
+    // and O += P V with online-softmax state in registers.  Q and P enter as
+    // bf16 hi + lo pairs (two MMAs), which keeps them to fp32 accuracy.
+    const int qrow = lane >> 2, c2 = (lane & 3) * 2;
+    const bool qon = qrow < MT && qrow < a.M && s_seq[min(qrow, MT - 1)] >= 0;
+    const int qpos = qon ? s_pos[qrow] : -1;
+    const int qgrp = qrow / rpg;
+    uint32_t qhi[4][2], qlo[4][2];  // A-fragment registers 0 and 2 of each k-step (rows g + 8 are zero)
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int k = ks * 16 + hh * 8 + c2;
+            const float q0 = qon ? qs[qrow * HEAD_DIM + k] : 0.f, q1 = qon ? qs[qrow * HEAD_DIM + k + 1] : 0.f;
+            split_bf16x2(q0, q1, qhi[ks][hh], qlo[ks][hh]);
+        }
+    float m_run = -INFINITY, l_run = 0.f;
+    float o[8][4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) o[j][i] = 0.f;
     const int G = (a.M + rpg - 1) / rpg;
-    // page slots: the dedicated staging area, then the q|k|v weight area, free after the projection
-    const int slot_elems = 2 * P * HEAD_DIM;  // keys then values of one page
-    const int n_ded = ATT_TILE / P;
-    const int n_slots = n_ded + (int)((size_t)QROWS * d * sizeof(WT) / ((size_t)slot_elems * 2));
-    __nv_bfloat16* const wq_slots = reinterpret_cast<__nv_bfloat16*>(smem + L.wqkv);
     auto slot_keys = [&](int i) -> __nv_bfloat16* {
         return i < n_ded ? Ks + (size_t)i * slot_elems : wq_slots + (size_t)(i - n_ded) * slot_elems;
     };
     uint32_t phase = 1;  // phase 0 of the barrier brought the weights
+    bool first_batch = true;
     for (int g = 0; g < G; ++g) {
         const int seq = s_gseq[g], old_len = s_gold[g], K_tot = s_gktot[g];
         if (seq < 0) continue;
@@ -691,28 +780,13 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         for (int bp = pg0; bp < pg1; bp += n_slots) {
             const int nb = min(n_slots, pg1 - bp);
             const int nk = nb * P;
-            const int first = (g == 0 && bp == pg0) ? s_pre : 0;  // slots already filled before the wait
             __syncthreads();  // every reader of the slots is done with the previous batch
-            if (tid == 0) {
-                uint32_t bytes = 0;
-                for (int p = first; p < nb; ++p)
-                    if (a.block_table[(size_t)seq * a.bt_stride + bp + p] >= 0) bytes += (uint32_t)slot_elems * 2;
-                if (bytes) {
-                    mbar_arrive_expect_tx(&bar, bytes);
-                    for (int p = first; p < nb; ++p) {
-                        const int phys = a.block_table[(size_t)seq * a.bt_stride + bp + p];
-                        if (phys < 0) {
-                            atomicOr(a.err, ERR_BOUNDS);
-                            continue;
-                        }
-                        const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
-                        bulk_copy_g2s(slot_keys(p), base, (uint32_t)P * HEAD_DIM * 2, &bar);
-                        bulk_copy_g2s(slot_keys(p) + P * HEAD_DIM, base + v_off, (uint32_t)P * HEAD_DIM * 2, &bar);
-                    }
-                }
-                s_armed = bytes > 0;
+            if (!(first_batch && g == 0)) {  // group 0's first batch was requested after the projection
+                if (tid == 0) s_armed = issue_pages(a, seq, bp, 0, nb, slot_elems, kv_head, v_off, Ks, wq_slots,
+                                                    n_ded, &bar);
+                __syncthreads();
             }
-            __syncthreads();
+            first_batch = false;
             if (s_armed) {
                 if (!mbar_wait(&bar, phase & 1, a.err)) mbar_wait(&bar, phase & 1, nullptr);
                 ++phase;
@@ -722,123 +796,116 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 for (int i = tid; i < (k1 - k0) * HEAD_DIM; i += NTHREADS) {
                     const int key = k0 + i / HEAD_DIM, dd = i % HEAD_DIM;
                     const int m = g * rpg + (key - old_len);
-                    __nv_bfloat16* kp = slot_keys((key - bp * P) / P) + ((key - bp * P) % P) * HEAD_DIM + dd;
+                    const int t = (key - bp * P) % P;
+                    __nv_bfloat16* kp = slot_keys((key - bp * P) / P) + t * HEAD_DIM + kv_col(t, dd);
                     kp[0] = __float2bfloat16_rn(qkvf[(HEAD_DIM + dd) * MT + m]);
                     kp[P * HEAD_DIM] = __float2bfloat16_rn(qkvf[(2 * HEAD_DIM + dd) * MT + m]);
                 }
             }
             __syncthreads();
-            // scores: thread t = key t of the batch, rows of this group
-            for (int t = tid; t < nk; t += NTHREADS) {
-                const __nv_bfloat16* krow = slot_keys(t / P) + (t % P) * HEAD_DIM;
-                float scv[MT];
+            for (int kt = warp * 16; kt < nk; kt += NWARPS * 16) {
+                const int r0 = kt % P;  // first key row of the tile in its page
+                const uint32_t kb = smem_addr(slot_keys(kt / P)), vb = kb + P * HEAD_DIM * 2;
+                float sfr[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+                {
+                    const int key = r0 + (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
 #pragma unroll
-                for (int j = 0; j < MT; ++j) scv[j] = 0.f;
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const int cc = (c + t) & 7;
-                    const uint4 kr = *reinterpret_cast<const uint4*>(krow + cc * 8);
-                    const float kf[8] = {bf16_lo(kr.x), bf16_hi(kr.x), bf16_lo(kr.y), bf16_hi(kr.y),
-                                         bf16_lo(kr.z), bf16_hi(kr.z), bf16_lo(kr.w), bf16_hi(kr.w)};
-#pragma unroll
-                    for (int j = 0; j < MT; ++j) {
-                        const float4 q0 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8);
-                        const float4 q1 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8 + 4);
-                        float v = scv[j];
-                        v = fmaf(q0.x, kf[0], v); v = fmaf(q0.y, kf[1], v);
-                        v = fmaf(q0.z, kf[2], v); v = fmaf(q0.w, kf[3], v);
-                        v = fmaf(q1.x, kf[4], v); v = fmaf(q1.y, kf[5], v);
-                        v = fmaf(q1.z, kf[6], v); v = fmaf(q1.w, kf[7], v);
-                        scv[j] = v;
+                    for (int ks = 0; ks < 4; ++ks) {
+                        uint32_t b[4];
+                        ldsm_x4(b, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & 7)) << 4));
+                        const uint32_t ah[4] = {qhi[ks][0], 0u, qhi[ks][1], 0u};
+                        const uint32_t al[4] = {qlo[ks][0], 0u, qlo[ks][1], 0u};
+                        const uint32_t b0[2] = {b[0], b[1]}, b1[2] = {b[2], b[3]};
+                        mma_bf16(sfr[0], ah, b0);
+                        mma_bf16(sfr[0], al, b0);
+                        mma_bf16(sfr[1], ah, b1);
+                        mma_bf16(sfr[1], al, b1);
                     }
                 }
-                const int kp = bp * P + t;
+                // this lane's scores: row qrow, keys kt + {c2, c2 + 1, 8 + c2, 9 + c2} of the batch
+                float sv[4] = {sfr[0][0], sfr[0][1], sfr[1][0], sfr[1][1]};
+                float tmax = -INFINITY;
 #pragma unroll
-                for (int j = 0; j < MT; ++j) {
-                    const bool vis = j < a.M && s_seq[j] >= 0 && j / rpg == g && kp <= s_pos[j] && kp < K_tot;
-                    sc[j * SC_STRIDE + t] = vis ? scv[j] : -INFINITY;
+                for (int i = 0; i < 4; ++i) {
+                    const int kp = bp * P + kt + (i >> 1) * 8 + c2 + (i & 1);
+                    const bool vis = qon && qgrp == g && kp <= qpos && kp < K_tot;
+                    sv[i] = vis ? sv[i] : -INFINITY;
+                    tmax = fmaxf(tmax, sv[i]);
                 }
-            }
-            __syncthreads();
-            // softmax statistics: every warp of a row reads all of the row's scores
-            const bool mine = row_on && grp_j == g;
-            float* pr = sc + row_j * SC_STRIDE;
-            float m_new = m_run, corr = 1.f, lsum = 0.f;
-            if (mine) {
-                float bmax = -INFINITY;
-                for (int t = lane; t < nk; t += 32) bmax = fmaxf(bmax, pr[t]);
-                m_new = fmaxf(m_run, warp_max(bmax));
-                if (m_new != -INFINITY) {
-                    corr = expf(m_run - m_new);
-                    for (int t = lane; t < nk; t += 32) lsum += expf(pr[t] - m_new);
-                    lsum = warp_sum(lsum);
-                }
-            }
-            __syncthreads();  // scores read: each warp may now overwrite its own key range
-            if (mine && m_new != -INFINITY) {
-                const int kend = min(nk, pos_j - bp * P + 1);
-                const int chunk = (kend + WPR - 1) / WPR;
-                const int kb = min(kend, row_part * chunk), ke = min(kend, kb + chunk);
-                for (int t = kb + lane; t < ke; t += 32) pr[t] = expf(pr[t] - m_new);
-                l_run = l_run * corr + lsum;
-                acc0 *= corr;
-                acc1 *= corr;
+                tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 1));
+                tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 2));
+                const float m_new = fmaxf(m_run, tmax);
+                const float corr = m_new == -INFINITY ? 1.f : (m_run == -INFINITY ? 0.f : expf(m_run - m_new));
+                float pv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) pv[i] = sv[i] == -INFINITY ? 0.f : expf(sv[i] - m_new);
+                l_run = l_run * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
                 m_run = m_new;
-                __syncwarp();
-                float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
-                for (int p0 = kb; p0 < ke;) {  // page by page
-                    const int pg = p0 / P;
-                    const __nv_bfloat16* vpage = slot_keys(pg) + P * HEAD_DIM + 2 * lane;
-                    const int pend = min(ke, (pg + 1) * P);
-                    int t = p0;
-                    for (; t + 4 <= pend; t += 4) {
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const float p = pr[t + u];
-                            const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t + u - pg * P) * HEAD_DIM);
-                            a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
-                            a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
-                        }
-                    }
-                    for (; t < pend; ++t) {
-                        const float p = pr[t];
-                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(vpage + (t - pg * P) * HEAD_DIM);
-                        a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
-                        a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
-                    }
-                    p0 = pend;
+                for (int j = 0; j < 8; ++j) {
+                    o[j][0] *= corr;
+                    o[j][1] *= corr;
                 }
-                acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
-                acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
+                uint32_t ph[4] = {0u, 0u, 0u, 0u}, pl[4] = {0u, 0u, 0u, 0u};
+                split_bf16x2(pv[0], pv[1], ph[0], pl[0]);
+                split_bf16x2(pv[2], pv[3], ph[2], pl[2]);
+                const int vkey = r0 + (lane & 7) + (((lane >> 3) & 1) << 3), vhalf = lane >> 4;
+#pragma unroll
+                for (int dp = 0; dp < 4; ++dp) {
+                    uint32_t v[4];
+                    ldsm_x4_t(v, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & 7)) << 4));
+                    const uint32_t v0[2] = {v[0], v[1]}, v1[2] = {v[2], v[3]};
+                    mma_bf16(o[2 * dp], ph, v0);
+                    mma_bf16(o[2 * dp], pl, v0);
+                    mma_bf16(o[2 * dp + 1], ph, v1);
+                    mma_bf16(o[2 * dp + 1], pl, v1);
+                }
             }
         }
     }
+    // merge the warps' (max, sum, out) states into part through the weight
+    // area (free once every warp is past its last tile): [NWARPS][MT][PARTW]
+    l_run += __shfl_xor_sync(FULL_MASK, l_run, 1);
+    l_run += __shfl_xor_sync(FULL_MASK, l_run, 2);
     __syncthreads();
-    float* pvred = reinterpret_cast<float*>(smem + L.pvred);  // [NWARPS][64]: P.V of each warp's key range
-    if (WPR > 1 && row_j < MT) {
-        pvred[warp * HEAD_DIM + 2 * lane] = acc0;
-        pvred[warp * HEAD_DIM + 2 * lane + 1] = acc1;
+    float* wst = reinterpret_cast<float*>(smem + L.wqkv);
+    if (qrow < MT) {
+        float* ws = wst + ((size_t)warp * MT + qrow) * PARTW;
+        if (c2 == 0) {
+            ws[0] = m_run;
+            ws[1] = l_run;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) *reinterpret_cast<float2*>(ws + 2 + j * 8 + c2) = make_float2(o[j][0], o[j][1]);
     }
     __syncthreads();
-    if (row_j < MT && row_part == 0) {
-        float* pj = part + row_j * PARTW;
-        if (lane == 0) {
-            pj[0] = m_run;
-            pj[1] = l_run;
+    for (int i = tid; i < MT * (2 + HEAD_DIM); i += NTHREADS) {
+        const int m = i / (2 + HEAD_DIM), c = i % (2 + HEAD_DIM);
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NWARPS; ++w) M = fmaxf(M, wst[((size_t)w * MT + m) * PARTW]);
+        float y = M;
+        if (c > 0) {
+            y = 0.f;
+            if (M != -INFINITY) {
+#pragma unroll
+                for (int w = 0; w < NWARPS; ++w) {
+                    const float* ws = wst + ((size_t)w * MT + m) * PARTW;
+                    if (ws[0] != -INFINITY) y = fmaf(expf(ws[0] - M), ws[c], y);
+                }
+            }
         }
-        for (int w = 1; w < WPR; ++w) {
-            acc0 += pvred[(warp + w) * HEAD_DIM + 2 * lane];
-            acc1 += pvred[(warp + w) * HEAD_DIM + 2 * lane + 1];
-        }
-        pj[2 + 2 * lane] = acc0;
-        pj[3 + 2 * lane] = acc1;
+        part[m * PARTW + c] = y;
     }
+    __syncthreads();
 
     trace_mark(a.trace, 5);  // attention partials done
     // ---- 5. merge the splits (DSMEM) and apply this CTA's W_o rows ----
     cluster.sync();
     trace_mark(a.trace, 6);
-    if (row_on && row_part == 0) {
+    const int row_j = warp;  // warp m merges fed row m
+    const bool row_on = row_j < MT && row_j < a.M && s_seq[min(row_j, MT - 1)] >= 0;
+    if (row_on) {
         float ms = -INFINITY, ls = 0.f, o0[CA], o1[CA];
 #pragma unroll
         for (int r = 0; r < CA; ++r) {
@@ -862,7 +929,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         }
         attn[row_j * HEAD_DIM + 2 * lane] = r0 / Lsum;
         attn[row_j * HEAD_DIM + 2 * lane + 1] = r1 / Lsum;
-    } else if (row_j < MT && row_part == 0) {
+    } else if (row_j < MT) {
         attn[row_j * HEAD_DIM + 2 * lane] = 0.f;
         attn[row_j * HEAD_DIM + 2 * lane + 1] = 0.f;
     }
@@ -870,22 +937,28 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     if (BF) {  // head output as bf16, then W_o rows on the tensor cores
         __nv_bfloat16* ab = reinterpret_cast<__nv_bfloat16*>(smem + L.attn_b);  // [MT][64 + 8]
         float* ytile = reinterpret_cast<float*>(smem + L.ytile);                  // [MT][orows]
-        for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS)
-            ab[(i / HEAD_DIM) * (HEAD_DIM + 8) + i % HEAD_DIM] = __float2bfloat16_rn(attn[i]);
+        for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS) {
+            const __nv_bfloat16 hi = __float2bfloat16_rn(attn[i]);
+            const int at = (i / HEAD_DIM) * (HEAD_DIM + 8) + i % HEAD_DIM;
+            ab[at] = hi;
+            ab[MT * (HEAD_DIM + 8) + at] = __float2bfloat16_rn(attn[i] - __bfloat162float(hi));
+        }
         __syncthreads();
         mma_rows_tiles<MT>(wo, orows, HEAD_DIM, 0, ab, ytile);
         __syncthreads();
-        for (int o = tid; o < orows * MT; o += NTHREADS) {
+#pragma unroll
+        for (int k = 0; k < RES_N; ++k) {
+            const int o = tid + k * NTHREADS;
             const int m = o / orows, t = o % orows;  // a warp adds 32 consecutive floats
-            if (m >= a.M || s_seq[m] < 0) continue;
-            float y = ytile[o];
-            if (h == 0) y += res[m * orows + t];
-            atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
+            if (o >= orows * MT || m >= a.M || s_seq[m] < 0) continue;
+            atomicAdd(a.x_out + (size_t)m * d + s * orows + t, ytile[o] + resr[k]);
         }
     } else {
-        for (int o = tid; o < orows * MT; o += NTHREADS) {
+#pragma unroll
+        for (int k = 0; k < RES_N; ++k) {
+            const int o = tid + k * NTHREADS;
             const int m = o / orows, t = o % orows;  // fed row m, W_o row t: a warp adds 32 consecutive floats
-            if (m >= a.M || s_seq[m] < 0) continue;
+            if (o >= orows * MT || m >= a.M || s_seq[m] < 0) continue;
             const WT* wr = wo + (size_t)t * HEAD_DIM;
             float acc[4] = {0.f, 0.f, 0.f, 0.f};  // four independent chains
 #pragma unroll
@@ -901,8 +974,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 v = fmaf(w4[3], av.w, v);
                 acc[c & 3] = v;
             }
-            float y = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-            if (h == 0) y += res[m * orows + t];
+            const float y = (acc[0] + acc[1]) + (acc[2] + acc[3]) + resr[k];
             atomicAdd(a.x_out + (size_t)m * d + s * orows + t, y);
         }
     }
@@ -937,7 +1009,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     const int rpad = L.rpad;
     __nv_bfloat16* xb = reinterpret_cast<__nv_bfloat16*>(smem + L.xb);
     float* accs = reinterpret_cast<float*>(smem + L.accs);
-    __nv_bfloat16* ub = reinterpret_cast<__nv_bfloat16*>(smem + L.ub);  // [MT][rpad + 8]
+    __nv_bfloat16* ub = reinterpret_cast<__nv_bfloat16*>(smem + L.ub);  // hi, lo: [MT][rpad + 8] each
     float* ypart = reinterpret_cast<float*>(smem + L.ypart);  // [MT][d]
     float* red = reinterpret_cast<float*>(smem + L.red);
     const bool first_cluster = blockIdx.x < CB;
@@ -1012,8 +1084,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     zero_slice(a.x_zero, (size_t)MAX_ROWS * d, blockIdx.x, gridDim.x);
     layer_norm_rows<MT>(xr, d, gam, bet, a.ln_eps, ln_part, ln_stat);
     if (BF) {
-        store_rows_bf16<MT>(xr, d, xb);
-        for (int i = tid; i < rpc * 8; i += NTHREADS) accs[i] = 0.f;
+        store_rows_split<MT>(xr, d, xb);
     }
 
     trace_mark(a.trace, 0);  // inputs loaded, LN2 done
@@ -1028,14 +1099,16 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     trace_mark(a.trace, 1);  // weights in shared memory
     if (BF) {
         // u = GELU(LN2(x) W1^T + b1) for this CTA's FFN rows, as bf16 [MT][rpad]
-        if (R > 0) mma_rows_ksplit<MT>(w1, R, d, f0, xb, accs);
+        if (R > 0) mma_rows_ksplit<MT>(w1, R, d, f0, xb, red, accs);
         __syncthreads();
         for (int k = 0; k < 2; ++k) {
             const int o = tid + k * NTHREADS;
             if (o >= MT * rpad) continue;
             const int m = o / rpad, f = o % rpad;
-            const float v = f < R ? gelu_erf(accs[f * 8 + m] + b1v[k]) : 0.f;
-            ub[m * (rpad + 8) + f] = __float2bfloat16_rn(v);
+            const float v = f < R ? gelu_erf(accs[f * MT + m] + b1v[k]) : 0.f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+            ub[m * (rpad + 8) + f] = hi;
+            ub[(MT + m) * (rpad + 8) + f] = __float2bfloat16_rn(v - __bfloat162float(hi));
         }
         __syncthreads();
         trace_mark(a.trace, 2);  // u done
