@@ -83,7 +83,7 @@ cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool
 // One transformer block over <= MAX_ROWS fed rows: attn_block (LN1, q|k|v,
 // key/value append, attention, W_o) and mlp (LN2, W1, GELU, W2), each
 // accumulating into a zeroed residual buffer.
-constexpr int MLP_CLUSTER = 8;   // CTAs per cluster of the MLP kernel
+constexpr int MLP_CLUSTER = 4;   // CTAs per cluster of the MLP kernel (4: 36 clusters fit one CTA per SM)
 
 struct LayerArgs {
     const float* x_in;        // [M][d] input rows of the kernel

@@ -39,7 +39,10 @@ namespace {
 
 constexpr int CA = 8;                    // CTAs per head (cluster of kernel A)
 constexpr int QROWS = 3 * HEAD_DIM / CA;  // projection rows per CTA (24)
-constexpr int MIN_TILE = 64;              // keys staged per batch: at least this many, whole pages
+constexpr int MAX_PRE_KEYS = 192;         // cached keys per CTA staged before the dependency wait
+// dynamic shared memory of kernel A: small enough for two CTAs per SM (16
+// clusters of 8 fit at once only so)
+constexpr size_t A_SMEM_CAP = 113664;
 constexpr int PARTW = 2 + HEAD_DIM;       // (max, sum, out[64])
 constexpr int NTHREADS = 256;
 constexpr int NWARPS = NTHREADS / 32;
@@ -48,43 +51,49 @@ __host__ __device__ inline size_t al128(size_t x) { return (x + 127) & ~(size_t)
 
 // ---- shared-memory layouts (host and device compute the same offsets) ----
 struct ALayout {
-    size_t wqkv, wo, ks, qkvp, qkvf, qs, part, attn, uni, total;
-    size_t xb, red, attn_b, ytile;  // inside the union (phases do not overlap)
+    size_t wqkv, ks, wo, qkvp, qkvf, part, attn, uni, total;
+    size_t xb, red, attn_b, ytile;  // xb and red share W_o's space; attn_b, ytile the union
     int tile;  // keys of the dedicated staging slots (filled before the dependency wait)
     __host__ __device__ ALayout(int d, int wbytes, int mt, int page) {
-        const int groups = (QROWS * mt + 31) / 32;
         const size_t wq_bytes = (size_t)QROWS * d * wbytes, slot_bytes = (size_t)2 * page * HEAD_DIM * 2;
-        // whole pages, at least MIN_TILE keys; none at 8 rows when the weight area holds a page
-        // (the 8-row inputs need the space; every page then arrives after the projection)
-        tile = mt >= 8 && wq_bytes >= slot_bytes ? 0 : (MIN_TILE + page - 1) / page * page;
-        // the q|k|v slice and the dedicated page slots are adjacent: after the
-        // attention they hold the warps' softmax states [NWARPS][mt][PARTW]
-        size_t ks_bytes = (size_t)2 * tile * HEAD_DIM * 2;
+        // dedicated page slots: as many whole pages as keep two CTAs per SM (at most
+        // MAX_PRE_KEYS keys), and one at least when the weight area holds no page
+        place(d, wbytes, mt, wq_bytes, 0);
+        int pages = total < A_SMEM_CAP ? (int)((A_SMEM_CAP - total) / slot_bytes) : 0;
+        pages = min(pages, max(1, MAX_PRE_KEYS / page));
+        if (wq_bytes < slot_bytes) pages = max(pages, 1);
+        tile = pages * page;
+        // the q|k|v slice and the dedicated slots are adjacent: after the attention
+        // they hold the warps' softmax states [NWARPS][mt][PARTW]
+        size_t ks_bytes = (size_t)pages * slot_bytes;
         const size_t merge_bytes = (size_t)NWARPS * mt * PARTW * 4;
         if (wq_bytes + ks_bytes < merge_bytes) ks_bytes = merge_bytes - wq_bytes;
+        place(d, wbytes, mt, wq_bytes, ks_bytes);
+    }
+    __host__ __device__ void place(int d, int wbytes, int mt, size_t wq_bytes, size_t ks_bytes) {
+        const int groups = (QROWS * mt + 31) / 32;
         wqkv = 0;
         ks = al128(wqkv + wq_bytes);  // page slots: [keys | values] each
+        // W_o's slice arrives after the projection; until then its space holds the
+        // bf16 hi/lo inputs and then the warps' tile sums (tensor cores), or the
+        // reduce-scatter scratch (fp32)
         wo = al128(ks + ks_bytes);
-        qkvp = al128(wo + (size_t)(d / CA) * HEAD_DIM * wbytes);
+        xb = wo;
+        red = wo;
+        size_t xbytes = (size_t)(d / CA) * HEAD_DIM * wbytes;
+        const size_t ibytes = (size_t)2 * mt * (d + 8) * 2;
+        const size_t rbytes = wbytes == 2 ? (size_t)NWARPS * QROWS * 8 * 4 : (size_t)NWARPS * groups * 32 * 4;
+        if (ibytes > xbytes) xbytes = ibytes;
+        if (rbytes > xbytes) xbytes = rbytes;
+        qkvp = al128(wo + xbytes);
         qkvf = al128(qkvp + (size_t)QROWS * mt * 4);
-        qs = al128(qkvf + (size_t)3 * HEAD_DIM * mt * 4);
-        part = al128(qs + (size_t)mt * HEAD_DIM * 4);
+        part = al128(qkvf + (size_t)3 * HEAD_DIM * mt * 4);
         attn = al128(part + (size_t)mt * PARTW * 4);
         uni = al128(attn + (size_t)mt * HEAD_DIM * 4);
-        // projection: bf16 hi/lo inputs, then (same space) the warps' tile sums (tensor cores),
-        // or the reduce-scatter scratch (fp32); qkvf, qs, part and attn are written only after
-        // the projection, so it may start there
-        xb = qkvf;
-        red = xb;  // the tile sums are reduced into qkvp, outside this space
-        size_t xbytes = (size_t)2 * mt * (d + 8) * 2;
-        const size_t rbytes = wbytes == 2 ? (size_t)NWARPS * QROWS * 8 * 4 : (size_t)NWARPS * groups * 32 * 4;
-        if (rbytes > xbytes) xbytes = rbytes;
-        const size_t p1 = xb + xbytes;
         // output projection: bf16 hi/lo head output, projected rows
         attn_b = uni;
         ytile = al128(attn_b + (size_t)2 * mt * (HEAD_DIM + 8) * 2);
-        const size_t p3 = ytile + (size_t)mt * (d / CA) * 4;
-        total = al128(p1 > p3 ? p1 : p3);
+        total = al128(ytile + (size_t)mt * (d / CA) * 4);
     }
 };
 
@@ -97,12 +106,16 @@ struct BLayout {
         rpad = (rows + 15) / 16 * 16;
         w1 = 0;
         w2 = al128(w1 + (size_t)rows * d * wbytes);
+        // bf16 hi/lo inputs, then (same space) the warps' tile sums; fp32: the reduce-scatter scratch
         xb = al128(w2 + (size_t)rows * d * wbytes);
-        accs = al128(xb + (size_t)2 * mt * (d + 8) * 2);
-        ub = al128(accs + (size_t)rows * 8 * 4);
-        u = al128(ub + (size_t)2 * mt * (rpad + 8) * 2);
-        red = al128(u + (wbytes == 2 ? 0 : (size_t)rows * mt * 4));
-        size_t end = al128(red + (wbytes == 2 ? (size_t)NWARPS * rows * 8 * 4 : (size_t)NWARPS * groups * 32 * 4));
+        red = xb;
+        size_t xbytes = wbytes == 2 ? (size_t)2 * mt * (d + 8) * 2 : 0;
+        const size_t rbytes = wbytes == 2 ? (size_t)NWARPS * rows * 8 * 4 : (size_t)NWARPS * groups * 32 * 4;
+        if (rbytes > xbytes) xbytes = rbytes;
+        accs = al128(xb + xbytes);                      // [rows][mt] FFN pre-activations
+        ub = al128(accs + (size_t)rows * mt * 4);        // bf16 hi/lo GELU outputs
+        u = al128(ub + (size_t)2 * mt * (rpad + 8) * 2);  // fp32 GELU outputs
+        size_t end = al128(u + (wbytes == 2 ? 0 : (size_t)rows * mt * 4));
         const size_t ybytes = (size_t)mt * d * 4;
         // the partial outputs reuse W1's space once u is known, when it fits
         if ((size_t)rows * d * wbytes >= ybytes) {
@@ -174,12 +187,13 @@ __device__ __forceinline__ void mma_rows_ksplit(const void* w, int R, int K, int
     const int brow = (lane & 7) < MT ? (lane & 7) : 0;  // tokens past MT repeat token 0 (ignored)
     const int bhalf = (lane >> 3) & 1;
     const int arow = lane & 15, ahalf = lane >> 4;
-    float acc[4][4];
+    float acc[4][4], accl[4][4];  // hi and lo products in separate chains
 #pragma unroll
     for (int t = 0; t < 4; ++t)
 #pragma unroll
-        for (int i = 0; i < 4; ++i) acc[t][i] = 0.f;
+        for (int i = 0; i < 4; ++i) acc[t][i] = accl[t][i] = 0.f;
     const uint32_t xlo = (uint32_t)MT * xstride;
+#pragma unroll 2
     for (int k0 = warp * kslice; k0 < (warp + 1) * kslice; k0 += 16) {
         uint32_t bh[2], bl[2];
         ldsm_x2(bh, xbase + brow * xstride + (k0 + bhalf * 8) * 2);
@@ -191,10 +205,14 @@ __device__ __forceinline__ void mma_rows_ksplit(const void* w, int R, int K, int
                 uint32_t a[4];
                 ldsm_x4(a, wchunk(wb, row, row_bytes, (k0 >> 3) + ahalf, key0 + row));
                 mma_bf16(acc[t], a, bh);
-                mma_bf16(acc[t], a, bl);
+                mma_bf16(accl[t], a, bl);
             }
         }
     }
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[t][i] += accl[t][i];
     __syncthreads();  // every warp is done with x
     const int g = lane >> 2, c2 = (lane & 3) * 2;
     float* mine = wpart + (size_t)warp * R * 8;
@@ -496,6 +514,7 @@ __device__ __forceinline__ int issue_pages(const LayerArgs& a, int seq, int bp, 
     for (int p = first; p < nb; ++p)
         if (a.block_table[(size_t)seq * a.bt_stride + bp + p] >= 0) bytes += (uint32_t)slot_elems * 2;
     if (!bytes) return 0;
+    fence_proxy_async();  // the slots were last read by this CTA's threads
     mbar_arrive_expect_tx(bar, bytes);
     for (int p = first; p < nb; ++p) {
         const int phys = a.block_table[(size_t)seq * a.bt_stride + bp + p];
@@ -522,6 +541,8 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     __shared__ int s_seq[MT], s_pos[MT], s_page[MT];
     __shared__ int s_gseq[MT], s_gold[MT], s_gktot[MT];
     __shared__ int s_pre, s_armed;
+    __shared__ uint64_t bar_o;  // W_o slice, requested after the projection
+    __shared__ float s_scale[NWARPS][MT];
     TraceEnd trace_guard(a.trace);
     cg::cluster_group cluster = cg::this_cluster();
 
@@ -536,7 +557,6 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem + L.ks);
     float* qkvp = reinterpret_cast<float*>(smem + L.qkvp);  // [QROWS][MT]
     float* qkvf = reinterpret_cast<float*>(smem + L.qkvf);  // [192][MT]
-    float* qs = reinterpret_cast<float*>(smem + L.qs);      // [MT][64]
     float* part = reinterpret_cast<float*>(smem + L.part);  // [MT][PARTW]
     float* attn = reinterpret_cast<float*>(smem + L.attn);  // [MT][64]
     float* red = reinterpret_cast<float*>(smem + L.red);
@@ -561,6 +581,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     }
     if (tid == 0) {
         mbar_init(&bar, 1);
+        mbar_init(&bar_o, 1);
         fence_barrier_init();
         s_pre = 0;
     }
@@ -583,7 +604,6 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     __syncthreads();
     if (tid == 0) {
         const uint32_t wq = (uint32_t)QROWS * d * sizeof(WT);
-        const uint32_t wob = (uint32_t)orows * HEAD_DIM * sizeof(WT);
         uint32_t kvb = 0;
         int n_pre = 0, pg0 = 0;
         const int seq = s_gseq[0];
@@ -593,18 +613,17 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
             const int pps = (n_pg + CA - 1) / CA;
             pg0 = s * pps;
             const int pg1 = min(n_pg, pg0 + pps);
-            int pre_end = min(min(pg1, pg0 + ATT_TILE / P), old_len / P);
+            (void)old_len;  // rows of the fed keys are filled in shared memory after the copy
+            int pre_end = min(pg1, pg0 + ATT_TILE / P);
             for (int p = pg0; p < pre_end; ++p)
                 if (a.block_table[(size_t)seq * a.bt_stride + p] < 0) pre_end = p;
             n_pre = max(0, pre_end - pg0);
             kvb = 2u * (uint32_t)n_pre * P * HEAD_DIM * 2;
         }
-        mbar_arrive_expect_tx(&bar, wq + wob + kvb);
+        mbar_arrive_expect_tx(&bar, wq + kvb);
         const char* srcq = reinterpret_cast<const char*>(a.wqkv) + ((size_t)h * 3 * HEAD_DIM + s * QROWS) * d * sizeof(WT);
         for (uint32_t off = 0; off < wq; off += 32768)
             bulk_copy_g2s(smem + L.wqkv + off, srcq + off, min(32768u, wq - off), &bar);
-        const char* srco = reinterpret_cast<const char*>(a.wo) + ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT);
-        bulk_copy_g2s(smem + L.wo, srco, wob, &bar);
         for (int i = 0; i < n_pre; ++i) {
             const int phys = a.block_table[(size_t)seq * a.bt_stride + pg0 + i];
             const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
@@ -613,11 +632,18 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                           &bar);
         }
         s_pre = n_pre;
-        if (seq >= 0) {  // the split's other cached pages, into L2 (copied to shared memory later)
+    } else if (tid == 32) {  // L2 prefetches, issued beside the copies above
+        const uint32_t wq = (uint32_t)QROWS * d * sizeof(WT);
+        const uint32_t wob = (uint32_t)orows * HEAD_DIM * sizeof(WT);
+        const size_t offq = ((size_t)h * 3 * HEAD_DIM + s * QROWS) * d * sizeof(WT);
+        const size_t offo = ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT);
+        prefetch_l2(reinterpret_cast<const char*>(a.wo) + offo, wob);  // copied after the projection
+        const int seq = s_gseq[0];
+        if (seq >= 0) {  // the split's cached pages past the staged ones (copied to shared memory later)
             const int n_pg = (s_gktot[0] + P - 1) / P;
             const int pps = (n_pg + CA - 1) / CA;
-            const int pg1 = min(n_pg, pg0 + pps);
-            for (int p = pg0 + n_pre; p < pg1; ++p) {
+            const int pg0 = s * pps, pg1 = min(n_pg, pg0 + pps);
+            for (int p = pg0 + ATT_TILE / P; p < pg1; ++p) {
                 const int phys = a.block_table[(size_t)seq * a.bt_stride + p];
                 if (phys < 0) continue;
                 const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
@@ -626,11 +652,11 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
             }
         }
         if (a.next_w_a) {  // the next layer's slices of the same weights, into L2
-            prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + (srcq - reinterpret_cast<const char*>(a.wqkv)), wq);
-            prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + (srco - reinterpret_cast<const char*>(a.wo)), wob);
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + offq, wq);
+            prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + offo, wob);
         }
     }
-    float gam[4], bet[4], bq[2] = {0.f, 0.f};
+    float gam[4], bet[4], bq[1] = {0.f};
     {
         const int Kw = d / NWARPS;
         if (lane * 4 < Kw) {
@@ -640,10 +666,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
 #pragma unroll
             for (int i = 0; i < 4; ++i) gam[i] = bet[i] = 0.f;
         }
-        for (int u = 0; u < 2; ++u) {
-            const int o = tid + u * NTHREADS;
-            if (o < QROWS * MT) bq[u] = __ldg(a.bqkv + h * 3 * HEAD_DIM + s * QROWS + o / MT);
-        }
+        if (tid < QROWS * MT) bq[0] = __ldg(a.bqkv + h * 3 * HEAD_DIM + s * QROWS + tid / MT);
     }
 
     pdl_launch_dependents();
@@ -682,7 +705,33 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     } else {
         project_rows<WT, MT>(wqkv, QROWS, d, xr, red, qkvp);
     }
-    if (tid == 0) {  // group 0's first batch of cached pages into the slots, while the cluster gathers
+    // q|k|v rows with bias (QROWS * MT <= NTHREADS: one per thread), released to the cluster
+    const bool has_row = tid < QROWS * MT;
+    const float yrow = has_row ? qkvp[tid] + bq[0] : 0.f;
+    if (has_row) qkvp[tid] = yrow;
+    cluster_arrive_release();
+    if (has_row) {
+        const int row = s * QROWS + tid / MT, m = tid % MT;  // row within the head's q|k|v
+        if (row >= HEAD_DIM && s_seq[m] >= 0) {               // key or value: append to the cache
+            const int sec = row / HEAD_DIM, dd = row % HEAD_DIM;
+            const int page = s_page[m];
+            if (page < 0) {
+                atomicOr(a.err, ERR_BOUNDS);
+            } else {
+                const int t = s_pos[m] % P;  // key row of the page; its 16-byte chunks are stored swizzled
+                const long long idx = (long long)page * a.page_elems + a.layer_off + (sec - 1) * v_off + kv_head +
+                                      (long long)t * HEAD_DIM + kv_col(t, dd);
+                reinterpret_cast<uint16_t*>(a.kv_pool)[idx] = f32_to_bf16_bits(yrow);
+            }
+        }
+    }
+    if (tid == 0) {  // W_o's slice, and group 0's first batch of cached pages, while the cluster gathers
+        fence_proxy_async();  // the spaces were last written and read by this CTA's threads
+        const uint32_t wob = (uint32_t)orows * HEAD_DIM * sizeof(WT);
+        mbar_arrive_expect_tx(&bar_o, wob);
+        bulk_copy_g2s(smem + L.wo,
+                      reinterpret_cast<const char*>(a.wo) + ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT),
+                      wob, &bar_o);
         s_armed = 0;
         const int seq = s_gseq[0];
         if (seq >= 0) {
@@ -693,27 +742,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                                       wq_slots, n_ded, &bar);
         }
     }
-    for (int o = tid; o < QROWS * MT; o += NTHREADS) {
-        const float y = qkvp[o] + (o < NTHREADS ? bq[0] : bq[1]);
-        qkvp[o] = y;
-        const int row = s * QROWS + o / MT, m = o % MT;  // row within the head's q|k|v
-        if (row >= HEAD_DIM && s_seq[m] >= 0) {             // key or value: append to the cache
-            const int sec = row / HEAD_DIM, dd = row % HEAD_DIM;
-            const int page = s_page[m];
-            if (page < 0) {
-                atomicOr(a.err, ERR_BOUNDS);
-                continue;
-            }
-            const int t = s_pos[m] % P;  // key row of the page; its 16-byte chunks are stored swizzled
-            const long long idx = (long long)page * a.page_elems + a.layer_off + (sec - 1) * v_off + kv_head +
-                                  (long long)t * HEAD_DIM + kv_col(t, dd);
-            reinterpret_cast<uint16_t*>(a.kv_pool)[idx] = f32_to_bf16_bits(y);
-        }
-    }
-
     trace_mark(a.trace, 2);  // projection rows done
     // ---- 3. gather the head's q, k, v of the fed rows from the cluster ----
-    cluster.sync();
+    cluster_wait();
     trace_mark(a.trace, 3);
     {
         constexpr int PER = (3 * HEAD_DIM * MT + NTHREADS - 1) / NTHREADS;
@@ -724,7 +755,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
             v[u] = 0.f;
             if (i < 3 * HEAD_DIM * MT) {
                 const int row = i / MT;
-                v[u] = cluster.map_shared_rank(qkvp, row / QROWS)[(row % QROWS) * MT + i % MT];
+                v[u] = ld_dsmem(dsmem_addr(qkvp + (row % QROWS) * MT + i % MT, row / QROWS));
             }
         }
 #pragma unroll
@@ -735,10 +766,6 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         }
     }
     __syncthreads();
-    for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS) {
-        const int m = i / HEAD_DIM, dd = i % HEAD_DIM;
-        qs[i] = s_seq[m] >= 0 ? qkvf[dd * MT + m] * 0.125f : 0.f;  // 1/sqrt(64)
-    }
 
     trace_mark(a.trace, 4);  // gathered
     // ---- 4. attention over this CTA's split of each group's keys ----
@@ -756,7 +783,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             const int k = ks * 16 + hh * 8 + c2;
-            const float q0 = qon ? qs[qrow * HEAD_DIM + k] : 0.f, q1 = qon ? qs[qrow * HEAD_DIM + k + 1] : 0.f;
+            // the query scaled by 1/sqrt(64) (exact in binary)
+            const float q0 = qon ? qkvf[k * MT + qrow] * 0.125f : 0.f;
+            const float q1 = qon ? qkvf[(k + 1) * MT + qrow] * 0.125f : 0.f;
             split_bf16x2(q0, q1, qhi[ks][hh], qlo[ks][hh]);
         }
     float m_run = -INFINITY, l_run = 0.f;
@@ -807,6 +836,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                 const int r0 = kt % P;  // first key row of the tile in its page
                 const uint32_t kb = smem_addr(slot_keys(kt / P)), vb = kb + P * HEAD_DIM * 2;
                 float sfr[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+                float sfl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // lo parts: own chains
                 {
                     const int key = r0 + (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
 #pragma unroll
@@ -817,13 +847,14 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
                         const uint32_t al[4] = {qlo[ks][0], 0u, qlo[ks][1], 0u};
                         const uint32_t b0[2] = {b[0], b[1]}, b1[2] = {b[2], b[3]};
                         mma_bf16(sfr[0], ah, b0);
-                        mma_bf16(sfr[0], al, b0);
+                        mma_bf16(sfl[0], al, b0);
                         mma_bf16(sfr[1], ah, b1);
-                        mma_bf16(sfr[1], al, b1);
+                        mma_bf16(sfl[1], al, b1);
                     }
                 }
                 // this lane's scores: row qrow, keys kt + {c2, c2 + 1, 8 + c2, 9 + c2} of the batch
-                float sv[4] = {sfr[0][0], sfr[0][1], sfr[1][0], sfr[1][1]};
+                float sv[4] = {sfr[0][0] + sfl[0][0], sfr[0][1] + sfl[0][1], sfr[1][0] + sfl[1][0],
+                               sfr[1][1] + sfl[1][1]};
                 float tmax = -INFINITY;
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
@@ -879,22 +910,21 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         for (int j = 0; j < 8; ++j) *reinterpret_cast<float2*>(ws + 2 + j * 8 + c2) = make_float2(o[j][0], o[j][1]);
     }
     __syncthreads();
-    for (int i = tid; i < MT * (2 + HEAD_DIM); i += NTHREADS) {
-        const int m = i / (2 + HEAD_DIM), c = i % (2 + HEAD_DIM);
+    if (tid < NWARPS * MT) {  // weight of warp w's state in row m: exp(max_w - common max)
+        const int w = tid / MT, m = tid % MT;
         float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < NWARPS; ++w) M = fmaxf(M, wst[((size_t)w * MT + m) * PARTW]);
-        float y = M;
-        if (c > 0) {
-            y = 0.f;
-            if (M != -INFINITY) {
+        for (int v = 0; v < NWARPS; ++v) M = fmaxf(M, wst[((size_t)v * MT + m) * PARTW]);
+        const float mw = wst[((size_t)w * MT + m) * PARTW];
+        s_scale[w][m] = mw == -INFINITY ? 0.f : expf(mw - M);
+        if (w == 0) part[m * PARTW] = M;
+    }
+    __syncthreads();
+    for (int i = tid; i < MT * (1 + HEAD_DIM); i += NTHREADS) {
+        const int m = i / (1 + HEAD_DIM), c = 1 + i % (1 + HEAD_DIM);
+        float y = 0.f;
 #pragma unroll
-                for (int w = 0; w < NWARPS; ++w) {
-                    const float* ws = wst + ((size_t)w * MT + m) * PARTW;
-                    if (ws[0] != -INFINITY) y = fmaf(expf(ws[0] - M), ws[c], y);
-                }
-            }
-        }
+        for (int w = 0; w < NWARPS; ++w) y = fmaf(s_scale[w][m], wst[((size_t)w * MT + m) * PARTW + c], y);
         part[m * PARTW + c] = y;
     }
     __syncthreads();
@@ -907,16 +937,17 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     const bool row_on = row_j < MT && row_j < a.M && s_seq[min(row_j, MT - 1)] >= 0;
     if (row_on) {
         float ms = -INFINITY, ls = 0.f, o0[CA], o1[CA];
+        const float* mine = part + row_j * PARTW;
+        float2 st = make_float2(-INFINITY, 0.f);
+        if (lane < CA) st = ld_dsmem2(dsmem_addr(mine, lane));  // (max, sum) of split `lane`
 #pragma unroll
         for (int r = 0; r < CA; ++r) {
-            const float* peer = cluster.map_shared_rank(part, r) + row_j * PARTW;
-            if (lane == r) {
-                ms = peer[0];
-                ls = peer[1];
-            }
-            o0[r] = peer[2 + 2 * lane];
-            o1[r] = peer[3 + 2 * lane];
+            const float2 ov = ld_dsmem2(dsmem_addr(mine + 2 + 2 * lane, r));
+            o0[r] = ov.x;
+            o1[r] = ov.y;
         }
+        ms = st.x;
+        ls = st.y;
         const float M = warp_max(ms);
         const float w = (ms == -INFINITY) ? 0.f : expf(ms - M);
         const float Lsum = warp_sum(lane < CA ? w * ls : 0.f);
@@ -933,8 +964,13 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         attn[row_j * HEAD_DIM + 2 * lane] = 0.f;
         attn[row_j * HEAD_DIM + 2 * lane + 1] = 0.f;
     }
+    cluster_arrive_relaxed();  // done reading the peers' partials (waited for before exiting)
     __syncthreads();
-    if (BF) {  // head output as bf16, then W_o rows on the tensor cores
+    bool okw = mbar_wait(&bar_o, 0, a.err);
+    okw = __syncthreads_and(okw) != 0;
+    if (!okw) {
+        mbar_wait(&bar_o, 0, nullptr);
+    } else if (BF) {  // head output as bf16 hi/lo, then W_o rows on the tensor cores
         __nv_bfloat16* ab = reinterpret_cast<__nv_bfloat16*>(smem + L.attn_b);  // [MT][64 + 8]
         float* ytile = reinterpret_cast<float*>(smem + L.ytile);                  // [MT][orows]
         for (int i = tid; i < MT * HEAD_DIM; i += NTHREADS) {
@@ -979,7 +1015,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         }
     }
     trace_mark(a.trace, 7);  // output projection added
-    cluster.sync();  // peers may still read this CTA's shared memory
+    cluster_wait();  // peers may still read this CTA's shared memory
 }
 
 // ============================================================ kernel B ====
@@ -1034,10 +1070,11 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
             bulk_copy_g2s(smem + L.w1 + off, s1 + off, min(32768u, wb - off), &bar);
             bulk_copy_g2s(smem + L.w2 + off, s2 + off, min(32768u, wb - off), &bar);
         }
-        if (a.next_w_a) {  // the next layer's slices, into L2
-            prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + off0, wb);
-            prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + off0, wb);
-        }
+    } else if (tid == 32 && R > 0 && a.next_w_a) {  // the next layer's slices, into L2
+        const uint32_t wb = (uint32_t)R * d * sizeof(WT);
+        const size_t off0 = (size_t)f0 * d * sizeof(WT);
+        prefetch_l2(reinterpret_cast<const char*>(a.next_w_a) + off0, wb);
+        prefetch_l2(reinterpret_cast<const char*>(a.next_w_b) + off0, wb);
     }
     float gam[4], bet[4], b1v[2] = {0.f, 0.f};
     {
@@ -1160,7 +1197,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
         float4 y = resv[k];
 #pragma unroll
         for (int r = 0; r < CB; ++r) {
-            const float4 p = *reinterpret_cast<const float4*>(cluster.map_shared_rank(ypart, r) + (size_t)m * d + c);
+            const float4 p = ld_dsmem4(dsmem_addr(ypart + (size_t)m * d + c, r));
             y.x += p.x;
             y.y += p.y;
             y.z += p.z;
@@ -1169,7 +1206,8 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
         atomicAdd(reinterpret_cast<float4*>(a.x_out + (size_t)m * d + c), y);
     }
     trace_mark(a.trace, 5);  // cluster sums added
-    cluster.sync();
+    cluster_arrive_relaxed();  // done reading the peers' partials
+    cluster_wait();            // peers may still read this CTA's shared memory
 }
 
 template <typename T>
