@@ -160,18 +160,31 @@ def cpu_baseline(max_steps: int = 60):
                       f"({toks} tokens), float64 numpy, {dt:.1f} s"}
 
 
+KERNEL_SOURCES = ("paper_2410_13839_gb300/csrc/layer_fused.cu", "paper_2410_13839_gb300/csrc/common.cuh",
+                  "paper_2410_13839_gb300/csrc/kernels.cuh")
+
+
+def kernel_source_sha1() -> str:
+    """Hash of the block kernels' sources (the ncu traffic figure is valid only for these)."""
+    h = hashlib.sha1()
+    for rel in KERNEL_SOURCES:
+        h.update(open(os.path.join(ROOT, rel), "rb").read())
+    return h.hexdigest()
+
+
 def _traffic_for(kind: str):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    """DRAM bytes per launch from the committed ncu summary, if the kernel sources are unchanged.
+
+    profiles/traffic.txt holds lines `<kernel kind> <sources sha1> <dram bytes per launch>`."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
-    entry = json.load(open(path)).get(kind)
-    if not entry:
-        return None
-    src = os.path.join(ROOT, entry["source"])
-    if not os.path.exists(src) or hashlib.sha1(open(src, "rb").read()).hexdigest() != entry["source_sha1"]:
-        return None
-    return entry["dram_bytes_per_launch"]
+    sha = kernel_source_sha1()
+    for line in open(path):
+        parts = line.split()
+        if len(parts) == 3 and parts[0] == kind and parts[1] == sha:
+            return int(parts[2])
+    return None
 
 
 def run_reference(args):
