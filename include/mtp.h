@@ -300,6 +300,21 @@ MTP_API int mtp_attention(const mtp_attention_args* args, void* workspace, size_
 #define MTP_ATTENTION_NOALLOC_SCRATCH_BYTES (4u << 20)
 MTP_API int mtp_attention_noalloc(const mtp_attention_args* args, void* cuda_stream);
 
+/* The batched path's tensor-core projection (the block's linear layers,
+ * Sec. III-A, for many fed rows at once):
+ *   out[i][f] (+)= sum_k (a_hi[i][k] + a_lo[i][k]) * w[f][k]
+ * w: device bf16 [n_w][k] row-major; a_hi, a_lo: device bf16 [m][k]
+ * row-major, the two parts of fp32 activations (a_lo = a - a_hi); out:
+ * device fp32 [m][n_w].  n_w a multiple of 128, k a multiple of 64 with
+ * (k / 64) divisible by splits, 1 <= m <= 4096; all pointers 16-byte
+ * aligned.  splits > 1 splits the reduction across CTAs and requires
+ * accumulate = 1 (fp32 atomic adds into out, so the summation order and the
+ * last bits vary between runs); accumulate = 0 stores.  Runs on cuda_stream
+ * and synchronises it before returning.  Errors: MTP_ERR_INVALID (shapes,
+ * alignment), MTP_ERR_CUDA, MTP_ERR_DEVICE (a bounded wait ran out). */
+MTP_API int mtp_gemm_bf16x2(const void* w, const void* a_hi, const void* a_lo, float* out, int n_w, int k, int m,
+                            int splits, int accumulate, void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

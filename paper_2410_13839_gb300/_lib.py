@@ -75,6 +75,7 @@ def _load() -> ctypes.CDLL:
         "mtp_attention_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),
         "mtp_attention": (i32, [ctypes.POINTER(MtpAttentionArgs), vp, sz, vp]),
         "mtp_attention_noalloc": (i32, [ctypes.POINTER(MtpAttentionArgs), vp]),
+        "mtp_gemm_bf16x2": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

@@ -6,6 +6,7 @@
 // depend on it (weights, old keys/values), then waits (griddepcontrol.wait).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -178,6 +179,29 @@ cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStrea
 // copy each slot's last fed row (row_last) of x [MAX_ROWS][d] into h_last [slot][d]
 cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
                              unsigned long long* trace, cudaStream_t s, bool pdl);
+
+// ------------------------------------------------ tensor-core GEMM ----
+// out[n][f] (+)= sum_k (a_hi[n][k] + a_lo[n][k]) w[f][k] with tcgen05 (tc_gemm.cu).
+struct TcGemmArgs {
+    float* out; int ldo;          // [m][ldo] fp32, column f = weight row
+    const float* bias;            // [n_w] added once (by K split 0), or null
+    int m;                        // activation rows
+    int k_chunks;                 // 64-wide k-chunks per CTA (K / 64 / splits)
+    int w_rows_per_kchunk;        // 0: weight k-chunk kc at columns 64 kc; else at rows kc * this (W_o per head)
+    int accumulate;               // 1: atomicAdd into out; 0: store (one K split only)
+    int* err;
+};
+struct TcGemm {
+    CUtensorMap w, a_hi, a_lo;    // boxes: 64 x 128 weight rows, 64 x nt activation rows
+    TcGemmArgs args;
+    int n_w, splits, nt;          // weight rows (multiple of 128), K splits, activation rows per tile
+};
+// 2-D bf16 tensor map [rows][inner] with a 64 x box_rows box; pre_swizzled: the
+// tensor already stores chunk c of row r at c ^ (r & 7) (copied verbatim).
+int tc_encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                 bool pre_swizzled);
+int tc_tile_rows(int m);          // activation rows per tile for m rows: 32, 64 or 128
+cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl);
 
 // C-ABI error reporting shared by the translation units (message for mtp_last_error)
 int report_error(int code, const char* msg);

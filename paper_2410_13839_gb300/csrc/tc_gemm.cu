@@ -1,0 +1,370 @@
+// tc_gemm.cu -- tensor-core GEMM of the batched path (the block's
+// projections, Sec. III-A, once B * n fed rows make them a dense contraction):
+//
+//   out[n][f] (+)= sum_k (a_hi[n][k] + a_lo[n][k]) * w[f][k]
+//
+// w: bf16 weights, K-major ([N_w][K]); a_hi + a_lo: the fp32 activations as
+// two bf16 parts, K-major ([M][K]).  The weights are the MMA's M = 128 side
+// (one 128-row tile per CTA) and the activation rows its N side (NT per
+// tile), so a handful of fed rows still fills the tensor core; both parts of
+// the activations go through the same accumulator (two MMAs per k-step),
+// which keeps the product to fp32 accuracy.
+//
+// Per CTA: one elected thread streams 64-wide k-chunks of the weight tile
+// and of both activation parts into a 4-stage shared-memory ring with TMA
+// (128-byte swizzled tiles), a second elected thread issues tcgen05.mma
+// into a TMEM accumulator (128 lanes x NT fp32 columns) and releases each
+// stage with tcgen05.commit, and the four warps read the accumulator back
+// with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31, i.e. weight rows) and
+// store or atomically add it to out.  Grid: (N_w / 128 weight tiles, K
+// splits, activation tiles).  The weight copies of the first stages are
+// issued before griddepcontrol.wait; the activation copies after it.
+#include <cuda.h>
+
+#include <cstdio>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.cuh"
+#include "mtp.h"
+
+namespace mtp {
+namespace {
+
+constexpr int TC_M = 128;      // weight rows per CTA (MMA M)
+constexpr int TC_K = 64;       // k per stage: one 128-byte swizzle row of bf16
+constexpr int TC_STAGES = 4;
+constexpr int TC_THREADS = 128;
+constexpr uint32_t TC_W_BYTES = TC_M * TC_K * 2;
+
+// ---- PTX wrappers (tcgen05, TMA) ----
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {  // one whole warp
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(dst)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {  // the allocating warp
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc)
+        : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_addr(bar))
+                 : "memory");
+}
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (thread i: lane i).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor of a K-major tile stored as 128-byte rows
+// with the 128-byte swizzle (16-byte chunk c of row r at c ^ (r & 7), tile
+// base 1024-byte aligned): start address, stride between 8-row groups
+// (1024 B), descriptor version 1, layout "128-byte swizzle".
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;             // leading byte offset (unused by swizzled K-major tiles)
+    d |= (uint64_t)(1024 >> 4) << 32;   // stride byte offset
+    d |= (uint64_t)1 << 46;             // version
+    d |= (uint64_t)2 << 61;             // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, M = 128, N = nt.
+__host__ __device__ constexpr uint32_t tc_idesc(int nt) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(nt >> 3) << 17) | ((uint32_t)(TC_M >> 4) << 24);
+}
+
+template <int NT>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tw, const __grid_constant__ CUtensorMap tah,
+                   const __grid_constant__ CUtensorMap tal, const TcGemmArgs a) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    constexpr uint32_t A_BYTES = NT * TC_K * 2, STAGE = TC_W_BYTES + 2 * A_BYTES;
+    constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
+    __shared__ uint64_t full[TC_STAGES], empty[TC_STAGES], done;
+    __shared__ uint32_t tmem_base;
+    __shared__ int s_ok;
+    unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tile = blockIdx.x, split = blockIdx.y, ntile = blockIdx.z;
+    const int chunks = a.k_chunks;
+    const int kc0 = split * chunks;
+    const int arow = ntile * NT;
+
+    if (warp == 0) {
+        tmem_alloc(&tmem_base, TMEM_COLS);
+        tmem_relinquish();
+    }
+    if (tid == 32) {
+        for (int s = 0; s < TC_STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(&done, 1);
+        fence_barrier_init();
+        s_ok = 1;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    // weights of the first stages: independent of the previous kernel
+    auto w_coords = [&](int c, int& x, int& y) {
+        const int kc = kc0 + c;
+        if (a.w_rows_per_kchunk) {  // k-chunk kc is a block of rows (W_o stored per head)
+            x = 0;
+            y = kc * a.w_rows_per_kchunk + tile * TC_M;
+        } else {
+            x = kc * TC_K;
+            y = tile * TC_M;
+        }
+    };
+    const int pre = chunks < TC_STAGES ? chunks : TC_STAGES;
+    if (tid == 0) {
+        for (int c = 0; c < pre; ++c) {
+            unsigned char* st = smem + (size_t)c * STAGE;
+            mbar_arrive_expect_tx(&full[c], STAGE);
+            int x, y;
+            w_coords(c, x, y);
+            tma_load_2d(st, &tw, x, y, &full[c]);
+        }
+    }
+    pdl_launch_dependents();
+    pdl_wait();
+
+    if (tid == 0) {  // producer: activations of the first stages, then the rest of the ring
+        for (int c = 0; c < chunks; ++c) {
+            const int s = c % TC_STAGES;
+            unsigned char* st = smem + (size_t)s * STAGE;
+            if (c >= TC_STAGES) {
+                if (!mbar_wait(&empty[s], (uint32_t)((c / TC_STAGES) - 1) & 1, a.err)) {
+                    s_ok = 0;
+                    break;
+                }
+                mbar_arrive_expect_tx(&full[s], STAGE);
+                int x, y;
+                w_coords(c, x, y);
+                tma_load_2d(st, &tw, x, y, &full[s]);
+            }
+            const int kx = (kc0 + c) * TC_K;
+            tma_load_2d(st + TC_W_BYTES, &tah, kx, arow, &full[s]);
+            tma_load_2d(st + TC_W_BYTES + A_BYTES, &tal, kx, arow, &full[s]);
+        }
+    } else if (tid == 32) {  // MMA issuer
+        constexpr uint32_t IDESC = tc_idesc(NT);
+        int c = 0;
+        for (; c < chunks; ++c) {
+            const int s = c % TC_STAGES;
+            if (!mbar_wait(&full[s], (uint32_t)(c / TC_STAGES) & 1, a.err)) break;
+            tc_fence_after();
+            const uint32_t wb = smem_addr(smem + (size_t)s * STAGE);
+            const uint32_t hb = wb + TC_W_BYTES, lb = hb + A_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < TC_K / 16; ++kk) {
+                const uint64_t dw = sw128_desc(wb + kk * 32);
+                tc_mma(tmem, dw, sw128_desc(hb + kk * 32), IDESC, (c | kk) != 0);
+                tc_mma(tmem, dw, sw128_desc(lb + kk * 32), IDESC, 1u);
+            }
+            tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+        }
+        if (c < chunks) s_ok = 0;
+        tc_commit(&done);  // every MMA issued above has completed
+    }
+
+    // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
+    const bool fin = mbar_wait(&done, 0, a.err);
+    tc_fence_after();
+    __syncthreads();
+    if (fin && s_ok) {
+        const int f = tile * TC_M + warp * 32 + lane;
+        const float bias = a.bias && split == 0 ? a.bias[f] : 0.f;
+#pragma unroll 1
+        for (int j0 = 0; j0 < NT; j0 += 32) {
+            float v[32];
+            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)j0, v);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const int n = arow + j0 + j;
+                if (n < a.m) {
+                    float* o = a.out + (size_t)n * a.ldo + f;
+                    if (a.accumulate)
+                        atomicAdd(o, v[j] + bias);
+                    else
+                        *o = v[j] + bias;
+                }
+            }
+        }
+    } else if (!fin) {
+        // the MMAs may still be running: wait for them (bounded) before freeing TMEM
+        mbar_wait(&done, 0, nullptr);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
+}
+
+// ---- tensor maps ----
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encode_fn() {
+    static EncodeTiled fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiled>(p);
+    });
+    return fn;
+}
+
+template <int NT>
+size_t tc_smem() {
+    return (size_t)TC_STAGES * (TC_W_BYTES + 2u * NT * TC_K * 2) + 1024;
+}
+
+template <int NT>
+cudaError_t launch_nt(const TcGemm& g, cudaStream_t s, bool pdl) {
+    auto kern = tc_gemm_kernel<NT>;
+    static size_t configured = 0;
+    const size_t smem = tc_smem<NT>();
+    if (configured < smem) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = smem;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.n_w / TC_M, g.splits, (g.args.m + NT - 1) / NT);
+    cfg.blockDim = dim3(TC_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, g.w, g.a_hi, g.a_lo, g.args);
+}
+
+}  // namespace
+
+int tc_encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                 bool pre_swizzled) {
+    EncodeTiled fn = encode_fn();
+    if (!fn) return -1;
+    if ((reinterpret_cast<uintptr_t>(base) & 15) || (inner * 2) % 16 || box_rows == 0 || box_rows > 256) return -2;
+    const cuuint64_t dims[2] = {inner, rows};
+    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)TC_K, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    // pre-swizzled tensors already hold chunk c of row r at c ^ (r & 7): copy them verbatim
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          pre_swizzled ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? 0 : -3;
+}
+
+int tc_tile_rows(int m) { return m <= 32 ? 32 : (m <= 64 ? 64 : 128); }
+
+cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl) {
+    if (g.n_w % TC_M || g.args.k_chunks < 1 || g.splits < 1 || g.args.m < 1) return cudaErrorInvalidValue;
+    if (!g.args.accumulate && g.splits != 1) return cudaErrorInvalidValue;
+    switch (g.nt) {
+        case 32: return launch_nt<32>(g, s, pdl);
+        case 64: return launch_nt<64>(g, s, pdl);
+        case 128: return launch_nt<128>(g, s, pdl);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace mtp
+
+using namespace mtp;
+
+namespace {
+int gemm_fail(int code, const char* fmt, int a = 0, int b = 0, int c = 0, int d = 0, int e = 0) {
+    char buf[256];
+    snprintf(buf, sizeof(buf), fmt, a, b, c, d, e);
+    return report_error(code, buf);
+}
+}  // namespace
+
+extern "C" MTP_API int mtp_gemm_bf16x2(const void* w, const void* a_hi, const void* a_lo, float* out, int n_w, int k,
+                                       int m, int splits, int accumulate, void* stream) {
+    clear_error();
+    if (!w || !a_hi || !a_lo || !out) return gemm_fail(MTP_ERR_INVALID, "mtp_gemm_bf16x2: null pointer");
+    if (n_w < TC_M || n_w % TC_M || k < TC_K || k % TC_K || m < 1 || m > 4096 || splits < 1 ||
+        (k / TC_K) % splits || (!accumulate && splits != 1))
+        return gemm_fail(MTP_ERR_INVALID, "mtp_gemm_bf16x2: n_w=%d k=%d m=%d splits=%d accumulate=%d", n_w, k, m,
+                         splits, accumulate);
+    TcGemm g;
+    g.n_w = n_w;
+    g.splits = splits;
+    g.nt = tc_tile_rows(m);
+    g.args.out = out;
+    g.args.ldo = n_w;
+    g.args.bias = nullptr;
+    g.args.m = m;
+    g.args.k_chunks = k / TC_K / splits;
+    g.args.w_rows_per_kchunk = 0;
+    g.args.accumulate = accumulate;
+    int* d_err = nullptr;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaMallocAsync(&d_err, sizeof(int), st) != cudaSuccess)
+        return gemm_fail(MTP_ERR_CUDA, "mtp_gemm_bf16x2: error word allocation failed");
+    cudaMemsetAsync(d_err, 0, sizeof(int), st);
+    g.args.err = d_err;
+    int rc = 0;
+    if (tc_encode_2d(&g.w, w, (uint64_t)k, (uint64_t)n_w, TC_M, false) ||
+        tc_encode_2d(&g.a_hi, a_hi, (uint64_t)k, (uint64_t)m, (uint32_t)g.nt, false) ||
+        tc_encode_2d(&g.a_lo, a_lo, (uint64_t)k, (uint64_t)m, (uint32_t)g.nt, false)) {
+        rc = gemm_fail(MTP_ERR_INVALID, "mtp_gemm_bf16x2: tensor map encoding failed (alignment?)");
+    } else {
+        const cudaError_t e = launch_tc_gemm(g, st, false);
+        if (e != cudaSuccess) rc = report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
+    }
+    int h_err = 0;
+    cudaMemcpyAsync(&h_err, d_err, sizeof(int), cudaMemcpyDeviceToHost, st);
+    const cudaError_t es = cudaStreamSynchronize(st);
+    cudaFreeAsync(d_err, st);
+    if (rc) return rc;
+    if (es != cudaSuccess) return report_error(MTP_ERR_CUDA, cudaGetErrorString(es));
+    if (h_err) return gemm_fail(MTP_ERR_DEVICE, "mtp_gemm_bf16x2: device error word 0x%x", h_err);
+    return MTP_OK;
+}

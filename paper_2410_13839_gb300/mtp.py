@@ -206,6 +206,12 @@ def mtp_attention_noalloc(args: MtpAttentionArgs, stream=None) -> None:
     check(lib.mtp_attention_noalloc(ctypes.byref(args), _stream_handle(stream)))
 
 
+def mtp_gemm_bf16x2(w, a_hi, a_lo, out, n_w, k, m, splits=1, accumulate=0, stream=None) -> None:
+    """out (+)= (a_hi + a_lo) @ w.T on the tensor cores (the batched path's projection)."""
+    check(lib.mtp_gemm_bf16x2(_ptr(w), _ptr(a_hi), _ptr(a_lo), _ptr(out), n_w, k, m, splits, accumulate,
+                              _stream_handle(stream)))
+
+
 def _as_i32(x):
     if x is None:
         return None
