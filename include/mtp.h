@@ -178,9 +178,12 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *   MTP_OPT_PDL          1 = programmatic dependent launch between kernels (default)
  *   MTP_OPT_L2_PREFETCH  1 = each block kernel prefetches the next layer's weights into L2 (default)
  *   MTP_OPT_MLP_CLUSTERS thread-block clusters of the MLP kernel (>= 1; default: as many as
- *                        the GPU holds at once) */
+ *                        the GPU holds at once)
+ *   MTP_OPT_BATCHED      1 = decode steps whose fed rows (max_batch * n_heads) exceed one fused
+ *                        pass (8 rows) run the batched path: tensor-core projections over all
+ *                        rows at once (bf16 weights only; default); 0 = fused passes of 8 rows */
 typedef enum mtp_option {
-    MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3
+    MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
@@ -191,10 +194,15 @@ MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
  *   MLP         LN2, W1, GELU, W2
  *   HEADS       LN_f and the n heads' logits
  *   SELECT      log-softmax, top-k, Viterbi, acceptance
- *   SAVE        copy of each slot's last hidden state (multi-pass steps, prefill) */
+ *   SAVE        copy of each slot's last hidden state (multi-pass steps, prefill)
+ * and of the batched path (all slots' rows in one pass, bf16 weights):
+ *   PACK        LN / copy / GELU of the rows into bf16 hi + lo GEMM operands
+ *   GEMM        a tensor-core projection (q|k|v, W_o, W1 or W2)
+ *   QKV         query rows out, keys and values appended to the cache
+ *   ATTN        split-KV attention of the fed rows over the cache */
 typedef enum mtp_kernel_kind {
     MTP_K_EMBED = 0, MTP_K_ATTN_BLOCK = 1, MTP_K_MLP = 2, MTP_K_HEADS = 3, MTP_K_SELECT = 4,
-    MTP_K_SAVE = 5, MTP_K_COUNT = 6
+    MTP_K_SAVE = 5, MTP_K_PACK = 6, MTP_K_GEMM = 7, MTP_K_QKV = 8, MTP_K_ATTN = 9, MTP_K_COUNT = 10
 } mtp_kernel_kind;
 
 /* Run one decode step with each kernel launched alone (no graph, no PDL)

@@ -23,7 +23,8 @@ MTP_OPT_GRAPHS = 0
 MTP_OPT_PDL = 1
 MTP_OPT_L2_PREFETCH = 2
 MTP_OPT_MLP_CLUSTERS = 3
-KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save")
+MTP_OPT_BATCHED = 4
+KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save", "pack", "gemm", "qkv", "attn")
 
 
 class MtpConfig(ctypes.Structure):

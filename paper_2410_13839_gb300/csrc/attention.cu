@@ -172,10 +172,13 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
             float sc[RPG];
 #pragma unroll
             for (int j = 0; j < RPG; ++j) sc[j] = 0.f;
+            const int swz = a.kv_swizzled ? (t & 7) : 0;
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
-                const int cc = (c + t) & 7;  // rotate 16-byte chunks: conflict-free rows
-                const uint4 kr = *reinterpret_cast<const uint4*>(Ks + t * HEAD_DIM + cc * 8);
+                // logical chunk cc of row t; consecutive rows hit different banks either by the
+                // rotation (plain pages) or by the stored swizzle (physical chunk cc ^ (t & 7))
+                const int cc = a.kv_swizzled ? c : (c + t) & 7;
+                const uint4 kr = *reinterpret_cast<const uint4*>(Ks + t * HEAD_DIM + ((cc ^ swz) << 3));
                 const float kf[8] = {bf16_lo(kr.x), bf16_hi(kr.x), bf16_lo(kr.y), bf16_hi(kr.y),
                                      bf16_lo(kr.z), bf16_hi(kr.z), bf16_lo(kr.w), bf16_hi(kr.w)};
 #pragma unroll
@@ -218,20 +221,25 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
                 m_run = m_new;
                 __syncwarp();
                 const int kend = min(nk, pos_j - bp * P + 1);  // keys past the row's position weigh 0
+                // dims 2 lane, 2 lane + 1: chunk lane / 4 of the row, stored at (lane / 4) ^ (t & 7) if swizzled
+                const int vch = lane >> 2, vin = (2 * lane) & 7;
                 float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
                 int t = 0;
                 for (; t + 4 <= kend; t += 4) {  // four independent chains
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         const float p = pr[t + u];
-                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + (t + u) * HEAD_DIM + 2 * lane);
+                        const int tt = t + u;
+                        const int col = a.kv_swizzled ? (((vch ^ (tt & 7)) << 3) | vin) : 2 * lane;
+                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + tt * HEAD_DIM + col);
                         a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
                         a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
                     }
                 }
                 for (; t < kend; ++t) {
                     const float p = pr[t];
-                    const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + t * HEAD_DIM + 2 * lane);
+                    const int col = a.kv_swizzled ? (((vch ^ (t & 7)) << 3) | vin) : 2 * lane;
+                    const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + t * HEAD_DIM + col);
                     a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
                     a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
                 }

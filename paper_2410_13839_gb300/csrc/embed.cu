@@ -101,7 +101,7 @@ __global__ void slot_set_kernel(SlotSet s) {
 
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(MAX_ROWS);
+    cfg.gridDim = dim3(a.rows > MAX_ROWS ? a.rows : MAX_ROWS);  // rows past a.rows are written inactive
     cfg.blockDim = dim3(256);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -135,10 +135,10 @@ __global__ void __launch_bounds__(256) save_last_kernel(const float* x, const in
     for (int i = threadIdx.x; i < d; i += blockDim.x) h_last[(size_t)row_seq[r] * d + i] = x[(size_t)r * d + i];
 }
 
-cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
+cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d, int rows,
                              unsigned long long* trace, cudaStream_t s, bool pdl) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(MAX_ROWS);
+    cfg.gridDim = dim3(rows);
     cfg.blockDim = dim3(256);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];

@@ -73,6 +73,7 @@ struct AttnArgs {
     int val_seq, val_old, val_new;                           // PLAN_VALUE
     int* err;
     unsigned long long* trace;
+    int kv_swizzled;                                         // pages store chunk c of key row t at c ^ (t & 7)
 };
 
 size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
@@ -177,8 +178,33 @@ struct SlotSet {
 cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s);
 cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s);
 // copy each slot's last fed row (row_last) of x [MAX_ROWS][d] into h_last [slot][d]
-cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d,
+cudaError_t launch_save_last(const float* x, const int* row_seq, const int* row_last, float* h_last, int d, int rows,
                              unsigned long long* trace, cudaStream_t s, bool pdl);
+
+// ------------------------------------------------------- batched path ----
+enum PackMode : int { PACK_LN = 0, PACK_COPY = 1, PACK_GELU = 2 };
+struct PackArgs {
+    int mode;                     // PackMode
+    const float* x; int ldx;      // input rows [m][ldx], k columns used
+    float* zero_after;            // PACK_GELU: rows zeroed after reading (may be x), or null
+    const float* gamma; const float* beta; float eps;   // PACK_LN
+    const int* row_seq;           // rows with row_seq < 0 are packed as zeros
+    __nv_bfloat16* hi; __nv_bfloat16* lo;  // [m][k] bf16 parts: hi + lo = the fp32 row
+    int k, m;                     // k <= 4096
+    unsigned long long* trace;
+};
+struct QkvFinishArgs {
+    float* qkv;                   // [m][3d], features h*192 + {q,k,v}*64 + dd (bias included); zeroed after use
+    float* q;                     // [m][d] query rows, head h at columns 64h..64h+63
+    __nv_bfloat16* kv_pool; long long page_elems; long long layer_off; int page_size, n_heads;
+    const int* block_table; int bt_stride;
+    const int* row_seq; const int* row_pos;
+    int m;
+    int* err;
+    unsigned long long* trace;
+};
+cudaError_t launch_pack_rows(const PackArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------ tensor-core GEMM ----
 // out[n][f] (+)= sum_k (a_hi[n][k] + a_lo[n][k]) w[f][k] with tcgen05 (tc_gemm.cu).

@@ -102,6 +102,21 @@ struct mtp_ctx {
     const void *tok_phone = nullptr, *tok_codec = nullptr, *w_heads = nullptr;
     const float *lnf_g = nullptr, *lnf_b = nullptr, *b_heads = nullptr, *log_q = nullptr;
     std::vector<Layer> layers;
+    // batched path (bf16 weights; more fed rows than one fused pass takes): tensor-core
+    // projections over all rows of a step, row-wise glue kernels, split-KV attention
+    bool use_batched = true, batched_ok = false;
+    int bm_max = 0;  // rows of the batched buffers: max_batch * n_heads_max
+    uint16_t* d_w2p = nullptr;  // W2 [layers][d][F] as stored in the blob (the fused kernels keep it transposed)
+    float *d_bx = nullptr, *d_bqkv = nullptr, *d_bq = nullptr, *d_batt = nullptr, *d_bh = nullptr;
+    float* d_bws = nullptr;  // attention split partials
+    int* d_bwc = nullptr;    // attention split counters
+    int battn_splits = 1;
+    __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
+    struct LayerMaps {
+        CUtensorMap wqkv, wo, w1, w2;
+    };
+    std::vector<LayerMaps> lmaps;
+    CUtensorMap amap_hi[3], amap_lo[3], umap_hi[3], umap_lo[3];  // activation tiles of 32, 64, 128 rows
     float* d_pe = nullptr;
     // KV cache
     uint16_t* d_kv = nullptr;
@@ -256,6 +271,135 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
     return MTP_OK;
 }
 
+// K splits of a tensor-core GEMM: as many as keep one wave of CTAs (one per SM)
+// with a whole number of 64-wide k-chunks each.
+int gemm_splits(const mtp_ctx* c, int n_w, int k, int ntiles) {
+    const int tiles = n_w / 128 * ntiles, chunks = k / 64;
+    int s = 1;
+    while (chunks % (2 * s) == 0 && tiles * 2 * s <= c->num_sms) s *= 2;
+    return s;
+}
+
+int tile_index(int nt) { return nt == 32 ? 0 : (nt == 64 ? 1 : 2); }
+
+// The block stack over the M = max_batch * n rows the embedding put in d_bx
+// (slot b: rows b*n .. b*n + n - 1), as tensor-core projections plus row-wise
+// kernels; the final hidden rows stay in d_bx.
+int run_layers_batched(mtp_ctx* c, int M, int n, cudaStream_t s, bool pdl, Prof* prof) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
+    const int nt = tc_tile_rows(M), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
+    for (int l = 0; l < cf.layers; ++l) {
+        const Layer& L = c->layers[l];
+        const mtp_ctx::LayerMaps& W = c->lmaps[l];
+        auto pack = [&](int mode, const float* x, int k, const float* g, const float* bta, float* zero,
+                        __nv_bfloat16* hi, __nv_bfloat16* lo) -> int {
+            PackArgs pa;
+            std::memset(&pa, 0, sizeof(pa));
+            pa.mode = mode; pa.x = x; pa.ldx = k; pa.zero_after = zero; pa.gamma = g; pa.beta = bta;
+            pa.eps = cf.ln_eps; pa.row_seq = c->d_row_seq; pa.hi = hi; pa.lo = lo; pa.k = k; pa.m = M;
+            pa.trace = tslot(c, MTP_K_PACK);
+            LAUNCH(MTP_K_PACK, launch_pack_rows(pa, s, pdl));
+            return MTP_OK;
+        };
+        auto gemm = [&](const CUtensorMap& w, int n_w, int k, bool a_is_u, float* out, int ldo, const float* bias,
+                        int w_rows_per_kchunk) -> int {
+            TcGemm g;
+            g.w = w;
+            g.a_hi = a_is_u ? c->umap_hi[ti] : c->amap_hi[ti];
+            g.a_lo = a_is_u ? c->umap_lo[ti] : c->amap_lo[ti];
+            g.n_w = n_w; g.nt = nt;
+            g.splits = gemm_splits(c, n_w, k, ntiles);
+            g.args.out = out; g.args.ldo = ldo; g.args.bias = bias; g.args.m = M;
+            g.args.k_chunks = k / 64 / g.splits; g.args.w_rows_per_kchunk = w_rows_per_kchunk;
+            g.args.accumulate = 1; g.args.err = c->d_err;
+            LAUNCH(MTP_K_GEMM, launch_tc_gemm(g, s, pdl));
+            return MTP_OK;
+        };
+        // LN1 -> q|k|v (split-K accumulation into the zeroed buffer, bias once)
+        MTP_TRY(pack(PACK_LN, c->d_bx, d, L.ln1_g, L.ln1_b, nullptr, c->d_ahi, c->d_alo));
+        MTP_TRY(gemm(W.wqkv, 3 * d, d, false, c->d_bqkv, 3 * d, L.bqkv, 0));
+        QkvFinishArgs qf;
+        std::memset(&qf, 0, sizeof(qf));
+        qf.qkv = c->d_bqkv; qf.q = c->d_bq;
+        qf.kv_pool = reinterpret_cast<__nv_bfloat16*>(c->d_kv); qf.page_elems = c->page_elems;
+        qf.layer_off = (long long)l * 2 * H * P * HEAD_DIM; qf.page_size = P; qf.n_heads = H;
+        qf.block_table = c->d_block_table; qf.bt_stride = c->pages_per_seq;
+        qf.row_seq = c->d_row_seq; qf.row_pos = c->d_row_pos; qf.m = M; qf.err = c->d_err;
+        qf.trace = tslot(c, MTP_K_QKV);
+        LAUNCH(MTP_K_QKV, launch_qkv_finish(qf, s, pdl));
+        // attention of every slot's fed rows over its cached keys
+        AttnArgs at;
+        std::memset(&at, 0, sizeof(at));
+        at.q = c->d_bq; at.ldq = d;
+        at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(c->d_kv); at.page_elems = c->page_elems;
+        at.layer_off = qf.layer_off;
+        at.block_table = c->d_block_table; at.bt_stride = c->pages_per_seq;
+        at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
+        at.out = c->d_batt; at.ldo = d;
+        at.ws_part = c->d_bws; at.ws_count = c->d_bwc;
+        at.rows_per_group = n; at.n_heads = H; at.page_size = P; at.n_splits = c->battn_splits;
+        at.plan = PLAN_DEVICE; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = 0;
+        at.err = c->d_err; at.kv_swizzled = 1;
+        at.trace = tslot(c, MTP_K_ATTN);
+        LAUNCH(MTP_K_ATTN, launch_attention(at, cf.max_batch, s, pdl));
+        // x += attention W_o^T + b_o (the per-head W_o blocks are the k-chunks)
+        MTP_TRY(pack(PACK_COPY, c->d_batt, d, nullptr, nullptr, nullptr, c->d_ahi, c->d_alo));
+        MTP_TRY(gemm(W.wo, d, d, false, c->d_bx, d, L.bo, d));
+        // x += GELU(LN2(x) W1^T + b1) W2^T + b2
+        MTP_TRY(pack(PACK_LN, c->d_bx, d, L.ln2_g, L.ln2_b, nullptr, c->d_ahi, c->d_alo));
+        MTP_TRY(gemm(W.w1, F, d, false, c->d_bh, F, L.b1, 0));
+        MTP_TRY(pack(PACK_GELU, c->d_bh, F, nullptr, nullptr, c->d_bh, c->d_uhi, c->d_ulo));
+        MTP_TRY(gemm(W.w2, d, F, true, c->d_bx, d, L.b2, 0));
+    }
+    return MTP_OK;
+}
+
+// Buffers and tensor maps of the batched path (bf16 weights only).
+int setup_batched(mtp_ctx* c) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
+    c->bm_max = cf.max_batch * cf.n_heads_max;
+    if (c->wbytes != 2 || c->bm_max <= MAX_ROWS || !c->d_w2p) return MTP_OK;
+    const size_t M = (size_t)c->bm_max;
+    MTP_TRY(c->alloc(&c->d_bx, M * d));
+    MTP_TRY(c->alloc(&c->d_bqkv, M * 3 * d));
+    MTP_TRY(c->alloc(&c->d_bq, M * d));
+    MTP_TRY(c->alloc(&c->d_batt, M * d));
+    MTP_TRY(c->alloc(&c->d_bh, M * F));
+    uint16_t *ahi, *alo, *uhi, *ulo;
+    MTP_TRY(c->alloc(&ahi, M * d));
+    MTP_TRY(c->alloc(&alo, M * d));
+    MTP_TRY(c->alloc(&uhi, M * F));
+    MTP_TRY(c->alloc(&ulo, M * F));
+    c->d_ahi = reinterpret_cast<__nv_bfloat16*>(ahi);
+    c->d_alo = reinterpret_cast<__nv_bfloat16*>(alo);
+    c->d_uhi = reinterpret_cast<__nv_bfloat16*>(uhi);
+    c->d_ulo = reinterpret_cast<__nv_bfloat16*>(ulo);
+    c->battn_splits = attn_splits_for(cf.max_batch, H, P, cf.max_ctx, c->num_sms);
+    MTP_TRY(c->alloc(&c->d_bws, attn_workspace_floats(cf.max_batch, H, c->battn_splits, cf.n_heads_max)));
+    MTP_TRY(c->alloc(&c->d_bwc, (size_t)cf.max_batch * H));
+    c->lmaps.resize(cf.layers);
+    int bad = 0;
+    for (int l = 0; l < cf.layers; ++l) {
+        const Layer& L = c->layers[l];
+        mtp_ctx::LayerMaps& W = c->lmaps[l];
+        bad |= tc_encode_2d(&W.wqkv, L.wqkv, (uint64_t)d, (uint64_t)3 * d, 128, true);
+        bad |= tc_encode_2d(&W.wo, L.wo, (uint64_t)HEAD_DIM, (uint64_t)H * d, 128, true);
+        bad |= tc_encode_2d(&W.w1, L.w1, (uint64_t)d, (uint64_t)F, 128, true);
+        bad |= tc_encode_2d(&W.w2, c->d_w2p + (size_t)l * d * F, (uint64_t)F, (uint64_t)d, 128, false);
+    }
+    const int nts[3] = {32, 64, 128};
+    for (int t = 0; t < 3; ++t) {
+        bad |= tc_encode_2d(&c->amap_hi[t], c->d_ahi, (uint64_t)d, M, (uint32_t)nts[t], false);
+        bad |= tc_encode_2d(&c->amap_lo[t], c->d_alo, (uint64_t)d, M, (uint32_t)nts[t], false);
+        bad |= tc_encode_2d(&c->umap_hi[t], c->d_uhi, (uint64_t)F, M, (uint32_t)nts[t], false);
+        bad |= tc_encode_2d(&c->umap_lo[t], c->d_ulo, (uint64_t)F, M, (uint32_t)nts[t], false);
+    }
+    c->batched_ok = bad == 0;  // without tensor maps the fused path serves every batch
+    return MTP_OK;
+}
+
 EmbedArgs embed_base(mtp_ctx* c) {
     EmbedArgs e;
     std::memset(&e, 0, sizeof(e));
@@ -311,6 +455,25 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
     const int spc = std::max(1, MAX_ROWS / n);
     const bool single = B <= spc;  // one pass feeds every slot: the heads read its rows directly
     float* final_x = nullptr;
+    if (!single && c->use_batched && c->batched_ok) {  // every slot's rows in one batched pass
+        const int M = B * n;
+        EmbedArgs e = embed_base(c);
+        e.mode = 0; e.rows = M; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
+        e.trace = tslot(c, MTP_K_EMBED);
+        LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
+        MTP_TRY(run_layers_batched(c, M, n, s, pdl, prof));
+        unsigned long long* tr = tslot(c, MTP_K_SAVE);
+        LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
+        for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
+            const int m = std::min(MAX_ROWS, B - b0);
+            MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, nullptr,
+                                 b0, s, pdl, prof));
+        }
+        SelectArgs sa = select_base(c, n, k);
+        sa.trace = tslot(c, MTP_K_SELECT);
+        LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
+        return MTP_OK;
+    }
     for (int b0 = 0; b0 < B; b0 += spc) {
         const int G = std::min(spc, B - b0), M = G * n;
         EmbedArgs e = embed_base(c);
@@ -320,7 +483,8 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
         if (!single) {
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
-            LAUNCH(MTP_K_SAVE, launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, d, tr, s, pdl));
+            LAUNCH(MTP_K_SAVE,
+                   launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, d, MAX_ROWS, tr, s, pdl));
         }
     }
     for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
@@ -535,6 +699,11 @@ int upload_weights(mtp_ctx* c, const void* blob, size_t bytes) {
             }
             src = tmp.data();
         }
+        if (j == 10 && c->wbytes == 2) {  // W2 [d][F] as given, for the batched path's tensor-core GEMM
+            if (!c->d_w2p) MTP_TRY(c->alloc(&c->d_w2p, (size_t)cf.layers * cf.d_model * cf.d_ffn));
+            const int l = (int)((i - 2) / 12);
+            CUDA_TRY(cudaMemcpy(c->d_w2p + (size_t)l * cf.d_model * cf.d_ffn, b + off, nb, cudaMemcpyHostToDevice));
+        }
         CUDA_TRY(cudaMemcpy(dw + dev_off[i], src, nb, cudaMemcpyHostToDevice));
     }
     size_t i = 0;
@@ -661,8 +830,10 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_cand_logp, (size_t)lb * nm * MAX_TOPK)) ||
         (r = c->alloc(&c->d_cand_ids, (size_t)lb * nm * MAX_TOPK)) || (r = c->alloc(&c->d_path, (size_t)lb * nm)) ||
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
-        (r = c->alloc(&c->d_row_seq, MAX_ROWS)) || (r = c->alloc(&c->d_row_pos, MAX_ROWS)) ||
-        (r = c->alloc(&c->d_row_last, MAX_ROWS)) || (r = c->alloc(&c->d_err, 1)))
+        (r = c->alloc(&c->d_row_seq, std::max(MAX_ROWS, B * nm))) ||
+        (r = c->alloc(&c->d_row_pos, std::max(MAX_ROWS, B * nm))) ||
+        (r = c->alloc(&c->d_row_last, std::max(MAX_ROWS, B * nm))) || (r = c->alloc(&c->d_err, 1)) ||
+        (r = setup_batched(c)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
     if (cudaMemcpy(c->d_block_table, c->h_block_table.data(), c->h_block_table.size() * sizeof(int),
@@ -695,6 +866,9 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
     } else if (option == MTP_OPT_L2_PREFETCH) {
         changed = c->use_l2_prefetch != (value != 0);
         c->use_l2_prefetch = value != 0;
+    } else if (option == MTP_OPT_BATCHED) {
+        changed = c->use_batched != (value != 0);
+        c->use_batched = value != 0;
     } else if (option == MTP_OPT_MLP_CLUSTERS) {
         if (value < 1 || value > std::max(1, 2 * c->num_sms / MLP_CLUSTER))
             return fail(MTP_ERR_INVALID, "MLP clusters %d out of range", value);
@@ -727,6 +901,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_PDL: *value = c->use_pdl; break;
         case MTP_OPT_L2_PREFETCH: *value = c->use_l2_prefetch; break;
         case MTP_OPT_MLP_CLUSTERS: *value = c->mlp_clusters; break;
+        case MTP_OPT_BATCHED: *value = c->use_batched && c->batched_ok; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;
@@ -783,7 +958,7 @@ MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph,
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
         MTP_TRY(run_layers(c, m, 1, m, PLAN_VALUE, 0, slot, p0, m, s, c->use_pdl, prof, &final_x));
     }
-    LAUNCH(MTP_K_SAVE, launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, nullptr, s,
+    LAUNCH(MTP_K_SAVE, launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, MAX_ROWS, nullptr, s,
                                         c->use_pdl));
     MTP_TRY(slot_set(c, slot, (int)T, -1, -1, -1, -1, -1));
     // pageable host prompts: copies above are complete when the call returns

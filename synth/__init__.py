@@ -132,6 +132,9 @@ TINY = ModelConfig(layers=2, d_model=256, n_attn_heads=4, d_ffn=1024, phone_voca
                    weight_dtype="f32")
 VALLE = ModelConfig(layers=12, d_model=1024, n_attn_heads=16, d_ffn=4096, phone_vocab=512,
                     weight_dtype="bf16")
+# the tiny model with bf16 matrices: small batched-path (tensor-core) parity cases
+TINY_BF16 = ModelConfig(layers=2, d_model=256, n_attn_heads=4, d_ffn=1024, phone_vocab=128,
+                        weight_dtype="bf16")
 
 
 def weight_names(cfg: ModelConfig) -> list[str]:
