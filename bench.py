@@ -102,6 +102,98 @@ def _decode_bytes_total(d, F, V, L, n, wb, prompt_len, gen):
     return total
 
 
+B32 = 32
+B32_WORKLOAD = ("VALL-E-sized batched serving: B=32, prompts U[32,128] phonemes + U[150,450] acoustic, "
+                "generation U[375,1500] with per-sequence EOS, n=4, top_k=4")
+
+
+def b32_sequences(batch=B32):
+    """Prompt lengths, prompts and generation budgets of the batched-serving workload."""
+    seqs = []
+    for i in range(batch):
+        n_ph = synth.make_lengths(i, 32, 128, "serve_phonemes")
+        n_ac = synth.make_lengths(i, 150, 450, "serve_acoustic")
+        gen = synth.make_lengths(i, 375, 1500, "serve_generate")
+        ph, ac = synth.make_prompt(i, n_ph, n_ac, MODEL.phone_vocab)
+        seqs.append((ph, ac, gen))
+    return seqs
+
+
+def _batched_decode_bytes(prompt_lens, gens, d, F, V, L, n, wb):
+    """Algorithmic bytes of the decode steps of a batch run in lockstep: weights and
+    heads once per step, cached keys/values read and the fed rows' written per active sequence."""
+    weights = L * ((3 * d * d + d * d + 2 * d * F) * wb + (3 * d + d + F + d + 4 * d) * 4)
+    heads = n * V * d * wb + n * V * 4 + 2 * d * 4
+    cached, produced, fed = list(prompt_lens), [0] * len(gens), [0] * len(gens)
+    total = 0
+    while any(p < g for p, g in zip(produced, gens)):
+        kv, any_fed = 0, False
+        for i, g in enumerate(gens):
+            if produced[i] >= g:
+                continue
+            if fed[i]:
+                kv += L * (cached[i] + fed[i]) * d * 4 + L * fed[i] * d * 4
+                cached[i] += fed[i]
+                any_fed = True
+            a = min(n, g - produced[i])
+            produced[i] += a
+            fed[i] = a
+        total += heads + (weights + kv if any_fed else 0)
+    return total
+
+
+def run_b32(mtp, stream, warmup, steps):
+    """Whole-job codec tokens/s of the batched-serving workload on this GPU (prefill + decode)."""
+    import torch
+    seqs = b32_sequences()
+    max_ctx = max(len(p) + len(a) + g for p, a, g in seqs) + MODEL.n_heads_max + 8
+    w = synth.make_weights(MODEL)
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, B32, max_ctx, stream=stream)
+    ctx = dec.ctx
+    dev = [(torch.from_numpy(p).cuda(), torch.from_numpy(a).cuda(), g) for p, a, g in seqs]
+    lens = torch.zeros(B32, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+
+    def job(ev=None):
+        if ev:
+            ev[0].record(stream)
+        for b, (p, a, g) in enumerate(dev):
+            mtp.mtp_prefill(ctx, b, p, a, g)
+        if ev:
+            ev[1].record(stream)
+        n_steps = mtp.mtp_generate(ctx, N_HEADS, TOP_K, None, 0, lens)
+        if ev:
+            ev[2].record(stream)
+        return n_steps
+
+    for _ in range(warmup):
+        job()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    dsteps = 0
+    for i in range(steps):
+        dsteps += job(evs[i])
+    torch.cuda.synchronize()
+    tokens = int(lens.sum().item())
+    total_ms = sum(e[0].elapsed_time(e[2]) for e in evs)
+    decode_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    prefill_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    d, F, V, L = MODEL.d_model, MODEL.d_ffn, MODEL.codec_vocab, MODEL.layers
+    dec_bytes = _batched_decode_bytes([len(p) + len(a) for p, a, _ in seqs], [g for _, _, g in seqs],
+                                      d, F, V, L, N_HEADS, 2)
+    peak, peak_kind = _peaks()
+    batched = mtp.mtp_get_option(ctx, mtp.MTP_OPT_BATCHED)
+    dec.close()
+    return {"value": tokens * steps / (total_ms / 1e3), "unit": "codec tokens/s", "batch": B32,
+            "workload": B32_WORKLOAD, "tokens_per_job": tokens, "jobs": steps, "warmup_jobs": warmup,
+            "ms_per_job": total_ms / steps, "prefill_ms": prefill_ms, "decode_ms": decode_ms,
+            "decode_steps_per_job": dsteps // steps, "decode_tokens_per_s": tokens / (decode_ms / 1e3),
+            "path": "batched (tensor-core projections)" if batched else "fused 8-row passes",
+            "decode_roofline": {"decode_bytes": dec_bytes, "achieved_gbs": dec_bytes / (decode_ms / 1e3) / 1e9,
+                                "peak": peak, "peak_source": peak_kind,
+                                "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak}}
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples while the timed region runs."""
 
@@ -331,6 +423,8 @@ def run_ours(args):
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
             "clocks": clk.summary(), "kernel_ms": {k: v[0] for k, v in prof.items()}}
     dec.close()
+    if not args.no_b32:
+        line["b32"] = run_b32(mtp, stream, max(1, min(args.warmup, 2)), max(1, min(args.steps, 3)))
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:
@@ -344,6 +438,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-b32", action="store_true", help="skip the batch-32 serving measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -101,7 +101,8 @@ __global__ void slot_set_kernel(SlotSet s) {
 
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.rows > MAX_ROWS ? a.rows : MAX_ROWS);  // rows past a.rows are written inactive
+    // rows past a.rows (up to the next multiple of 8) are written inactive
+    cfg.gridDim = dim3(a.rows > MAX_ROWS ? (a.rows + 7) / 8 * 8 : MAX_ROWS);
     cfg.blockDim = dim3(256);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];

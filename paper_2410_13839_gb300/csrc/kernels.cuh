@@ -15,6 +15,7 @@ namespace mtp {
 
 constexpr int HEAD_DIM = 64;     // attention head width (fixed by the kernels)
 constexpr int MAX_ROWS = 8;      // rows per weight-streaming pass (B * n_heads per chunk)
+constexpr int PREFILL_ROWS = 128; // prompt positions per batched-path prefill chunk
 constexpr int MAX_TOPK = 32;     // one warp lane per candidate
 constexpr int MAX_NHEADS = 8;    // prediction heads
 constexpr int MAX_VOCAB = 1056;  // 33 logits per lane in the top-k warp

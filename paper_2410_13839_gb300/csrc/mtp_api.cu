@@ -110,7 +110,7 @@ struct mtp_ctx {
     float *d_bx = nullptr, *d_bqkv = nullptr, *d_bq = nullptr, *d_batt = nullptr, *d_bh = nullptr;
     float* d_bws = nullptr;  // attention split partials
     int* d_bwc = nullptr;    // attention split counters
-    int battn_splits = 1;
+    int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -282,10 +282,12 @@ int gemm_splits(const mtp_ctx* c, int n_w, int k, int ntiles) {
 
 int tile_index(int nt) { return nt == 32 ? 0 : (nt == 64 ? 1 : 2); }
 
-// The block stack over the M = max_batch * n rows the embedding put in d_bx
-// (slot b: rows b*n .. b*n + n - 1), as tensor-core projections plus row-wise
-// kernels; the final hidden rows stay in d_bx.
-int run_layers_batched(mtp_ctx* c, int M, int n, cudaStream_t s, bool pdl, Prof* prof) {
+// The block stack over the M rows the embedding put in d_bx, as tensor-core
+// projections plus row-wise kernels; the final hidden rows stay in d_bx.
+// Attention groups: `groups` runs of rpg rows, each of one slot (decode:
+// slot b's fed rows b*n.., plan PLAN_DEVICE; prefill: 8 consecutive prompt
+// positions, plan PLAN_ROWS).
+int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStream_t s, bool pdl, Prof* prof) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
     const int nt = tc_tile_rows(M), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
@@ -338,11 +340,14 @@ int run_layers_batched(mtp_ctx* c, int M, int n, cudaStream_t s, bool pdl, Prof*
         at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
         at.out = c->d_batt; at.ldo = d;
         at.ws_part = c->d_bws; at.ws_count = c->d_bwc;
-        at.rows_per_group = n; at.n_heads = H; at.page_size = P; at.n_splits = c->battn_splits;
-        at.plan = PLAN_DEVICE; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = 0;
+        at.rows_per_group = rpg; at.n_heads = H; at.page_size = P;
+        at.n_splits = std::min(attn_splits_for(groups, H, P, cf.max_ctx, c->num_sms),
+                               c->battn_ws_units / std::max(1, groups));
+        at.n_splits = std::max(1, at.n_splits);
+        at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = 0;
         at.err = c->d_err; at.kv_swizzled = 1;
         at.trace = tslot(c, MTP_K_ATTN);
-        LAUNCH(MTP_K_ATTN, launch_attention(at, cf.max_batch, s, pdl));
+        LAUNCH(MTP_K_ATTN, launch_attention(at, groups, s, pdl));
         // x += attention W_o^T + b_o (the per-head W_o blocks are the k-chunks)
         MTP_TRY(pack(PACK_COPY, c->d_batt, d, nullptr, nullptr, nullptr, c->d_ahi, c->d_alo));
         MTP_TRY(gemm(W.wo, d, d, false, c->d_bx, d, L.bo, d));
@@ -359,8 +364,8 @@ int run_layers_batched(mtp_ctx* c, int M, int n, cudaStream_t s, bool pdl, Prof*
 int setup_batched(mtp_ctx* c) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
-    c->bm_max = cf.max_batch * cf.n_heads_max;
-    if (c->wbytes != 2 || c->bm_max <= MAX_ROWS || !c->d_w2p) return MTP_OK;
+    c->bm_max = std::max(cf.max_batch * cf.n_heads_max, PREFILL_ROWS);
+    if (c->wbytes != 2 || !c->d_w2p) return MTP_OK;
     const size_t M = (size_t)c->bm_max;
     MTP_TRY(c->alloc(&c->d_bx, M * d));
     MTP_TRY(c->alloc(&c->d_bqkv, M * 3 * d));
@@ -376,9 +381,13 @@ int setup_batched(mtp_ctx* c) {
     c->d_alo = reinterpret_cast<__nv_bfloat16*>(alo);
     c->d_uhi = reinterpret_cast<__nv_bfloat16*>(uhi);
     c->d_ulo = reinterpret_cast<__nv_bfloat16*>(ulo);
-    c->battn_splits = attn_splits_for(cf.max_batch, H, P, cf.max_ctx, c->num_sms);
-    MTP_TRY(c->alloc(&c->d_bws, attn_workspace_floats(cf.max_batch, H, c->battn_splits, cf.n_heads_max)));
-    MTP_TRY(c->alloc(&c->d_bwc, (size_t)cf.max_batch * H));
+    {  // attention workspace for the decode groups (slots) and the prefill groups (8-row runs)
+        const int gd = cf.max_batch, gp = (c->bm_max + 7) / 8;
+        c->battn_ws_units = std::max(gd * attn_splits_for(gd, H, P, cf.max_ctx, c->num_sms),
+                                     gp * attn_splits_for(gp, H, P, cf.max_ctx, c->num_sms));
+        MTP_TRY(c->alloc(&c->d_bws, attn_workspace_floats(c->battn_ws_units, H, 1, MAX_ROWS)));
+        MTP_TRY(c->alloc(&c->d_bwc, (size_t)std::max(gd, gp) * H));
+    }
     c->lmaps.resize(cf.layers);
     int bad = 0;
     for (int l = 0; l < cf.layers; ++l) {
@@ -455,13 +464,13 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
     const int spc = std::max(1, MAX_ROWS / n);
     const bool single = B <= spc;  // one pass feeds every slot: the heads read its rows directly
     float* final_x = nullptr;
-    if (!single && c->use_batched && c->batched_ok) {  // every slot's rows in one batched pass
+    if (!single && c->use_batched && c->batched_ok && B * n <= c->bm_max) {  // every slot's rows in one pass
         const int M = B * n;
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
         e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
-        MTP_TRY(run_layers_batched(c, M, n, s, pdl, prof));
+        MTP_TRY(run_layers_batched(c, M, n, B, PLAN_DEVICE, s, pdl, prof));
         unsigned long long* tr = tslot(c, MTP_K_SAVE);
         LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
         for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
@@ -817,6 +826,7 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
                              sb, sh));
     }
     const int lb = std::max(B, MAX_ROWS);
+    const int row_cap = (std::max(std::max(MAX_ROWS, B * nm), PREFILL_ROWS) + 7) / 8 * 8;  // rows of one pass
     if ((r = c->alloc(&c->d_pe, (size_t)cf.max_ctx * d)) ||
         (r = c->alloc(&c->d_kv, (size_t)c->n_pages * c->page_elems)) ||
         (r = c->alloc(&c->d_block_table, (size_t)B * c->pages_per_seq)) ||
@@ -830,9 +840,8 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_cand_logp, (size_t)lb * nm * MAX_TOPK)) ||
         (r = c->alloc(&c->d_cand_ids, (size_t)lb * nm * MAX_TOPK)) || (r = c->alloc(&c->d_path, (size_t)lb * nm)) ||
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
-        (r = c->alloc(&c->d_row_seq, std::max(MAX_ROWS, B * nm))) ||
-        (r = c->alloc(&c->d_row_pos, std::max(MAX_ROWS, B * nm))) ||
-        (r = c->alloc(&c->d_row_last, std::max(MAX_ROWS, B * nm))) || (r = c->alloc(&c->d_err, 1)) ||
+        (r = c->alloc(&c->d_row_seq, row_cap)) || (r = c->alloc(&c->d_row_pos, row_cap)) ||
+        (r = c->alloc(&c->d_row_last, row_cap)) || (r = c->alloc(&c->d_err, 1)) ||
         (r = setup_batched(c)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
@@ -951,6 +960,21 @@ MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph,
     MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0));
     Prof* prof = nullptr;
     float* final_x = nullptr;
+    if (c->use_batched && c->batched_ok) {  // chunks of PREFILL_ROWS positions through the batched path
+        for (int p0 = 0; p0 < T; p0 += PREFILL_ROWS) {
+            const int m = (int)std::min<long long>(PREFILL_ROWS, T - p0);
+            const int rows = (m + 7) / 8 * 8;
+            EmbedArgs e = embed_base(c);
+            e.mode = 1; e.rows = m; e.slot = slot; e.p0 = p0; e.n_ph = n_ph; e.total = (int)T;
+            e.x = c->d_bx; e.zero_buf = nullptr;
+            LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
+            MTP_TRY(run_layers_batched(c, rows, 8, rows / 8, PLAN_ROWS, s, c->use_pdl, prof));
+            LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, rows,
+                                                nullptr, s, c->use_pdl));
+        }
+        MTP_TRY(slot_set(c, slot, (int)T, -1, -1, -1, -1, -1));
+        return MTP_OK;
+    }
     for (int p0 = 0; p0 < T; p0 += MAX_ROWS) {
         const int m = (int)std::min<long long>(MAX_ROWS, T - p0);
         EmbedArgs e = embed_base(c);

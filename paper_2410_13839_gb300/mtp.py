@@ -12,7 +12,7 @@ import struct
 import numpy as np
 
 from . import _lib
-from ._lib import MTPError, MtpAttentionArgs, MtpConfig, check, lib
+from ._lib import MTP_OPT_BATCHED, MTPError, MtpAttentionArgs, MtpConfig, check, lib  # noqa: F401
 
 BLOB_MAGIC = b"MTPWGT01"
 
