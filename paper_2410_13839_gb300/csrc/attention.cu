@@ -2,16 +2,21 @@
 // (the attention of each block, Sec. III-A), split along the key axis.
 //
 // Grid (split, head, group).  A group is the rows of one slot (the n tokens
-// fed this step, or a prefill chunk).  Each CTA takes a contiguous range of
-// pages of its slot, stages their keys and values for its head in shared
-// memory, and runs a per-row online softmax over them; partial results
-// (max, sum, unnormalised output) of the splits are merged with a log-sum-exp
-// by the CTA that finishes last (an atomic counter per group and head, reset
-// by that CTA), so no second kernel is needed.
+// fed this step, or 8 consecutive positions of a prefill chunk).  Each CTA
+// takes a contiguous range of pages of its slot and streams their keys and
+// values for its head through two halves of shared memory with
+// cp.async.bulk (one half is filled while the other is read).  Each warp
+// takes 16-key tiles: S = Q K^T and O += P V on the tensor cores (mma.sync;
+// the fed rows are the M side, Q and P enter as bf16 hi + lo pairs, which
+// keeps them to fp32 accuracy) with its online-softmax state in registers;
+// the warps' states are merged in shared memory.  Partial results (max,
+// sum, unnormalised output) of the splits are merged with a log-sum-exp by
+// the CTA that finishes last (an atomic counter per group and head, reset by
+// that CTA), so no second kernel is needed.
 //
-// Under programmatic dependent launch the pages that hold only keys cached by
-// earlier steps are fetched with cp.async.bulk before griddepcontrol.wait;
-// the pages touched by this step's appends are read after it.
+// Under programmatic dependent launch the first pages that hold only keys
+// cached by earlier steps are fetched before griddepcontrol.wait; the pages
+// touched by this step's appends are read after it.
 #include <math.h>
 
 #include <cstdio>
@@ -31,15 +36,68 @@ constexpr int PART = 2 + HEAD_DIM;  // (max, sum, out[64]) per row and split
 constexpr int MAX_SPLITS = 32;     // one warp lane per split in the merge
 static_assert(HEAD_DIM == 64, "score scale 0.125 assumes 64-wide heads");
 
-__device__ __forceinline__ void load_page_block(__nv_bfloat16* dst, const __nv_bfloat16* src, int elems) {
-    const uint4* s = reinterpret_cast<const uint4*>(src);
-    uint4* d = reinterpret_cast<uint4*>(dst);
-    for (int i = threadIdx.x; i < elems / 8; i += ATT_THREADS) d[i] = s[i];
+constexpr int HALF_KEYS = ATT_KEYS / 2;  // keys per staging half
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+// x0, x1 as bf16 pairs hi + lo (hi + lo = x to about 2^-16 relative; low halves hold x0)
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+    const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
+    const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+    hi = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    lo = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+}
+
+// Bulk copies of pages [p_from, p_to) of `seq` (this head) into the half
+// that starts at key `key0` of the staging arrays, completing on `bar`.
+// One thread calls it; returns whether anything was requested.
+__device__ __forceinline__ bool stage_pages(const AttnArgs& a, int seq, int p_from, int p_to, int slot0,
+                                            __nv_bfloat16* Ks, __nv_bfloat16* Vs, long long kv_head_off,
+                                            long long v_off, uint64_t* bar) {
+    const int P = a.page_size;
+    const uint32_t blk = (uint32_t)P * HEAD_DIM * 2;
+    uint32_t bytes = 0;
+    for (int p = p_from; p < p_to; ++p)
+        if (a.block_table[(size_t)seq * a.bt_stride + p] >= 0) bytes += 2 * blk;
+    if (!bytes) return false;
+    fence_proxy_async();  // the half was last read by this CTA's threads
+    mbar_arrive_expect_tx(bar, bytes);
+    for (int p = p_from; p < p_to; ++p) {
+        const int phys = a.block_table[(size_t)seq * a.bt_stride + p];
+        if (phys < 0) {  // unreserved page: report, never read
+            if (a.err) atomicOr(a.err, ERR_BOUNDS);
+            continue;
+        }
+        const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head_off;
+        const int slot = slot0 + (p - p_from);
+        bulk_copy_g2s(Ks + (size_t)slot * P * HEAD_DIM, base, blk, bar);
+        bulk_copy_g2s(Vs + (size_t)slot * P * HEAD_DIM, base + v_off, blk, bar);
+    }
+    return true;
 }
 
 __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
-    __shared__ uint64_t bar;
+    __shared__ uint64_t bar;         // pages staged before the dependency wait
+    __shared__ uint64_t hbar[2];     // the two staging halves
+    __shared__ int s_armed[2];
+    __shared__ float s_scale[ATT_THREADS / 32][RPG];
     __shared__ int s_pos[RPG];
     __shared__ int s_act[RPG];
     __shared__ int s_rseq[RPG];
@@ -52,13 +110,14 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem);
     __nv_bfloat16* Vs = Ks + ATT_KEYS * HEAD_DIM;
     float* qs = reinterpret_cast<float*>(Vs + ATT_KEYS * HEAD_DIM);  // [RPG][64], pre-scaled
-    float* Ps = qs + RPG * HEAD_DIM;                                  // [RPG][ATT_KEYS]
-    const int pages_per_batch = ATT_KEYS / P;
+    const int pages_per_batch = HALF_KEYS / P;  // pages per staging half
     const long long kv_head_off = (long long)h * P * HEAD_DIM;
     const long long v_off = (long long)H * P * HEAD_DIM;
 
     if (tid == 0) {
         mbar_init(&bar, 1);
+        mbar_init(&hbar[0], 1);
+        mbar_init(&hbar[1], 1);
         fence_barrier_init();
         s_pre = 0;
     }
@@ -80,7 +139,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
             const int n_pg = (old_len + n_new + P - 1) / P;
             const int pps = (n_pg + S - 1) / S;
             const int pg0 = sp * pps, pg1 = min(n_pg, pg0 + pps);
-            int pre_end = min(min(pg1, pg0 + pages_per_batch), old_len / P);
+            int pre_end = min(min(pg1, pg0 + pages_per_batch), old_len / P);  // half 0 at most
             for (int p = pg0; p < pre_end; ++p)  // only reserved pages are fetched early
                 if (a.block_table[(size_t)seq * a.bt_stride + p] < 0) pre_end = p;
             if (pre_end > pg0) {
@@ -137,117 +196,160 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
         const int j = i / HEAD_DIM, dd = i % HEAD_DIM;
         qs[i] = s_act[j] ? a.q[(size_t)(g * rpg + j) * a.ldq + h * HEAD_DIM + dd] * 0.125f : 0.f;  // 1/sqrt(64)
     }
+    // batches of one staging half each: batch i = pages pg0 + i*ppb .. in half i & 1
+    const int n_batches = (pg1 - pg0 + pages_per_batch - 1) / pages_per_batch;
+    if (tid == 0) {
+        s_armed[0] = s_armed[1] = 0;
+        for (int i = 0; i < 2 && i < n_batches; ++i) {
+            const int b0 = pg0 + i * pages_per_batch, b1 = min(pg1, b0 + pages_per_batch);
+            const int from = i == 0 ? b0 + n_pre : b0;  // batch 0's first pages came before the wait
+            s_armed[i] = stage_pages(a, seq, from, b1, i * pages_per_batch + (from - b0), Ks, Vs, kv_head_off,
+                                     v_off, &hbar[i]);
+        }
+    }
+    __syncthreads();
 
-    float m_run = -INFINITY, l_run = 0.f, acc0 = 0.f, acc1 = 0.f;  // warp j = row j, lane: dims 2l, 2l+1
+    // per-warp tensor-core tiles: fragment rows = fed rows (rows >= RPG zero)
+    const int qrow = lane >> 2, c2 = (lane & 3) * 2;
+    const bool qon = qrow < RPG && s_act[qrow];
+    const int qpos = qon ? s_pos[qrow] : -1;
+    uint32_t qhi[4][2], qlo[4][2];
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int k = ks * 16 + hh * 8 + c2;
+            split2(qon ? qs[qrow * HEAD_DIM + k] : 0.f, qon ? qs[qrow * HEAD_DIM + k + 1] : 0.f, qhi[ks][hh],
+                   qlo[ks][hh]);
+        }
+    float m_w = -INFINITY, l_w = 0.f;
+    float o[8][4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) o[j][i] = 0.f;
+    const int swz = a.kv_swizzled ? 7 : 0;
+    bool ok = true;
+    uint32_t hphase[2] = {0u, 0u};
+    for (int i = 0; i < n_batches; ++i) {
+        const int half = i & 1;
+        const int bp = pg0 + i * pages_per_batch;
+        const int nk = min(pages_per_batch, pg1 - bp) * P;
+        if (i == 0 && n_pre > 0) ok = mbar_wait(&bar, 0, a.err) && ok;
+        if (s_armed[half]) {
+            ok = mbar_wait(&hbar[half], hphase[half], a.err) && ok;
+            hphase[half] ^= 1u;
+        }
+        const uint32_t kb = smem_addr(Ks + (size_t)half * HALF_KEYS * HEAD_DIM);
+        const uint32_t vb = smem_addr(Vs + (size_t)half * HALF_KEYS * HEAD_DIM);
+        for (int kt = warp * 16; kt < nk && ok; kt += (ATT_THREADS / 32) * 16) {
+            float sh[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            float sl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            {
+                const int key = kt + (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks) {
+                    uint32_t b[4];
+                    ldsm_x4(b, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & swz)) << 4));
+                    const uint32_t ah[4] = {qhi[ks][0], 0u, qhi[ks][1], 0u};
+                    const uint32_t al[4] = {qlo[ks][0], 0u, qlo[ks][1], 0u};
+                    const uint32_t b0[2] = {b[0], b[1]}, b1[2] = {b[2], b[3]};
+                    mma_bf16(sh[0], ah, b0);
+                    mma_bf16(sl[0], al, b0);
+                    mma_bf16(sh[1], ah, b1);
+                    mma_bf16(sl[1], al, b1);
+                }
+            }
+            // this lane's scores: row qrow, keys kt + {c2, c2 + 1, 8 + c2, 9 + c2} of the batch
+            float sv[4] = {sh[0][0] + sl[0][0], sh[0][1] + sl[0][1], sh[1][0] + sl[1][0], sh[1][1] + sl[1][1]};
+            float tmax = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int kp = bp * P + kt + (q >> 1) * 8 + c2 + (q & 1);
+                sv[q] = qon && kp <= qpos ? sv[q] : -INFINITY;
+                tmax = fmaxf(tmax, sv[q]);
+            }
+            tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 1));
+            tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 2));
+            const float m_new = fmaxf(m_w, tmax);
+            const float corr = m_new == -INFINITY ? 1.f : (m_w == -INFINITY ? 0.f : expf(m_w - m_new));
+            float pv[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) pv[q] = sv[q] == -INFINITY ? 0.f : expf(sv[q] - m_new);
+            l_w = l_w * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
+            m_w = m_new;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                o[j][0] *= corr;
+                o[j][1] *= corr;
+            }
+            uint32_t ph[4] = {0u, 0u, 0u, 0u}, pl[4] = {0u, 0u, 0u, 0u};
+            split2(pv[0], pv[1], ph[0], pl[0]);
+            split2(pv[2], pv[3], ph[2], pl[2]);
+            const int vkey = kt + (lane & 7) + (((lane >> 3) & 1) << 3), vhalf = lane >> 4;
+#pragma unroll
+            for (int dp = 0; dp < 4; ++dp) {
+                uint32_t v[4];
+                ldsm_x4_t(v, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & swz)) << 4));
+                const uint32_t v0[2] = {v[0], v[1]}, v1[2] = {v[2], v[3]};
+                mma_bf16(o[2 * dp], ph, v0);
+                mma_bf16(o[2 * dp], pl, v0);
+                mma_bf16(o[2 * dp + 1], ph, v1);
+                mma_bf16(o[2 * dp + 1], pl, v1);
+            }
+        }
+        __syncthreads();  // every warp is done with this half
+        if (tid == 0 && i + 2 < n_batches) {
+            const int b0 = pg0 + (i + 2) * pages_per_batch, b1 = min(pg1, b0 + pages_per_batch);
+            s_armed[half] = stage_pages(a, seq, b0, b1, half * pages_per_batch, Ks, Vs, kv_head_off, v_off,
+                                        &hbar[half]);
+        }
+        __syncthreads();
+    }
+    if (!__syncthreads_and(ok)) {  // error word set; let copies in flight land before leaving
+        if (n_pre > 0) mbar_wait(&bar, 0, nullptr);
+        for (int hb = 0; hb < 2; ++hb)
+            if (s_armed[hb]) mbar_wait(&hbar[hb], hphase[hb], nullptr);
+        return;
+    }
+    // merge the warps' (max, sum, out) per row through the staging area:
+    // warp j then holds row j's (m_run, l_run) and output dims 2 lane, 2 lane + 1
+    l_w += __shfl_xor_sync(FULL_MASK, l_w, 1);
+    l_w += __shfl_xor_sync(FULL_MASK, l_w, 2);
+    float* wst = reinterpret_cast<float*>(Ks);  // [warps][RPG][PART]
+    if (qrow < RPG) {
+        float* ws = wst + ((size_t)warp * RPG + qrow) * PART;
+        if (c2 == 0) {
+            ws[0] = m_w;
+            ws[1] = l_w;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) *reinterpret_cast<float2*>(ws + 2 + j * 8 + c2) = make_float2(o[j][0], o[j][1]);
+    }
+    __syncthreads();
+    constexpr int NW = ATT_THREADS / 32;
+    if (tid < NW * RPG) {
+        const int w = tid / RPG, j = tid % RPG;
+        float M = -INFINITY;
+#pragma unroll
+        for (int v = 0; v < NW; ++v) M = fmaxf(M, wst[((size_t)v * RPG + j) * PART]);
+        const float mw = wst[((size_t)w * RPG + j) * PART];
+        s_scale[w][j] = mw == -INFINITY ? 0.f : expf(mw - M);
+    }
+    __syncthreads();
     const int row_j = warp;
     const bool row_on = warp < RPG && s_act[min(warp, RPG - 1)];
-    const int pos_j = row_on ? s_pos[warp] : -1;
-
-    for (int bp = pg0; bp < pg1; bp += pages_per_batch) {
-        const int nb = min(pages_per_batch, pg1 - bp);
-        const int nk = nb * P;
-        const int first_plain = (bp == pg0) ? n_pre : 0;
-        for (int p = first_plain; p < nb; ++p) {
-            const int phys = a.block_table[(size_t)seq * a.bt_stride + bp + p];
-            if (phys < 0) {  // unreserved page: report, never read
-                if (tid == 0 && a.err) atomicOr(a.err, ERR_BOUNDS);
-                continue;
-            }
-            const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head_off;
-            load_page_block(Ks + p * P * HEAD_DIM, base, P * HEAD_DIM);
-            load_page_block(Vs + p * P * HEAD_DIM, base + v_off, P * HEAD_DIM);
+    float m_run = -INFINITY, l_run = 0.f, acc0 = 0.f, acc1 = 0.f;
+    if (warp < RPG) {
+#pragma unroll
+        for (int w = 0; w < NW; ++w) {
+            const float sc = s_scale[w][row_j];
+            const float* ws = wst + ((size_t)w * RPG + row_j) * PART;
+            m_run = fmaxf(m_run, ws[0]);
+            l_run = fmaf(sc, ws[1], l_run);
+            acc0 = fmaf(sc, ws[2 + 2 * lane], acc0);
+            acc1 = fmaf(sc, ws[3 + 2 * lane], acc1);
         }
-        if (bp == pg0 && n_pre > 0) {
-            bool ok = mbar_wait(&bar, 0, a.err);
-            ok = __syncthreads_and(ok) != 0;
-            if (!ok) {  // error word set; let copies in flight land before leaving
-                mbar_wait(&bar, 0, nullptr);
-                return;
-            }
-        }
-        __syncthreads();
-
-        // scores: thread t = key t of the batch
-        for (int t = tid; t < nk; t += ATT_THREADS) {
-            float sc[RPG];
-#pragma unroll
-            for (int j = 0; j < RPG; ++j) sc[j] = 0.f;
-            const int swz = a.kv_swizzled ? (t & 7) : 0;
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                // logical chunk cc of row t; consecutive rows hit different banks either by the
-                // rotation (plain pages) or by the stored swizzle (physical chunk cc ^ (t & 7))
-                const int cc = a.kv_swizzled ? c : (c + t) & 7;
-                const uint4 kr = *reinterpret_cast<const uint4*>(Ks + t * HEAD_DIM + ((cc ^ swz) << 3));
-                const float kf[8] = {bf16_lo(kr.x), bf16_hi(kr.x), bf16_lo(kr.y), bf16_hi(kr.y),
-                                     bf16_lo(kr.z), bf16_hi(kr.z), bf16_lo(kr.w), bf16_hi(kr.w)};
-#pragma unroll
-                for (int j = 0; j < RPG; ++j) {
-                    const float4 q0 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8);
-                    const float4 q1 = *reinterpret_cast<const float4*>(qs + j * HEAD_DIM + cc * 8 + 4);
-                    float s = sc[j];
-                    s = fmaf(q0.x, kf[0], s); s = fmaf(q0.y, kf[1], s);
-                    s = fmaf(q0.z, kf[2], s); s = fmaf(q0.w, kf[3], s);
-                    s = fmaf(q1.x, kf[4], s); s = fmaf(q1.y, kf[5], s);
-                    s = fmaf(q1.z, kf[6], s); s = fmaf(q1.w, kf[7], s);
-                    sc[j] = s;
-                }
-            }
-            const int kp = bp * P + t;
-#pragma unroll
-            for (int j = 0; j < RPG; ++j)
-                Ps[j * ATT_KEYS + t] = (s_act[j] && kp <= s_pos[j]) ? sc[j] : -INFINITY;
-        }
-        __syncthreads();
-
-        if (row_on) {
-            float* pr = Ps + row_j * ATT_KEYS;
-            float bmax = -INFINITY;
-            for (int t = lane; t < nk; t += 32) bmax = fmaxf(bmax, pr[t]);
-            bmax = warp_max(bmax);
-            const float m_new = fmaxf(m_run, bmax);
-            if (m_new != -INFINITY) {
-                const float corr = expf(m_run - m_new);  // 0 when m_run = -inf
-                float lsum = 0.f;
-                for (int t = lane; t < nk; t += 32) {
-                    const float p = expf(pr[t] - m_new);
-                    pr[t] = p;
-                    lsum += p;
-                }
-                lsum = warp_sum(lsum);
-                l_run = l_run * corr + lsum;
-                acc0 *= corr;
-                acc1 *= corr;
-                m_run = m_new;
-                __syncwarp();
-                const int kend = min(nk, pos_j - bp * P + 1);  // keys past the row's position weigh 0
-                // dims 2 lane, 2 lane + 1: chunk lane / 4 of the row, stored at (lane / 4) ^ (t & 7) if swizzled
-                const int vch = lane >> 2, vin = (2 * lane) & 7;
-                float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
-                int t = 0;
-                for (; t + 4 <= kend; t += 4) {  // four independent chains
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float p = pr[t + u];
-                        const int tt = t + u;
-                        const int col = a.kv_swizzled ? (((vch ^ (tt & 7)) << 3) | vin) : 2 * lane;
-                        const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + tt * HEAD_DIM + col);
-                        a0[u] = fmaf(p, bf16_lo(v2), a0[u]);
-                        a1[u] = fmaf(p, bf16_hi(v2), a1[u]);
-                    }
-                }
-                for (; t < kend; ++t) {
-                    const float p = pr[t];
-                    const int col = a.kv_swizzled ? (((vch ^ (t & 7)) << 3) | vin) : 2 * lane;
-                    const uint32_t v2 = *reinterpret_cast<const uint32_t*>(Vs + t * HEAD_DIM + col);
-                    a0[0] = fmaf(p, bf16_lo(v2), a0[0]);
-                    a1[0] = fmaf(p, bf16_hi(v2), a1[0]);
-                }
-                acc0 += (a0[0] + a0[1]) + (a0[2] + a0[3]);
-                acc1 += (a1[0] + a1[1]) + (a1[2] + a1[3]);
-            }
-        }
-        __syncthreads();
     }
 
     float* out_row = a.out + (size_t)(g * rpg + row_j) * a.ldo + h * HEAD_DIM + 2 * lane;
@@ -315,7 +417,7 @@ size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int /*rows_p
 }
 
 size_t attn_smem_bytes(int /*page_size*/) {
-    return (size_t)2 * ATT_KEYS * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4 + (size_t)RPG * ATT_KEYS * 4;
+    return (size_t)2 * ATT_KEYS * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4;
 }
 
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms) {
@@ -326,7 +428,7 @@ int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int nu
 }
 
 cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl) {
-    if (a.rows_per_group < 1 || a.rows_per_group > RPG || ATT_KEYS % a.page_size != 0 || a.n_splits < 1)
+    if (a.rows_per_group < 1 || a.rows_per_group > RPG || HALF_KEYS % a.page_size != 0 || a.n_splits < 1)
         return cudaErrorInvalidValue;
     static bool configured = false;
     const size_t smem = attn_smem_bytes(a.page_size);
