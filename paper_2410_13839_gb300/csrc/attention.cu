@@ -29,14 +29,17 @@
 namespace mtp {
 namespace {
 
-constexpr int ATT_THREADS = 256;
-constexpr int ATT_KEYS = 256;    // keys staged per batch: 32 KB of keys + 32 KB of values
+constexpr int ATT_THREADS = 128;  // four warps: four CTAs per SM
+constexpr int ATT_KEYS = 256;    // most keys staged at once (two halves; pages of 128 keys need 128 per half)
 constexpr int RPG = MAX_ROWS;    // rows per group, upper bound
 constexpr int PART = 2 + HEAD_DIM;  // (max, sum, out[64]) per row and split
 constexpr int MAX_SPLITS = 32;     // one warp lane per split in the merge
 static_assert(HEAD_DIM == 64, "score scale 0.125 assumes 64-wide heads");
 
-constexpr int HALF_KEYS = ATT_KEYS / 2;  // keys per staging half
+
+
+// keys per staging half: 64, or a whole page when pages are longer
+__host__ __device__ constexpr int half_keys(int page_size) { return page_size > 64 ? page_size : 64; }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
@@ -92,7 +95,7 @@ __device__ __forceinline__ bool stage_pages(const AttnArgs& a, int seq, int p_fr
     return true;
 }
 
-__global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;         // pages staged before the dependency wait
     __shared__ uint64_t hbar[2];     // the two staging halves
@@ -107,9 +110,10 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
     TraceEnd trace_guard(a.trace);
     const int H = a.n_heads, P = a.page_size, S = a.n_splits;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int HALF_KEYS = half_keys(P);  // keys per staging half
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem);
-    __nv_bfloat16* Vs = Ks + ATT_KEYS * HEAD_DIM;
-    float* qs = reinterpret_cast<float*>(Vs + ATT_KEYS * HEAD_DIM);  // [RPG][64], pre-scaled
+    __nv_bfloat16* Vs = Ks + 2 * HALF_KEYS * HEAD_DIM;
+    float* qs = reinterpret_cast<float*>(Vs + 2 * HALF_KEYS * HEAD_DIM);  // [RPG][64], pre-scaled
     const int pages_per_batch = HALF_KEYS / P;  // pages per staging half
     const long long kv_head_off = (long long)h * P * HEAD_DIM;
     const long long v_off = (long long)H * P * HEAD_DIM;
@@ -337,39 +341,51 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
         s_scale[w][j] = mw == -INFINITY ? 0.f : expf(mw - M);
     }
     __syncthreads();
-    const int row_j = warp;
-    const bool row_on = warp < RPG && s_act[min(warp, RPG - 1)];
-    float m_run = -INFINITY, l_run = 0.f, acc0 = 0.f, acc1 = 0.f;
-    if (warp < RPG) {
+    // rows warp, warp + NW, ...: (max, sum, output dims 2 lane, 2 lane + 1) over this CTA's keys
+    constexpr int RPW = (RPG + NW - 1) / NW;  // rows per warp
+    float m_run[RPW], l_run[RPW], acc0[RPW], acc1[RPW];
+#pragma unroll
+    for (int q = 0; q < RPW; ++q) {
+        const int row_j = warp + q * NW;
+        m_run[q] = -INFINITY;
+        l_run[q] = acc0[q] = acc1[q] = 0.f;
+        if (row_j >= RPG) continue;
 #pragma unroll
         for (int w = 0; w < NW; ++w) {
             const float sc = s_scale[w][row_j];
             const float* ws = wst + ((size_t)w * RPG + row_j) * PART;
-            m_run = fmaxf(m_run, ws[0]);
-            l_run = fmaf(sc, ws[1], l_run);
-            acc0 = fmaf(sc, ws[2 + 2 * lane], acc0);
-            acc1 = fmaf(sc, ws[3 + 2 * lane], acc1);
+            m_run[q] = fmaxf(m_run[q], ws[0]);
+            l_run[q] = fmaf(sc, ws[1], l_run[q]);
+            acc0[q] = fmaf(sc, ws[2 + 2 * lane], acc0[q]);
+            acc1[q] = fmaf(sc, ws[3 + 2 * lane], acc1[q]);
         }
     }
-
-    float* out_row = a.out + (size_t)(g * rpg + row_j) * a.ldo + h * HEAD_DIM + 2 * lane;
+    auto out_row = [&](int row_j) { return a.out + (size_t)(g * rpg + row_j) * a.ldo + h * HEAD_DIM + 2 * lane; };
     if (S == 1) {
-        if (row_on) {
-            out_row[0] = acc0 / l_run;
-            out_row[1] = acc1 / l_run;
+#pragma unroll
+        for (int q = 0; q < RPW; ++q) {
+            const int row_j = warp + q * NW;
+            if (row_j < RPG && s_act[row_j]) {
+                float* o = out_row(row_j);
+                o[0] = acc0[q] / l_run[q];
+                o[1] = acc1[q] / l_run[q];
+            }
         }
         return;
     }
 
     float* part = a.ws_part + (((size_t)(g * H + h) * S + sp) * RPG) * PART;
-    if (warp < RPG) {
-        float* pj = part + warp * PART;
+#pragma unroll
+    for (int q = 0; q < RPW; ++q) {
+        const int row_j = warp + q * NW;
+        if (row_j >= RPG) continue;
+        float* pj = part + row_j * PART;
         if (lane == 0) {
-            pj[0] = m_run;
-            pj[1] = l_run;
+            pj[0] = m_run[q];
+            pj[1] = l_run[q];
         }
-        pj[2 + 2 * lane] = acc0;
-        pj[3 + 2 * lane] = acc1;
+        pj[2 + 2 * lane] = acc0[q];
+        pj[3 + 2 * lane] = acc1[q];
     }
     __threadfence();
     __syncthreads();
@@ -378,7 +394,9 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
     if (!s_last) return;
     __threadfence();
 
-    if (row_on) {
+#pragma unroll 1
+    for (int row_j = warp; row_j < RPG; row_j += NW) {
+        if (!s_act[row_j]) continue;
         // lane s holds split s's (max, sum); every split's output pair is
         // loaded before any is used, so the merge costs one L2 round trip
         const float* base = a.ws_part + ((size_t)(g * H + h) * S * RPG) * PART + row_j * PART;
@@ -390,22 +408,23 @@ __global__ void __launch_bounds__(ATT_THREADS, 2) attn_kernel(const AttnArgs a) 
         }
         float o0[MAX_SPLITS], o1[MAX_SPLITS];
 #pragma unroll
-        for (int s = 0; s < MAX_SPLITS; ++s) {
-            o0[s] = s < S ? __ldcg(base + s * sstride + 2 + 2 * lane) : 0.f;
-            o1[s] = s < S ? __ldcg(base + s * sstride + 3 + 2 * lane) : 0.f;
+        for (int sx = 0; sx < MAX_SPLITS; ++sx) {
+            o0[sx] = sx < S ? __ldcg(base + sx * sstride + 2 + 2 * lane) : 0.f;
+            o1[sx] = sx < S ? __ldcg(base + sx * sstride + 3 + 2 * lane) : 0.f;
         }
         const float M = warp_max(ms);
         const float w = (ms == -INFINITY) ? 0.f : expf(ms - M);
         const float L = warp_sum(w * ls);
         float r0 = 0.f, r1 = 0.f;
 #pragma unroll
-        for (int s = 0; s < MAX_SPLITS; ++s) {
-            const float ws = __shfl_sync(FULL_MASK, w, s);
-            r0 = fmaf(ws, o0[s], r0);
-            r1 = fmaf(ws, o1[s], r1);
+        for (int sx = 0; sx < MAX_SPLITS; ++sx) {
+            const float ws = __shfl_sync(FULL_MASK, w, sx);
+            r0 = fmaf(ws, o0[sx], r0);
+            r1 = fmaf(ws, o1[sx], r1);
         }
-        out_row[0] = r0 / L;
-        out_row[1] = r1 / L;
+        float* o = out_row(row_j);
+        o[0] = r0 / L;
+        o[1] = r1 / L;
     }
     if (tid == 0) a.ws_count[g * H + h] = 0;
 }
@@ -416,8 +435,8 @@ size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int /*rows_p
     return (size_t)groups * n_heads * n_splits * RPG * PART;
 }
 
-size_t attn_smem_bytes(int /*page_size*/) {
-    return (size_t)2 * ATT_KEYS * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4;
+size_t attn_smem_bytes(int page_size) {
+    return (size_t)4 * half_keys(page_size) * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4;
 }
 
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms) {
@@ -428,14 +447,15 @@ int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int nu
 }
 
 cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl) {
-    if (a.rows_per_group < 1 || a.rows_per_group > RPG || HALF_KEYS % a.page_size != 0 || a.n_splits < 1)
+    if (a.rows_per_group < 1 || a.rows_per_group > RPG || half_keys(a.page_size) % a.page_size != 0 ||
+        a.n_splits < 1)
         return cudaErrorInvalidValue;
-    static bool configured = false;
+    static size_t configured = 0;
     const size_t smem = attn_smem_bytes(a.page_size);
-    if (!configured) {
+    if (configured < smem) {
         cudaError_t e = cudaFuncSetAttribute(attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        configured = true;
+        configured = smem;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.n_splits, a.n_heads, groups);

@@ -89,7 +89,12 @@ __global__ void __launch_bounds__(PK_THREADS) pack_rows_kernel(const PackArgs a)
     }
 }
 
-__global__ void __launch_bounds__(PK_THREADS) qkv_finish_kernel(const QkvFinishArgs a) {
+constexpr int QF_THREADS = 128;
+
+// One CTA per row; each thread takes 8 consecutive features (one 16-byte
+// chunk of a key/value row): two float4 loads, then the query as two float4
+// stores or the key/value chunk as one 16-byte store at its swizzled place.
+__global__ void __launch_bounds__(QF_THREADS) qkv_finish_kernel(const QkvFinishArgs a) {
     const int r = blockIdx.x, tid = threadIdx.x;
     TraceEnd trace_guard(a.trace);
     pdl_launch_dependents();
@@ -104,27 +109,39 @@ __global__ void __launch_bounds__(PK_THREADS) qkv_finish_kernel(const QkvFinishA
         if (page < 0 && tid == 0) atomicOr(a.err, ERR_BOUNDS);
     }
     const int t = pos % P;
-    for (int i = tid; i < 3 * d; i += PK_THREADS) {
-        const float y = row[i];
-        row[i] = 0.f;
+    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = tid; c < 3 * d / 8; c += QF_THREADS) {
+        float4* src = reinterpret_cast<float4*>(row + c * 8);
+        const float4 y0 = src[0], y1 = src[1];
+        src[0] = zero;
+        src[1] = zero;
         if (seq < 0) continue;
-        const int h = i / (3 * HEAD_DIM), sec = (i / HEAD_DIM) % 3, dd = i % HEAD_DIM;
+        const int i = c * 8, h = i / (3 * HEAD_DIM), sec = (i / HEAD_DIM) % 3, dd = i % HEAD_DIM;
         if (sec == 0) {
-            a.q[(size_t)r * d + h * HEAD_DIM + dd] = y;
+            float4* q = reinterpret_cast<float4*>(a.q + (size_t)r * d + h * HEAD_DIM + dd);
+            q[0] = y0;
+            q[1] = y1;
         } else if (page >= 0) {
+            uint4 pk;
+            auto pair = [](float lo, float hi) {
+                return (uint32_t)f32_to_bf16_bits(lo) | ((uint32_t)f32_to_bf16_bits(hi) << 16);
+            };
+            pk.x = pair(y0.x, y0.y);
+            pk.y = pair(y0.z, y0.w);
+            pk.z = pair(y1.x, y1.y);
+            pk.w = pair(y1.z, y1.w);
             const long long idx = (long long)page * a.page_elems + a.layer_off + (long long)(sec - 1) * H * P * HEAD_DIM +
-                                  (long long)h * P * HEAD_DIM + (long long)t * HEAD_DIM +
-                                  ((((dd >> 3) ^ (t & 7)) << 3) | (dd & 7));
-            reinterpret_cast<uint16_t*>(a.kv_pool)[idx] = f32_to_bf16_bits(y);
+                                  (long long)h * P * HEAD_DIM + (long long)t * HEAD_DIM + (((dd >> 3) ^ (t & 7)) << 3);
+            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(a.kv_pool) + idx) = pk;
         }
     }
 }
 
 template <typename K, typename A>
-cudaError_t launch_rows(K kern, const A& args, int rows, cudaStream_t s, bool pdl) {
+cudaError_t launch_rows(K kern, const A& args, int rows, cudaStream_t s, bool pdl, int threads = PK_THREADS) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(rows);
-    cfg.blockDim = dim3(PK_THREADS);
+    cfg.blockDim = dim3(threads);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -143,7 +160,7 @@ cudaError_t launch_pack_rows(const PackArgs& a, cudaStream_t s, bool pdl) {
 
 cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl) {
     if (a.m < 1) return cudaErrorInvalidValue;
-    return launch_rows(qkv_finish_kernel, a, a.m, s, pdl);
+    return launch_rows(qkv_finish_kernel, a, a.m, s, pdl, QF_THREADS);
 }
 
 }  // namespace mtp

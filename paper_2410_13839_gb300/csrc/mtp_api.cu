@@ -111,6 +111,7 @@ struct mtp_ctx {
     float* d_bws = nullptr;  // attention split partials
     int* d_bwc = nullptr;    // attention split counters
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
+    int gemm_max_splits = 16;
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -271,12 +272,13 @@ int run_layers(mtp_ctx* c, int M, int G, int rpg, int plan, int seq_base, int va
     return MTP_OK;
 }
 
-// K splits of a tensor-core GEMM: as many as keep one wave of CTAs (one per SM)
-// with a whole number of 64-wide k-chunks each.
+// K splits of a tensor-core GEMM: as many as keep one wave of CTAs (one per
+// SM) with a whole number of 64-wide k-chunks each, up to c->gemm_max_splits
+// (every split adds its partial tile to the output with fp32 atomics).
 int gemm_splits(const mtp_ctx* c, int n_w, int k, int ntiles) {
     const int tiles = n_w / 128 * ntiles, chunks = k / 64;
     int s = 1;
-    while (chunks % (2 * s) == 0 && tiles * 2 * s <= c->num_sms) s *= 2;
+    while (2 * s <= c->gemm_max_splits && chunks % (2 * s) == 0 && tiles * 2 * s <= c->num_sms) s *= 2;
     return s;
 }
 
@@ -875,6 +877,11 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
     } else if (option == MTP_OPT_L2_PREFETCH) {
         changed = c->use_l2_prefetch != (value != 0);
         c->use_l2_prefetch = value != 0;
+    } else if (option == MTP_OPT_GEMM_SPLITS) {
+        if (value < 1 || value > 64 || (value & (value - 1)))
+            return fail(MTP_ERR_INVALID, "GEMM splits %d: need a power of two in 1..64", value);
+        changed = c->gemm_max_splits != value;
+        c->gemm_max_splits = value;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -911,6 +918,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_L2_PREFETCH: *value = c->use_l2_prefetch; break;
         case MTP_OPT_MLP_CLUSTERS: *value = c->mlp_clusters; break;
         case MTP_OPT_BATCHED: *value = c->use_batched && c->batched_ok; break;
+        case MTP_OPT_GEMM_SPLITS: *value = c->gemm_max_splits; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;

@@ -203,27 +203,37 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
 
     // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
-    const bool fin = mbar_wait(&done, 0, a.err);
+    const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
     tc_fence_after();
-    __syncthreads();
     if (fin && s_ok) {
-        const int f = tile * TC_M + warp * 32 + lane;
-        const float bias = a.bias && split == 0 ? a.bias[f] : 0.f;
+        // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them),
+        // then float4 rows of T -> out, coalesced
+        constexpr int TP = TC_M + 4;  // row pitch (floats)
+        float* T = reinterpret_cast<float*>(smem);
 #pragma unroll 1
         for (int j0 = 0; j0 < NT; j0 += 32) {
             float v[32];
             tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)j0, v);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const int n = arow + j0 + j;
-                if (n < a.m) {
-                    float* o = a.out + (size_t)n * a.ldo + f;
-                    if (a.accumulate)
-                        atomicAdd(o, v[j] + bias);
-                    else
-                        *o = v[j] + bias;
-                }
+            for (int j = 0; j < 32; ++j) T[(j0 + j) * TP + warp * 32 + lane] = v[j];
+        }
+        __syncthreads();
+        const int rows = min(NT, a.m - arow);
+        for (int i = tid; i < rows * (TC_M / 4); i += TC_THREADS) {
+            const int j = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
+            const int f = tile * TC_M + f4;
+            float4 y = *reinterpret_cast<const float4*>(T + j * TP + f4);
+            if (a.bias && split == 0) {
+                y.x += a.bias[f];
+                y.y += a.bias[f + 1];
+                y.z += a.bias[f + 2];
+                y.w += a.bias[f + 3];
             }
+            float4* o = reinterpret_cast<float4*>(a.out + (size_t)(arow + j) * a.ldo + f);
+            if (a.accumulate)
+                atomicAdd(o, y);
+            else
+                *o = y;
         }
     } else if (!fin) {
         // the MMAs may still be running: wait for them (bounded) before freeing TMEM
