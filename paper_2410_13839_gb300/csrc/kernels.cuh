@@ -209,14 +209,26 @@ cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------ tensor-core GEMM ----
 // out[n][f] (+)= sum_k (a_hi[n][k] + a_lo[n][k]) w[f][k] with tcgen05 (tc_gemm.cu).
+enum TcEpilogue : int {
+    TC_STORE = 0,     // out[n][f] = acc + bias (one K split only)
+    TC_ACCUM = 1,     // out[n][f] += acc (+ bias from K split 0), fp32 atomics
+    TC_QKV = 2,       // q|k|v rows (head-major features): q -> q_out, k and v -> the paged cache (one K split)
+    TC_GELU_PACK = 3  // GELU(acc + bias) as bf16 hi + lo rows -> pack_hi / pack_lo (one K split)
+};
 struct TcGemmArgs {
-    float* out; int ldo;          // [m][ldo] fp32, column f = weight row
+    float* out; int ldo;          // [m][ldo] fp32, column f = weight row (TC_STORE, TC_ACCUM; TC_QKV: queries)
     const float* bias;            // [n_w] added once (by K split 0), or null
     int m;                        // activation rows
     int k_chunks;                 // 64-wide k-chunks per CTA (K / 64 / splits)
     int w_rows_per_kchunk;        // 0: weight k-chunk kc at columns 64 kc; else at rows kc * this (W_o per head)
-    int accumulate;               // 1: atomicAdd into out; 0: store (one K split only)
+    int epilogue;                 // TcEpilogue
+    const int* row_seq; const int* row_pos;   // TC_QKV, TC_GELU_PACK: rows of no sequence are skipped / zero
+    // TC_QKV: the paged cache (chunk c of key row t stored at c ^ (t & 7))
+    __nv_bfloat16* kv_pool; long long page_elems; long long layer_off; int page_size, n_heads;
+    const int* block_table; int bt_stride;
+    __nv_bfloat16* pack_hi; __nv_bfloat16* pack_lo;  // TC_GELU_PACK: [m][n_w]
     int* err;
+    unsigned long long* trace;
 };
 struct TcGemm {
     CUtensorMap w, a_hi, a_lo;    // boxes: 64 x 128 weight rows, 64 x nt activation rows

@@ -111,7 +111,7 @@ struct mtp_ctx {
     float* d_bws = nullptr;  // attention split partials
     int* d_bwc = nullptr;    // attention split counters
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
-    int gemm_max_splits = 16;
+    int gemm_max_splits = 4;
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -292,10 +292,13 @@ int tile_index(int nt) { return nt == 32 ? 0 : (nt == 64 ? 1 : 2); }
 int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStream_t s, bool pdl, Prof* prof) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
-    const int nt = tc_tile_rows(M), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
+    // 32-row activation tiles: the four projections each run one wave of CTAs with
+    // few K splits, and the q|k|v and W1 projections finish their rows in the epilogue
+    const int nt = 32, ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
     for (int l = 0; l < cf.layers; ++l) {
         const Layer& L = c->layers[l];
         const mtp_ctx::LayerMaps& W = c->lmaps[l];
+        const long long layer_off = (long long)l * 2 * H * P * HEAD_DIM;
         auto pack = [&](int mode, const float* x, int k, const float* g, const float* bta, float* zero,
                         __nv_bfloat16* hi, __nv_bfloat16* lo) -> int {
             PackArgs pa;
@@ -306,38 +309,37 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
             LAUNCH(MTP_K_PACK, launch_pack_rows(pa, s, pdl));
             return MTP_OK;
         };
-        auto gemm = [&](const CUtensorMap& w, int n_w, int k, bool a_is_u, float* out, int ldo, const float* bias,
-                        int w_rows_per_kchunk) -> int {
+        auto gemm = [&](const CUtensorMap& w, int n_w, int k, bool a_is_u, int epilogue, float* out, int ldo,
+                        const float* bias, int w_rows_per_kchunk) -> int {
             TcGemm g;
+            std::memset(&g, 0, sizeof(g));
             g.w = w;
             g.a_hi = a_is_u ? c->umap_hi[ti] : c->amap_hi[ti];
             g.a_lo = a_is_u ? c->umap_lo[ti] : c->amap_lo[ti];
             g.n_w = n_w; g.nt = nt;
-            g.splits = gemm_splits(c, n_w, k, ntiles);
-            g.args.out = out; g.args.ldo = ldo; g.args.bias = bias; g.args.m = M;
-            g.args.k_chunks = k / 64 / g.splits; g.args.w_rows_per_kchunk = w_rows_per_kchunk;
-            g.args.accumulate = 1; g.args.err = c->d_err;
+            g.splits = epilogue == TC_ACCUM ? gemm_splits(c, n_w, k, ntiles) : 1;
+            TcGemmArgs& ga = g.args;
+            ga.out = out; ga.ldo = ldo; ga.bias = bias; ga.m = M;
+            ga.k_chunks = k / 64 / g.splits; ga.w_rows_per_kchunk = w_rows_per_kchunk;
+            ga.epilogue = epilogue; ga.err = c->d_err;
+            ga.row_seq = c->d_row_seq; ga.row_pos = c->d_row_pos;
+            ga.kv_pool = reinterpret_cast<__nv_bfloat16*>(c->d_kv); ga.page_elems = c->page_elems;
+            ga.layer_off = layer_off; ga.page_size = P; ga.n_heads = H;
+            ga.block_table = c->d_block_table; ga.bt_stride = c->pages_per_seq;
+            ga.pack_hi = c->d_uhi; ga.pack_lo = c->d_ulo;
+            ga.trace = tslot(c, MTP_K_GEMM);
             LAUNCH(MTP_K_GEMM, launch_tc_gemm(g, s, pdl));
             return MTP_OK;
         };
-        // LN1 -> q|k|v (split-K accumulation into the zeroed buffer, bias once)
+        // LN1 -> q|k|v: queries out, keys and values appended to the cache
         MTP_TRY(pack(PACK_LN, c->d_bx, d, L.ln1_g, L.ln1_b, nullptr, c->d_ahi, c->d_alo));
-        MTP_TRY(gemm(W.wqkv, 3 * d, d, false, c->d_bqkv, 3 * d, L.bqkv, 0));
-        QkvFinishArgs qf;
-        std::memset(&qf, 0, sizeof(qf));
-        qf.qkv = c->d_bqkv; qf.q = c->d_bq;
-        qf.kv_pool = reinterpret_cast<__nv_bfloat16*>(c->d_kv); qf.page_elems = c->page_elems;
-        qf.layer_off = (long long)l * 2 * H * P * HEAD_DIM; qf.page_size = P; qf.n_heads = H;
-        qf.block_table = c->d_block_table; qf.bt_stride = c->pages_per_seq;
-        qf.row_seq = c->d_row_seq; qf.row_pos = c->d_row_pos; qf.m = M; qf.err = c->d_err;
-        qf.trace = tslot(c, MTP_K_QKV);
-        LAUNCH(MTP_K_QKV, launch_qkv_finish(qf, s, pdl));
-        // attention of every slot's fed rows over its cached keys
+        MTP_TRY(gemm(W.wqkv, 3 * d, d, false, TC_QKV, c->d_bq, d, L.bqkv, 0));
+        // attention of every group's fed rows over its cached keys
         AttnArgs at;
         std::memset(&at, 0, sizeof(at));
         at.q = c->d_bq; at.ldq = d;
         at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(c->d_kv); at.page_elems = c->page_elems;
-        at.layer_off = qf.layer_off;
+        at.layer_off = layer_off;
         at.block_table = c->d_block_table; at.bt_stride = c->pages_per_seq;
         at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
         at.out = c->d_batt; at.ldo = d;
@@ -352,12 +354,11 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         LAUNCH(MTP_K_ATTN, launch_attention(at, groups, s, pdl));
         // x += attention W_o^T + b_o (the per-head W_o blocks are the k-chunks)
         MTP_TRY(pack(PACK_COPY, c->d_batt, d, nullptr, nullptr, nullptr, c->d_ahi, c->d_alo));
-        MTP_TRY(gemm(W.wo, d, d, false, c->d_bx, d, L.bo, d));
-        // x += GELU(LN2(x) W1^T + b1) W2^T + b2
+        MTP_TRY(gemm(W.wo, d, d, false, TC_ACCUM, c->d_bx, d, L.bo, d));
+        // x += GELU(LN2(x) W1^T + b1) W2^T + b2 (W1's epilogue writes the GELU rows as bf16 hi + lo)
         MTP_TRY(pack(PACK_LN, c->d_bx, d, L.ln2_g, L.ln2_b, nullptr, c->d_ahi, c->d_alo));
-        MTP_TRY(gemm(W.w1, F, d, false, c->d_bh, F, L.b1, 0));
-        MTP_TRY(pack(PACK_GELU, c->d_bh, F, nullptr, nullptr, c->d_bh, c->d_uhi, c->d_ulo));
-        MTP_TRY(gemm(W.w2, d, F, true, c->d_bx, d, L.b2, 0));
+        MTP_TRY(gemm(W.w1, F, d, false, TC_GELU_PACK, nullptr, F, L.b1, 0));
+        MTP_TRY(gemm(W.w2, d, F, true, TC_ACCUM, c->d_bx, d, L.b2, 0));
     }
     return MTP_OK;
 }

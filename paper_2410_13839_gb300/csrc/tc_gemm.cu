@@ -22,6 +22,7 @@
 #include <cuda.h>
 
 #include <cstdio>
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -33,7 +34,9 @@ namespace {
 
 constexpr int TC_M = 128;      // weight rows per CTA (MMA M)
 constexpr int TC_K = 64;       // k per stage: one 128-byte swizzle row of bf16
-constexpr int TC_STAGES = 4;
+// ring stages per activation tile size: about 190 KB of copies in flight per CTA
+__host__ __device__ constexpr int tc_stages(int nt) { return nt <= 32 ? 8 : (nt <= 64 ? 6 : 4); }
+constexpr int TC_MAX_STAGES = 8;
 constexpr int TC_THREADS = 128;
 constexpr uint32_t TC_W_BYTES = TC_M * TC_K * 2;
 
@@ -111,10 +114,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     constexpr uint32_t A_BYTES = NT * TC_K * 2, STAGE = TC_W_BYTES + 2 * A_BYTES;
     constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
-    __shared__ uint64_t full[TC_STAGES], empty[TC_STAGES], done;
+    constexpr int TC_STAGES = tc_stages(NT);
+    __shared__ uint64_t full[TC_MAX_STAGES], empty[TC_MAX_STAGES], done;
     __shared__ uint32_t tmem_base;
     __shared__ int s_ok;
+    __shared__ long long s_rowbase[NT];  // TC_QKV: element offset of the row's key row in its page (-1: none)
+    __shared__ int s_rowt[NT];           // TC_QKV: key row within the page; TC_GELU_PACK: row of a sequence
     unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    TraceEnd trace_guard(a.trace);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int tile = blockIdx.x, split = blockIdx.y, ntile = blockIdx.z;
     const int chunks = a.k_chunks;
@@ -162,7 +169,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     pdl_launch_dependents();
     pdl_wait();
+    trace_wait(a.trace);
 
+    // The elected lanes run the ring; the rest of warps 0 and 1 wait at __syncwarp
+    // (not in the barrier poll below, which would hold up their elected lane).
     if (tid == 0) {  // producer: activations of the first stages, then the rest of the ring
         for (int c = 0; c < chunks; ++c) {
             const int s = c % TC_STAGES;
@@ -201,11 +211,29 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (c < chunks) s_ok = 0;
         tc_commit(&done);  // every MMA issued above has completed
     }
+    if (warp < 2) __syncwarp();
 
     // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
     const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
     tc_fence_after();
     if (fin && s_ok) {
+        if (tid < NT && (a.epilogue == TC_QKV || a.epilogue == TC_GELU_PACK)) {  // per-row facts, once
+            const int n = arow + tid;
+            const int seq = n < a.m ? a.row_seq[n] : -1;
+            long long base = -1;
+            int t = 0;
+            if (a.epilogue == TC_QKV && seq >= 0) {
+                const int pos = a.row_pos[n];
+                t = pos % a.page_size;
+                const int page = a.block_table[(size_t)seq * a.bt_stride + pos / a.page_size];
+                if (page < 0)
+                    atomicOr(a.err, ERR_BOUNDS);
+                else
+                    base = (long long)page * a.page_elems + a.layer_off + (long long)t * HEAD_DIM;
+            }
+            s_rowbase[tid] = seq >= 0 ? base : -2;  // -2: no sequence
+            s_rowt[tid] = a.epilogue == TC_QKV ? t : (seq >= 0);
+        }
         // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them),
         // then float4 rows of T -> out, coalesced
         constexpr int TP = TC_M + 4;  // row pitch (floats)
@@ -219,9 +247,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
         __syncthreads();
         const int rows = min(NT, a.m - arow);
+        const int P = a.page_size, H = a.n_heads, d = H * HEAD_DIM;
         for (int i = tid; i < rows * (TC_M / 4); i += TC_THREADS) {
             const int j = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
-            const int f = tile * TC_M + f4;
+            const int f = tile * TC_M + f4, n = arow + j;
             float4 y = *reinterpret_cast<const float4*>(T + j * TP + f4);
             if (a.bias && split == 0) {
                 y.x += a.bias[f];
@@ -229,11 +258,42 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 y.z += a.bias[f + 2];
                 y.w += a.bias[f + 3];
             }
-            float4* o = reinterpret_cast<float4*>(a.out + (size_t)(arow + j) * a.ldo + f);
-            if (a.accumulate)
-                atomicAdd(o, y);
-            else
-                *o = y;
+            if (a.epilogue == TC_ACCUM) {
+                atomicAdd(reinterpret_cast<float4*>(a.out + (size_t)n * a.ldo + f), y);
+            } else if (a.epilogue == TC_STORE) {
+                *reinterpret_cast<float4*>(a.out + (size_t)n * a.ldo + f) = y;
+            } else if (a.epilogue == TC_QKV) {  // features h*192 + {q,k,v}*64 + dd
+                const long long base = s_rowbase[j];
+                if (base == -2) continue;  // no sequence
+                const int h = f / (3 * HEAD_DIM), sec = (f / HEAD_DIM) % 3, dd = f % HEAD_DIM;
+                if (sec == 0) {
+                    *reinterpret_cast<float4*>(a.out + (size_t)n * d + h * HEAD_DIM + dd) = y;
+                    continue;
+                }
+                if (base < 0) continue;  // unreserved page (reported)
+                const int t = s_rowt[j];
+                const long long idx = base + (long long)(sec - 1) * H * P * HEAD_DIM + (long long)h * P * HEAD_DIM +
+                                      ((((dd >> 3) ^ (t & 7)) << 3) | (dd & 7));
+                uint2 pk;
+                pk.x = (uint32_t)f32_to_bf16_bits(y.x) | ((uint32_t)f32_to_bf16_bits(y.y) << 16);
+                pk.y = (uint32_t)f32_to_bf16_bits(y.z) | ((uint32_t)f32_to_bf16_bits(y.w) << 16);
+                *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(a.kv_pool) + idx) = pk;
+            } else {  // TC_GELU_PACK
+                const bool on = s_rowt[j] != 0;
+                const float v[4] = {on ? gelu_erf(y.x) : 0.f, on ? gelu_erf(y.y) : 0.f, on ? gelu_erf(y.z) : 0.f,
+                                    on ? gelu_erf(y.w) : 0.f};
+                uint32_t hi[2], lo[2];
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                    const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * q]), h1 = __float2bfloat16_rn(v[2 * q + 1]);
+                    const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * q] - __bfloat162float(h0));
+                    const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * q + 1] - __bfloat162float(h1));
+                    hi[q] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+                    lo[q] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+                }
+                *reinterpret_cast<uint2*>(a.pack_hi + (size_t)n * a.ldo + f) = make_uint2(hi[0], hi[1]);
+                *reinterpret_cast<uint2*>(a.pack_lo + (size_t)n * a.ldo + f) = make_uint2(lo[0], lo[1]);
+            }
         }
     } else if (!fin) {
         // the MMAs may still be running: wait for them (bounded) before freeing TMEM
@@ -265,7 +325,7 @@ EncodeTiled encode_fn() {
 
 template <int NT>
 size_t tc_smem() {
-    return (size_t)TC_STAGES * (TC_W_BYTES + 2u * NT * TC_K * 2) + 1024;
+    return (size_t)tc_stages(NT) * (TC_W_BYTES + 2u * NT * TC_K * 2) + 1024;
 }
 
 template <int NT>
@@ -314,7 +374,7 @@ int tc_tile_rows(int m) { return m <= 32 ? 32 : (m <= 64 ? 64 : 128); }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl) {
     if (g.n_w % TC_M || g.args.k_chunks < 1 || g.splits < 1 || g.args.m < 1) return cudaErrorInvalidValue;
-    if (!g.args.accumulate && g.splits != 1) return cudaErrorInvalidValue;
+    if (g.args.epilogue != TC_ACCUM && g.splits != 1) return cudaErrorInvalidValue;
     switch (g.nt) {
         case 32: return launch_nt<32>(g, s, pdl);
         case 64: return launch_nt<64>(g, s, pdl);
@@ -344,6 +404,7 @@ extern "C" MTP_API int mtp_gemm_bf16x2(const void* w, const void* a_hi, const vo
         return gemm_fail(MTP_ERR_INVALID, "mtp_gemm_bf16x2: n_w=%d k=%d m=%d splits=%d accumulate=%d", n_w, k, m,
                          splits, accumulate);
     TcGemm g;
+    std::memset(&g, 0, sizeof(g));
     g.n_w = n_w;
     g.splits = splits;
     g.nt = tc_tile_rows(m);
@@ -353,7 +414,7 @@ extern "C" MTP_API int mtp_gemm_bf16x2(const void* w, const void* a_hi, const vo
     g.args.m = m;
     g.args.k_chunks = k / TC_K / splits;
     g.args.w_rows_per_kchunk = 0;
-    g.args.accumulate = accumulate;
+    g.args.epilogue = accumulate ? TC_ACCUM : TC_STORE;
     int* d_err = nullptr;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaMallocAsync(&d_err, sizeof(int), st) != cudaSuccess)
