@@ -183,7 +183,7 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        pass (8 rows) run the batched path: tensor-core projections over all
  *                        rows at once (bf16 weights only; default); 0 = fused passes of 8 rows
  *   MTP_OPT_GEMM_SPLITS  most K splits of a batched-path projection (power of two 1..64; each
- *                        split adds its partial tile with fp32 atomics; default 4) */
+ *                        split adds its partial tile with fp32 atomics; default 16) */
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
     MTP_OPT_GEMM_SPLITS = 5

@@ -111,7 +111,7 @@ struct mtp_ctx {
     float* d_bws = nullptr;  // attention split partials
     int* d_bwc = nullptr;    // attention split counters
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
-    int gemm_max_splits = 4;
+    int gemm_max_splits = 16;
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -292,9 +292,11 @@ int tile_index(int nt) { return nt == 32 ? 0 : (nt == 64 ? 1 : 2); }
 int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStream_t s, bool pdl, Prof* prof) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
-    // 32-row activation tiles: the four projections each run one wave of CTAs with
-    // few K splits, and the q|k|v and W1 projections finish their rows in the epilogue
-    const int nt = 32, ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
+    // activation tiles: a weight tile is streamed once per activation tile.  32-row
+    // tiles keep enough CTAs streaming where K is short (q|k|v and W1 finish their
+    // rows in the epilogue, one K split; W_o splits K); W2 (K = 4 d) takes whole
+    // 128-row tiles and splits its long K instead
+    auto tile_rows = [&](int k) { return std::min(k > 1024 ? 128 : 32, tc_tile_rows(M)); };
     for (int l = 0; l < cf.layers; ++l) {
         const Layer& L = c->layers[l];
         const mtp_ctx::LayerMaps& W = c->lmaps[l];
@@ -311,6 +313,7 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         };
         auto gemm = [&](const CUtensorMap& w, int n_w, int k, bool a_is_u, int epilogue, float* out, int ldo,
                         const float* bias, int w_rows_per_kchunk) -> int {
+            const int nt = tile_rows(k), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
             TcGemm g;
             std::memset(&g, 0, sizeof(g));
             g.w = w;
