@@ -18,6 +18,17 @@ Parity pins (tests/test_oracle_mtp.py): n = 1 equals a plain greedy AR loop
 written separately, token for token; the first i heads at n = N give the same
 distributions as a run at n = i; the KV cache equals a cache-free recompute;
 append-rollback-append equals append.
+
+VERIFY_GREEDY (policy 1; speculative decoding with the heads as drafter,
+the paper's "speculative decoding" framing, Sec. I, II): each step feeds the
+confirmed token c and the drafts d_1..d_m proposed by the previous step.
+Head 1's argmax g_j at fed row j (c for j = 0, d_j after) is the greedy
+token after that row, so the drafts are kept while d_{j+1} = g_j; with a kept
+drafts, the other m - a cache rows are rolled back and the step emits
+d_1..d_a and then g_a.  The next drafts are the Viterbi path over the heads
+at the last kept row with position 1 forced to g_a (its top-1 candidate), so
+c' = g_a and d'_t = path[t].  The emitted sequence is the greedy AR
+sequence for every n and k (pinned in tests/test_oracle_verify.py).
 """
 from __future__ import annotations
 
@@ -43,6 +54,23 @@ class StepRecord:
     accepted: int
     done: bool
     margin: float            # min(top-k gap over heads, Viterbi runner-up gap)
+
+
+@dataclasses.dataclass
+class VerifyRecord:
+    """One VERIFY_GREEDY step."""
+    fed: np.ndarray          # [c, d_1..d_m] (empty on the first step)
+    greedy: np.ndarray       # head 1's argmax at every fed row (float32 scores)
+    kept: int                # drafts kept (a)
+    rollback: int            # cache rows rolled back (m - a)
+    emitted: np.ndarray      # d_1..d_a, g_a (cut at EOS / budget)
+    logits: np.ndarray       # [n, V] float64 heads at the last kept row
+    lse: np.ndarray
+    logp32: np.ndarray
+    cand_ids: np.ndarray     # [n, k]
+    cand_logp: np.ndarray    # [n, k], position 1 forced to its top-1
+    path: np.ndarray         # [n]: next step's confirmed token and drafts
+    done: bool
 
 
 class MTPOracle:
@@ -94,6 +122,52 @@ class MTPOracle:
         self.done = done
         return StepRecord(np.asarray(fed, np.int32), logits, lse, logp32, ids, vals, path,
                           a, done, margin)
+
+    # ---- VERIFY_GREEDY ----
+    def propose(self, n: int, k: int):
+        """Heads at h_last with position 1 forced to head 1's top-1 (the greedy token)."""
+        logits = head_logits(self.h_last, self.w, n, self.cfg.ln_eps)
+        logp, lse = log_softmax(logits)
+        logp32 = logp.astype(np.float32)
+        ids, vals = top_k_rows(logp32, k)
+        vals = vals.copy()
+        vals[0, 1:] = -np.inf  # position 1: the greedy token only
+        path, _, _ = viterbi(ids[None], vals[None], self.log_q)
+        return logits, lse, logp32, ids, vals, path[0]
+
+    def step_verify(self, n: int, k: int) -> "VerifyRecord":
+        """One VERIFY_GREEDY step (see the module docstring)."""
+        fed = self.pending
+        m = max(0, len(fed) - 1)  # drafts fed
+        g = np.zeros(0, np.int32)
+        if len(fed):
+            h = self.model.forward(np.asarray(fed, np.int64), np.zeros(len(fed), bool), self.cache)
+            l1 = np.stack([head_logits(h[j], self.w, 1, self.cfg.ln_eps)[0] for j in range(len(fed))])  # head 1
+            lp1 = log_softmax(l1)[0].astype(np.float32)
+            g = np.array([top_k_rows(lp1[j:j + 1], 1)[0][0, 0] for j in range(len(fed))], np.int32)
+            a = 0
+            while a < m and int(fed[a + 1]) == int(g[a]):
+                a += 1
+            self.cache.rollback(m - a)
+            self.h_last = h[a]
+        else:
+            a = 0
+        logits, lse, logp32, ids, vals, path = self.propose(n, k)
+        emit = [int(t) for t in fed[1:a + 1]] + [int(path[0])]
+        e, done = accept_all(np.asarray(emit, np.int32), self.cfg.eos_id, self.remaining)
+        emitted = np.asarray(emit[:e], np.int32)
+        self.generated.extend(int(t) for t in emitted)
+        self.remaining -= e
+        self.done = done
+        self.pending = np.zeros(0, np.int32) if done else path.astype(np.int32)
+        return VerifyRecord(np.asarray(fed, np.int32), g, a, m - a, emitted, logits, lse, logp32, ids, vals,
+                            path, done)
+
+    def generate_verify(self, n: int, k: int, max_steps: int | None = None) -> list["VerifyRecord"]:
+        records = []
+        while not self.done and (max_steps is None or len(records) < max_steps):
+            records.append(self.step_verify(n, k))
+        return records
 
     def generate(self, n: int, k: int, max_steps: int | None = None) -> list[StepRecord]:
         records = []
