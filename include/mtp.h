@@ -46,10 +46,18 @@ typedef enum mtp_status {
 
 typedef enum mtp_dtype { MTP_F32 = 0, MTP_BF16 = 1 } mtp_dtype;
 
-/* Acceptance of the selected path (Sec. III-C): the paper accepts the whole
- * Viterbi path each step; it is cut after the first EOS and at the
- * sequence's remaining token budget. */
-typedef enum mtp_accept { MTP_ACCEPT_ALL = 0 } mtp_accept;
+/* Acceptance of the selected path (Sec. III-C).
+ *   MTP_ACCEPT_ALL      the paper's rule: the whole Viterbi path is accepted each
+ *                       step, cut after the first EOS and at the remaining budget.
+ *   MTP_VERIFY_GREEDY   speculative decoding with the heads as drafter (the
+ *                       "speculative decoding" framing of Sec. I-II): a step feeds
+ *                       the confirmed token and the drafts of the previous step,
+ *                       keeps the drafts while each equals head 1's argmax at the
+ *                       row before it, rolls back the cache rows of the rest, and
+ *                       emits the kept drafts plus head 1's argmax at the last kept
+ *                       row.  The next drafts are the Viterbi path with position 1
+ *                       forced to that argmax.  The output equals greedy AR decoding. */
+typedef enum mtp_accept { MTP_ACCEPT_ALL = 0, MTP_VERIFY_GREEDY = 1 } mtp_accept;
 
 /* Model and capacity.  The model is a decoder-only transformer over one
  * concatenated sequence [phonemes ; acoustic prompt ; generated codes]
@@ -143,7 +151,9 @@ MTP_API int mtp_decode_step(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_t
                             int32_t* out_accepted, int32_t* out_done);
 
 /* Run decode steps until every active slot has finished, with no host
- * synchronisation between steps.  out_tokens (host or device, may be NULL)
+ * synchronisation between steps (ACCEPT_ALL: one round of ceil(budget / n)
+ * steps; VERIFY_GREEDY, which emits 1..n tokens a step: rounds of
+ * ceil(remaining / n) steps with one state read between rounds).  out_tokens (host or device, may be NULL)
  * receives each slot's generated tokens in row b at stride `out_stride`
  * (>= the slot's max_new_tokens); out_lens (may be NULL) their counts.
  * Returns the number of steps run (>= 0) or an error. */

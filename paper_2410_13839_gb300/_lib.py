@@ -19,6 +19,8 @@ MTP_ERR_WEIGHTS = -4
 MTP_ERR_DEVICE = -5
 MTP_F32 = 0
 MTP_BF16 = 1
+MTP_ACCEPT_ALL = 0
+MTP_VERIFY_GREEDY = 1
 MTP_OPT_GRAPHS = 0
 MTP_OPT_PDL = 1
 MTP_OPT_L2_PREFETCH = 2

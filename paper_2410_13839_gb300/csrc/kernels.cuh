@@ -157,8 +157,25 @@ struct SelectArgs {
     int* out_tokens; int* out_accepted;   // [B][n_max], [B]
     int* err;
     unsigned long long* trace;
+    int policy;               // mtp_accept
+    const int* kept;          // [B] VERIFY_GREEDY: drafts kept this step (verify_kernel)
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
+
+// VERIFY_GREEDY, per slot of one pass: head 1's top-1 at every fed row
+// (logits1 [rows][V], row = slot-in-pass * n + j), the drafts kept (pending
+// token j + 1 equal to the top-1 at row j), and the hidden row of the last
+// kept position copied to h_last.
+struct VerifyArgs {
+    const float* logits1;     // head 1 logits of the pass's fed rows
+    const float* x;           // the pass's final hidden rows [rows][d]
+    float* h_last;            // [slots][d]
+    int* kept;                // [slots]
+    const int* active; const int* done; const int* n_pending; const int* pending;
+    int n, V, d, n_max, seq_base;
+    unsigned long long* trace;
+};
+cudaError_t launch_verify(const VerifyArgs& a, int slots, cudaStream_t s, bool pdl);
 
 struct ViterbiArgs {
     int batch, n, k, vocab, eos_id;

@@ -136,6 +136,7 @@ struct mtp_ctx {
     int *d_row_seq = nullptr, *d_row_pos = nullptr, *d_row_last = nullptr, *d_cand_ids = nullptr, *d_path = nullptr,
         *d_out_tokens = nullptr, *d_out_accepted = nullptr;
     int* d_err = nullptr;
+    int* d_kept = nullptr;  // VERIFY_GREEDY: drafts kept this step, per slot
     std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;  // (n_heads, top_k, traced)
     std::map<std::tuple<int, int, int>, std::vector<int>> graph_kinds;
     int last_n = 0, last_k = 0;
@@ -462,23 +463,49 @@ SelectArgs select_base(mtp_ctx* c, int n, int k) {
     a.gen_tokens = c->d_gen_tokens; a.gen_stride = c->cfg.max_ctx;
     a.out_tokens = c->d_out_tokens; a.out_accepted = c->d_out_accepted;
     a.err = c->d_err;
+    a.policy = c->cfg.accept_policy; a.kept = c->d_kept;
     return a;
+}
+
+// VERIFY_GREEDY: head 1 at every fed row of one pass (x: the pass's final rows,
+// rows = slots * n, written to d_logits row by row), then the kept drafts and
+// the last kept row's hidden state of each slot.
+int enqueue_verify(mtp_ctx* c, const float* x, int slots, int n, int b0, cudaStream_t s, bool pdl, Prof* prof) {
+    const int d = c->cfg.d_model, V = c->cfg.codec_vocab, rows = slots * n;
+    for (int r0 = 0; r0 < rows; r0 += MAX_ROWS) {
+        const int m = std::min(MAX_ROWS, rows - r0);
+        MTP_TRY(launch_heads(c, x + (size_t)r0 * d, m, 1, c->d_logits + (size_t)r0 * V, nullptr, 0, s, pdl, prof));
+    }
+    VerifyArgs va;
+    std::memset(&va, 0, sizeof(va));
+    va.logits1 = c->d_logits; va.x = x; va.h_last = c->d_h_last; va.kept = c->d_kept;
+    va.active = c->d_active; va.done = c->d_done; va.n_pending = c->d_npend; va.pending = c->d_pending;
+    va.n = n; va.V = V; va.d = d; va.n_max = c->cfg.n_heads_max; va.seq_base = b0;
+    va.trace = tslot(c, MTP_K_SELECT);
+    LAUNCH(MTP_K_SELECT, launch_verify(va, slots, s, pdl));
+    return MTP_OK;
 }
 
 int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof) {
     const int B = c->cfg.max_batch, d = c->cfg.d_model, V = c->cfg.codec_vocab;
     const int spc = std::max(1, MAX_ROWS / n);
-    const bool single = B <= spc;  // one pass feeds every slot: the heads read its rows directly
+    const bool verify = c->cfg.accept_policy == MTP_VERIFY_GREEDY;
+    // one pass feeds every slot: the heads read its rows directly (VERIFY_GREEDY: the kept row, via h_last)
+    const bool single = B <= spc && !verify;
     float* final_x = nullptr;
-    if (!single && c->use_batched && c->batched_ok && B * n <= c->bm_max) {  // every slot's rows in one pass
+    if (B > spc && c->use_batched && c->batched_ok && B * n <= c->bm_max) {  // every slot's rows in one pass
         const int M = B * n;
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
         e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
         MTP_TRY(run_layers_batched(c, M, n, B, PLAN_DEVICE, s, pdl, prof));
-        unsigned long long* tr = tslot(c, MTP_K_SAVE);
-        LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
+        if (verify) {
+            MTP_TRY(enqueue_verify(c, c->d_bx, B, n, 0, s, pdl, prof));
+        } else {
+            unsigned long long* tr = tslot(c, MTP_K_SAVE);
+            LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
+        }
         for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
             const int m = std::min(MAX_ROWS, B - b0);
             MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, nullptr,
@@ -496,7 +523,9 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));  // full dependency on the previous pass
         MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
-        if (!single) {
+        if (verify) {
+            MTP_TRY(enqueue_verify(c, final_x, G, n, b0, s, pdl, prof));
+        } else if (!single) {
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
             LAUNCH(MTP_K_SAVE,
                    launch_save_last(final_x, c->d_row_seq, c->d_row_last, c->d_h_last, d, MAX_ROWS, tr, s, pdl));
@@ -600,7 +629,8 @@ int validate_config(const mtp_config& c) {
     if (c.n_pages < 0) return fail(MTP_ERR_INVALID, "n_pages %d", c.n_pages);
     if (c.weight_dtype != MTP_F32 && c.weight_dtype != MTP_BF16)
         return fail(MTP_ERR_INVALID, "weight_dtype %d", c.weight_dtype);
-    if (c.accept_policy != MTP_ACCEPT_ALL) return fail(MTP_ERR_INVALID, "accept_policy %d", c.accept_policy);
+    if (c.accept_policy != MTP_ACCEPT_ALL && c.accept_policy != MTP_VERIFY_GREEDY)
+        return fail(MTP_ERR_INVALID, "accept_policy %d", c.accept_policy);
     if (!(c.ln_eps > 0.f)) return fail(MTP_ERR_INVALID, "ln_eps must be > 0");
     return MTP_OK;
 }
@@ -847,7 +877,7 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_cand_ids, (size_t)lb * nm * MAX_TOPK)) || (r = c->alloc(&c->d_path, (size_t)lb * nm)) ||
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
         (r = c->alloc(&c->d_row_seq, row_cap)) || (r = c->alloc(&c->d_row_pos, row_cap)) ||
-        (r = c->alloc(&c->d_row_last, row_cap)) || (r = c->alloc(&c->d_err, 1)) ||
+        (r = c->alloc(&c->d_row_last, row_cap)) || (r = c->alloc(&c->d_err, 1)) || (r = c->alloc(&c->d_kept, B)) ||
         (r = setup_batched(c)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
@@ -1036,15 +1066,23 @@ MTP_API int mtp_generate(mtp_ctx* c, int n, int k, int32_t* out_tokens, int out_
     MTP_TRY(check_ctx(c));
     MTP_TRY(check_nk(c, n, k));
     if (out_tokens && out_stride < 1) return fail(MTP_ERR_INVALID, "out_stride %d", out_stride);
+    // Rounds of steps without host synchronisation: a step emits at most n tokens,
+    // so ceil(remaining / n) more steps are needed at least; ACCEPT_ALL (n tokens per
+    // step until EOS or the budget) finishes in one round, VERIFY_GREEDY (1..n) in a few.
     std::vector<int> rem, done, active;
-    MTP_TRY(read_slot_ints(c, c->d_remaining, rem));
-    MTP_TRY(read_slot_ints(c, c->d_done, done));
-    MTP_TRY(read_slot_ints(c, c->d_active, active));
     int steps = 0;
-    for (int b = 0; b < c->cfg.max_batch; ++b)
-        if (active[b] && !done[b]) steps = std::max(steps, (rem[b] + n - 1) / n);
-    for (int i = 0; i < steps; ++i) MTP_TRY(run_step(c, n, k));
-    MTP_TRY(check_device_error(c));
+    for (;;) {
+        MTP_TRY(read_slot_ints(c, c->d_remaining, rem));
+        MTP_TRY(read_slot_ints(c, c->d_done, done));
+        MTP_TRY(read_slot_ints(c, c->d_active, active));
+        int round = 0;
+        for (int b = 0; b < c->cfg.max_batch; ++b)
+            if (active[b] && !done[b]) round = std::max(round, (rem[b] + n - 1) / n);
+        if (round == 0) break;
+        for (int i = 0; i < round; ++i) MTP_TRY(run_step(c, n, k));
+        steps += round;
+        MTP_TRY(check_device_error(c));
+    }
     const int B = c->cfg.max_batch, gs = c->cfg.max_ctx;
     if (out_tokens) {
         const int w = std::min(out_stride, gs);

@@ -14,6 +14,11 @@
 // Acceptance (ACCEPT_ALL): the path is cut after its first EOS and at the
 // remaining budget; the slot's state (cached length, fed tokens, output
 // buffer, done flag) is updated on the device, so steps need no host sync.
+// VERIFY_GREEDY: verify_kernel finds the drafts kept (head 1's top-1 at each
+// fed row against the next fed token); select_kernel forces position 1 of
+// the lattice to its top-1 candidate, emits the kept drafts and path[0],
+// advances the cached length by the kept rows only (the rest is rolled
+// back) and feeds the path next step.
 #include <math.h>
 
 #include "common.cuh"
@@ -179,6 +184,8 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         head_topk_warp(a.logits + row * a.V, a.V, k, s_ids + warp * k, s_lp + warp * k, a.lse + row);
     }
     __syncthreads();
+    if (do_accept && a.policy == 1 && threadIdx.x > 0 && threadIdx.x < k) s_lp[threadIdx.x] = -INFINITY;  // force
+    __syncthreads();
     for (int i = threadIdx.x; i < n * k; i += blockDim.x) {
         a.cand_ids[(size_t)bl * n * k + i] = s_ids[i];
         a.cand_logp[(size_t)bl * n * k + i] = s_lp[i];
@@ -192,24 +199,66 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
 
     int acc, done;
     const int rem = a.remaining[b];
-    accept_all(s_path, n, a.eos_id, rem, acc, done);
-    a.seq_len[b] += a.n_pending[b];  // the tokens fed this step are now cached
     const int gc = a.gen_count[b];
+    int emit[MAX_NHEADS];  // tokens this step emits (before the EOS / budget cut)
+    int n_emit;
+    if (a.policy == 1) {  // kept drafts, then head 1's argmax at the last kept row
+        const int fed = a.n_pending[b];
+        const int kept = fed > 0 ? a.kept[b] : 0;
+        for (int t = 0; t < kept; ++t) emit[t] = a.pending[(size_t)b * a.n_max + 1 + t];
+        emit[kept] = s_path[0];
+        n_emit = kept + 1;
+        a.seq_len[b] += fed > 0 ? kept + 1 : 0;  // the confirmed token and the kept drafts stay cached
+    } else {
+        for (int t = 0; t < n; ++t) emit[t] = s_path[t];
+        n_emit = n;
+        a.seq_len[b] += a.n_pending[b];  // the tokens fed this step are now cached
+    }
+    accept_all(emit, n_emit, a.eos_id, rem, acc, done);
     if (gc + acc > a.gen_stride) {
         atomicOr(a.err, ERR_BOUNDS);
         acc = max(0, a.gen_stride - gc);
     }
-    for (int t = 0; t < a.n_max; ++t) a.out_tokens[(size_t)b * a.n_max + t] = t < acc ? s_path[t] : -1;
+    for (int t = 0; t < a.n_max; ++t) a.out_tokens[(size_t)b * a.n_max + t] = t < acc ? emit[t] : -1;
     for (int t = 0; t < n; ++t) a.path[(size_t)b * n + t] = s_path[t];
-    for (int t = 0; t < acc; ++t) {
-        a.pending[(size_t)b * a.n_max + t] = s_path[t];
-        a.gen_tokens[(size_t)b * a.gen_stride + gc + t] = s_path[t];
-    }
+    for (int t = 0; t < acc; ++t) a.gen_tokens[(size_t)b * a.gen_stride + gc + t] = emit[t];
+    const int n_next = a.policy == 1 ? n : acc;  // VERIFY_GREEDY feeds the path: confirmed token + drafts
+    for (int t = 0; t < n_next; ++t) a.pending[(size_t)b * a.n_max + t] = s_path[t];
     a.gen_count[b] = gc + acc;
     a.remaining[b] = rem - acc;
-    a.n_pending[b] = done ? 0 : acc;
+    a.n_pending[b] = done ? 0 : n_next;
     a.done[b] = done;
     a.out_accepted[b] = acc;
+}
+
+__global__ void __launch_bounds__(256) verify_kernel(const VerifyArgs a) {
+    __shared__ int s_g[MAX_NHEADS];
+    __shared__ float s_lp[MAX_NHEADS], s_lse[MAX_NHEADS];
+    __shared__ int s_kept;
+    const int bl = blockIdx.x, b = a.seq_base + bl;
+    const int warp = threadIdx.x >> 5;
+    TraceEnd trace_guard(a.trace);
+    pdl_launch_dependents();
+    pdl_wait();
+    trace_wait(a.trace);
+    if (!a.active[b] || a.done[b]) return;
+    const int fed = a.n_pending[b];
+    if (fed == 0) {  // first step after the prompt: h_last is the prompt's last row
+        if (threadIdx.x == 0) a.kept[b] = 0;
+        return;
+    }
+    if (warp < fed) head_topk_warp(a.logits1 + ((size_t)bl * a.n + warp) * a.V, a.V, 1, s_g + warp, s_lp + warp,
+                                   s_lse + warp);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int kept = 0;
+        while (kept < fed - 1 && a.pending[(size_t)b * a.n_max + kept + 1] == s_g[kept]) ++kept;
+        s_kept = kept;
+        a.kept[b] = kept;
+    }
+    __syncthreads();
+    const float* src = a.x + ((size_t)bl * a.n + s_kept) * a.d;
+    for (int i = threadIdx.x; i < a.d; i += blockDim.x) a.h_last[(size_t)b * a.d + i] = src[i];
 }
 
 // Stand-alone Viterbi: one warp per lattice, VIT_WARPS lattices per block;
@@ -261,6 +310,20 @@ cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaSt
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, select_kernel, a, do_accept ? 1 : 0);
+}
+
+cudaError_t launch_verify(const VerifyArgs& a, int slots, cudaStream_t s, bool pdl) {
+    if (a.n < 1 || a.n > MAX_NHEADS || a.V > MAX_VOCAB || slots < 1) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(slots);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, verify_kernel, a);
 }
 
 cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s) {

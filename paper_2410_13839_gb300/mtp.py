@@ -42,14 +42,15 @@ def _stream_handle(stream) -> int | None:
     return stream.cuda_stream
 
 
-def make_config(model, max_batch: int, max_ctx: int, page_size: int = 64, n_pages: int = 0) -> MtpConfig:
+def make_config(model, max_batch: int, max_ctx: int, page_size: int = 64, n_pages: int = 0,
+                accept_policy: int = 0) -> MtpConfig:
     """mtp_config of a synth.ModelConfig-like object plus capacity."""
     return MtpConfig(layers=model.layers, d_model=model.d_model, n_attn_heads=model.n_attn_heads,
                      d_ffn=model.d_ffn, phone_vocab=model.phone_vocab, codec_vocab=model.codec_vocab,
                      eos_id=model.eos_id, n_heads_max=model.n_heads_max, top_k_max=model.top_k_max,
                      max_batch=max_batch, max_ctx=max_ctx, page_size=page_size, n_pages=n_pages,
                      weight_dtype=_lib.MTP_BF16 if model.weight_dtype == "bf16" else _lib.MTP_F32,
-                     accept_policy=0, ln_eps=model.ln_eps)
+                     accept_policy=accept_policy, ln_eps=model.ln_eps)
 
 
 def pack_weights(tensors: list[tuple[np.ndarray, bool]], bf16: bool) -> bytes:
@@ -228,9 +229,10 @@ class MTPDecoder:
     """Owns one mtp_ctx: weights on the device, KV pages, slot state."""
 
     def __init__(self, model, weights: dict[str, np.ndarray], names: list[str], is_matrix,
-                 max_batch: int, max_ctx: int, page_size: int = 64, n_pages: int = 0, stream=None):
+                 max_batch: int, max_ctx: int, page_size: int = 64, n_pages: int = 0, stream=None,
+                 accept_policy: int = 0):
         self.model = model
-        self.config = make_config(model, max_batch, max_ctx, page_size, n_pages)
+        self.config = make_config(model, max_batch, max_ctx, page_size, n_pages, accept_policy)
         blob = pack_weights([(weights[n], is_matrix(n)) for n in names], model.weight_dtype == "bf16")
         self.ctx = mtp_create(self.config, blob, stream)
 

@@ -23,11 +23,12 @@ def lib_module():
     return mtp
 
 
-def decoder(model, max_batch=1, max_ctx=512, page_size=64, n_pages=0, eos_bias=synth.EOS_BIAS, seed=0):
+def decoder(model, max_batch=1, max_ctx=512, page_size=64, n_pages=0, eos_bias=synth.EOS_BIAS, seed=0,
+            accept_policy=0):
     mtp = lib_module()
     w = synth.make_weights(model, seed=seed, eos_bias=eos_bias)
     dec = mtp.MTPDecoder(model, w, synth.weight_names(model), synth.is_matrix, max_batch, max_ctx,
-                         page_size=page_size, n_pages=n_pages)
+                         page_size=page_size, n_pages=n_pages, accept_policy=accept_policy)
     return dec, w
 
 
