@@ -194,6 +194,41 @@ def run_b32(mtp, stream, warmup, steps):
                                 "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak}}
 
 
+SWEEP_GEN = 1500
+
+
+def run_sweep(mtp, stream):
+    """Head/beam sweep on the VALL-E-sized model (B=1, prompt 64+225, 1500 tokens): tokens/s
+    (prefill + decode) and mean accepted tokens per step for each (n, top_k); and the mean
+    accepted tokens per step of VERIFY_GREEDY at n=4, top_k=4 (random-init heads)."""
+    import torch
+    w = synth.make_weights(MODEL)
+    ph, ac = synth.make_prompt(0, N_PH, N_AC, MODEL.phone_vocab)
+    max_ctx = N_PH + N_AC + SWEEP_GEN + MODEL.n_heads_max + 8
+    rows = []
+    for policy in (0, 1):
+        dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, 1, max_ctx, stream=stream,
+                             accept_policy=policy)
+        ctx = dec.ctx
+        ph_d, ac_d = torch.from_numpy(ph).cuda(), torch.from_numpy(ac).cuda()
+        lens = torch.zeros(1, dtype=torch.int32, device="cuda")
+        grid = [(n, k) for n in (1, 2, 4, 8) for k in (1, 4, 8)] if policy == 0 else [(4, 4)]
+        for n, k in grid:
+            for rep in range(2):  # the first run captures the step graph
+                ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+                ev[0].record(stream)
+                mtp.mtp_prefill(ctx, 0, ph_d, ac_d, SWEEP_GEN)
+                steps = mtp.mtp_generate(ctx, n, k, None, 0, lens)
+                ev[1].record(stream)
+                torch.cuda.synchronize()
+            toks = int(lens[0].item())
+            rows.append({"policy": "VERIFY_GREEDY" if policy else "ACCEPT_ALL", "n": n, "top_k": k,
+                         "tokens": toks, "steps": steps, "mean_accepted": toks / max(1, steps),
+                         "tokens_per_s": toks / (ev[0].elapsed_time(ev[1]) / 1e3)})
+        dec.close()
+    return rows
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples while the timed region runs."""
 
@@ -425,6 +460,8 @@ def run_ours(args):
     dec.close()
     if not args.no_b32:
         line["b32"] = run_b32(mtp, stream, max(1, min(args.warmup, 2)), max(1, min(args.steps, 3)))
+    if not args.no_sweep:
+        line["sweep"] = run_sweep(mtp, stream)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:
@@ -439,6 +476,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b32", action="store_true", help="skip the batch-32 serving measurement")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the head/beam sweep")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
