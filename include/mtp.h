@@ -193,10 +193,13 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        pass (8 rows) run the batched path: tensor-core projections over all
  *                        rows at once (bf16 weights only; default); 0 = fused passes of 8 rows
  *   MTP_OPT_GEMM_SPLITS  most K splits of a batched-path projection (power of two 1..64; each
- *                        split adds its partial tile with fp32 atomics; default 16) */
+ *                        split adds its partial tile with fp32 atomics; default 16)
+ *   MTP_OPT_LATTICE      states of the Viterbi search (Sec. III-C): 0 = each position's own head
+ *                        top-k (default); 1 = the union of all heads' top-k at every position,
+ *                        each scored by that position's head (the paper's reduced m x m matrix) */
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
-    MTP_OPT_GEMM_SPLITS = 5
+    MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);

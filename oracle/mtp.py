@@ -38,7 +38,7 @@ import numpy as np
 
 from .model import ARDecoder
 from .select import (accept_all, head_logits, log_softmax, top_k_rows, topk_gap,
-                     viterbi, viterbi_margin)
+                     viterbi, viterbi_margin, viterbi_union)
 
 
 @dataclasses.dataclass
@@ -99,22 +99,29 @@ class MTPOracle:
             h = self.model.forward(tokens, np.zeros(tokens.shape[0], bool), self.cache)
             self.h_last = h[-1]
 
-    def select(self, n: int, k: int):
-        """Heads, log-softmax, top-k and Viterbi on the current h_last."""
+    def select(self, n: int, k: int, lattice: str = "A"):
+        """Heads, log-softmax, top-k and Viterbi on the current h_last.
+
+        lattice "A": each position's states are its own head's top-k; "B": the
+        union of all heads' top-k at every position (select.viterbi_union)."""
         logits = head_logits(self.h_last, self.w, n, self.cfg.ln_eps)
         logp, lse = log_softmax(logits)
         logp32 = logp.astype(np.float32)
         ids, vals = top_k_rows(logp32, k)
+        if lattice == "B":
+            path, _ = viterbi_union(ids, logp32, self.log_q)
+            margin = float(topk_gap(logp32, k).min())
+            return logits, lse, logp32, ids, vals, path, margin
         path, _, _ = viterbi(ids[None], vals[None], self.log_q)
         margin = min(float(topk_gap(logp32, k).min()),
                      float(viterbi_margin(ids[None], vals[None], self.log_q)[0]))
         return logits, lse, logp32, ids, vals, path[0], margin
 
-    def step(self, n: int, k: int, teacher=None) -> StepRecord:
+    def step(self, n: int, k: int, teacher=None, lattice: str = "A") -> StepRecord:
         """One decode step; `teacher` overrides the fed tokens (teacher forcing)."""
         fed = self.pending if teacher is None else np.asarray(teacher, dtype=np.int32)
         self.feed(fed)
-        logits, lse, logp32, ids, vals, path, margin = self.select(n, k)
+        logits, lse, logp32, ids, vals, path, margin = self.select(n, k, lattice)
         a, done = accept_all(path, self.cfg.eos_id, self.remaining)
         self.pending = path[:a].astype(np.int32)
         self.generated.extend(int(t) for t in self.pending)

@@ -27,6 +27,7 @@ MTP_OPT_L2_PREFETCH = 2
 MTP_OPT_MLP_CLUSTERS = 3
 MTP_OPT_BATCHED = 4
 MTP_OPT_GEMM_SPLITS = 5
+MTP_OPT_LATTICE = 6
 KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save", "pack", "gemm", "qkv", "attn")
 
 

@@ -159,6 +159,7 @@ struct SelectArgs {
     unsigned long long* trace;
     int policy;               // mtp_accept
     const int* kept;          // [B] VERIFY_GREEDY: drafts kept this step (verify_kernel)
+    int lattice;              // 0: per-head top-k states (reading A); 1: union of all heads' top-k (reading B)
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
 

@@ -112,6 +112,7 @@ struct mtp_ctx {
     int* d_bwc = nullptr;    // attention split counters
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
     int gemm_max_splits = 16;
+    int lattice = 0;  // MTP_OPT_LATTICE
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -463,7 +464,7 @@ SelectArgs select_base(mtp_ctx* c, int n, int k) {
     a.gen_tokens = c->d_gen_tokens; a.gen_stride = c->cfg.max_ctx;
     a.out_tokens = c->d_out_tokens; a.out_accepted = c->d_out_accepted;
     a.err = c->d_err;
-    a.policy = c->cfg.accept_policy; a.kept = c->d_kept;
+    a.policy = c->cfg.accept_policy; a.kept = c->d_kept; a.lattice = c->lattice;
     return a;
 }
 
@@ -916,6 +917,10 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
             return fail(MTP_ERR_INVALID, "GEMM splits %d: need a power of two in 1..64", value);
         changed = c->gemm_max_splits != value;
         c->gemm_max_splits = value;
+    } else if (option == MTP_OPT_LATTICE) {
+        if (value != 0 && value != 1) return fail(MTP_ERR_INVALID, "lattice %d: need 0 or 1", value);
+        changed = c->lattice != value;
+        c->lattice = value;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -953,6 +958,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_MLP_CLUSTERS: *value = c->mlp_clusters; break;
         case MTP_OPT_BATCHED: *value = c->use_batched && c->batched_ok; break;
         case MTP_OPT_GEMM_SPLITS: *value = c->gemm_max_splits; break;
+        case MTP_OPT_LATTICE: *value = c->lattice; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;

@@ -14,6 +14,11 @@
 // Acceptance (ACCEPT_ALL): the path is cut after its first EOS and at the
 // remaining budget; the slot's state (cached length, fed tokens, output
 // buffer, done flag) is updated on the device, so steps need no host sync.
+// Union lattice (reading B, option): the states of every position are the
+// m <= n*k distinct tokens of all heads' top-k (sorted by id), each scored by
+// head t's full fp32 log-softmax; the same recursion, add order and lowest-index
+// tie-breaks, one thread per state, transitions read from the L2-resident
+// log Q.
 // VERIFY_GREEDY: verify_kernel finds the drafts kept (head 1's top-1 at each
 // fed row against the next fed token); select_kernel forces position 1 of
 // the lattice to its top-1 candidate, emits the kept drafts and path[0],
@@ -161,6 +166,79 @@ __device__ __forceinline__ void accept_all(const int* path, int n, int eos, int 
     done = (eos_in && a >= 1 && path[a - 1] == eos) || remaining - a <= 0;
 }
 
+// Reading B over one sequence's lattice; `scratch` >= 20 KB of shared memory.
+// VERIFY_GREEDY forces position 1 to head 1's top-1 (other states -inf).
+__device__ void union_viterbi(const SelectArgs& a, int bl, int n, int k, const int* s_ids, unsigned char* scratch,
+                              int* s_path) {
+    constexpr int MS = MAX_NHEADS * MAX_TOPK;  // most states
+    int* states = reinterpret_cast<int*>(scratch);            // [MS]
+    int* first = states + MS;                                 // [MS]
+    float* em = reinterpret_cast<float*>(first + MS);         // [MAX_NHEADS][MS]
+    float* delta = em + MAX_NHEADS * MS;                      // [2][MS]
+    int* psi = reinterpret_cast<int*>(delta + 2 * MS);        // [MAX_NHEADS][MS]
+    __shared__ int s_m;
+    const int tid = threadIdx.x, N = n * k;
+    for (int t = tid; t < N; t += blockDim.x) {  // first occurrence of each id
+        int f = 1;
+        for (int j = 0; j < t; ++j)
+            if (s_ids[j] == s_ids[t]) f = 0;
+        first[t] = f;
+    }
+    __syncthreads();
+    for (int t = tid; t < N; t += blockDim.x)
+        if (first[t]) {  // rank among the distinct ids = its state index (ids ascending)
+            int r = 0;
+            for (int j = 0; j < N; ++j) r += first[j] && s_ids[j] < s_ids[t];
+            states[r] = s_ids[t];
+        }
+    if (tid == 0) {
+        int m = 0;
+        for (int j = 0; j < N; ++j) m += first[j];
+        s_m = m;
+    }
+    __syncthreads();
+    const int m = s_m;
+    for (int i = tid; i < n * m; i += blockDim.x) {  // emissions: logp of every state under every head
+        const int t = i / m, r = i % m;
+        const size_t row = (size_t)bl * n + t;
+        float v = __fsub_rn(a.logits[row * a.V + states[r]], a.lse[row]);
+        if (t == 0 && a.policy == 1 && states[r] != s_ids[0]) v = -INFINITY;  // VERIFY_GREEDY: forced
+        em[t * MS + r] = v;
+    }
+    __syncthreads();
+    for (int r = tid; r < m; r += blockDim.x) delta[r] = em[r];
+    __syncthreads();
+    for (int t = 1; t < n; ++t) {
+        const float* prev = delta + ((t - 1) & 1) * MS;
+        float* cur = delta + (t & 1) * MS;
+        for (int r = tid; r < m; r += blockDim.x) {
+            const float* lq_col = a.log_q + states[r];
+            float best = -INFINITY;
+            int arg = 0;
+            for (int i = 0; i < m; ++i) {
+                const float v = __fadd_rn(prev[i], lq_col[(size_t)states[i] * a.V]);
+                if (v > best) {
+                    best = v;
+                    arg = i;
+                }
+            }
+            cur[r] = __fadd_rn(best, em[t * MS + r]);
+            psi[t * MS + r] = arg;
+        }
+        __syncthreads();
+    }
+    if (tid == 0) {
+        const float* last = delta + ((n - 1) & 1) * MS;
+        int r = 0;
+        for (int i = 1; i < m; ++i)
+            if (last[i] > last[r]) r = i;
+        for (int t = n - 1; t >= 0; --t) {
+            s_path[t] = states[r];
+            if (t > 0) r = psi[t * MS + r];
+        }
+    }
+}
+
 __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_accept) {
     __shared__ int s_ids[MAX_NHEADS * MAX_TOPK];
     __shared__ float s_lp[MAX_NHEADS * MAX_TOPK];
@@ -191,9 +269,13 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         a.cand_logp[(size_t)bl * n * k + i] = s_lp[i];
     }
     if (!do_accept) return;
-    gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
-    __syncthreads();
-    if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_path, &s_score);
+    if (a.lattice == 1) {
+        union_viterbi(a, bl, n, k, s_ids, reinterpret_cast<unsigned char*>(s_lq), s_path);
+    } else {
+        gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
+        __syncthreads();
+        if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_path, &s_score);
+    }
     __syncthreads();
     if (threadIdx.x != 0) return;
 
