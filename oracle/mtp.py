@@ -29,6 +29,13 @@ d_1..d_a and then g_a.  The next drafts are the Viterbi path over the heads
 at the last kept row with position 1 forced to g_a (its top-1 candidate), so
 c' = g_a and d'_t = path[t].  The emitted sequence is the greedy AR
 sequence for every n and k (pinned in tests/test_oracle_verify.py).
+
+Path sampling (sample = (seed, slot); the top-k sampling of the Fig. 2
+caption): step 3 draws the path from the lattice's posterior instead of
+taking its maximum (select.sample_path), with the uniforms of
+select.path_uniform(seed, slot, tokens generated so far, position).  Under
+VERIFY_GREEDY only the drafts are drawn (position 1 stays forced), so the
+emitted sequence is still the greedy one.
 """
 from __future__ import annotations
 
@@ -37,8 +44,8 @@ import dataclasses
 import numpy as np
 
 from .model import ARDecoder
-from .select import (accept_all, head_logits, log_softmax, top_k_rows, topk_gap,
-                     viterbi, viterbi_margin, viterbi_union)
+from .select import (accept_all, head_logits, log_softmax, path_uniform, sample_path, sample_path_union,
+                     top_k_rows, topk_gap, viterbi, viterbi_margin, viterbi_union)
 
 
 @dataclasses.dataclass
@@ -99,15 +106,31 @@ class MTPOracle:
             h = self.model.forward(tokens, np.zeros(tokens.shape[0], bool), self.cache)
             self.h_last = h[-1]
 
-    def select(self, n: int, k: int, lattice: str = "A"):
+    def uniforms(self, sample, n: int) -> list[float]:
+        """The n uniforms of this step's path draw: sample = (seed, slot), the
+        counter also holds the number of tokens generated so far."""
+        seed, slot = sample
+        return [path_uniform(seed, slot, len(self.generated), t) for t in range(n)]
+
+    def select(self, n: int, k: int, lattice: str = "A", sample=None):
         """Heads, log-softmax, top-k and Viterbi on the current h_last.
 
         lattice "A": each position's states are its own head's top-k; "B": the
-        union of all heads' top-k at every position (select.viterbi_union)."""
+        union of all heads' top-k at every position (select.viterbi_union).
+        sample = (seed, slot): draw the path from the lattice's posterior
+        (select.sample_path) instead of taking its maximum; margin is then the
+        smallest draw margin."""
         logits = head_logits(self.h_last, self.w, n, self.cfg.ln_eps)
         logp, lse = log_softmax(logits)
         logp32 = logp.astype(np.float32)
         ids, vals = top_k_rows(logp32, k)
+        if sample is not None:
+            u = self.uniforms(sample, n)
+            if lattice == "B":
+                path, margin = sample_path_union(ids, logp32, self.log_q, u)
+            else:
+                path, margin = sample_path(ids, vals, self.log_q, u)
+            return logits, lse, logp32, ids, vals, path, min(margin, float(topk_gap(logp32, k).min()))
         if lattice == "B":
             path, _ = viterbi_union(ids, logp32, self.log_q)
             margin = float(topk_gap(logp32, k).min())
@@ -117,11 +140,11 @@ class MTPOracle:
                      float(viterbi_margin(ids[None], vals[None], self.log_q)[0]))
         return logits, lse, logp32, ids, vals, path[0], margin
 
-    def step(self, n: int, k: int, teacher=None, lattice: str = "A") -> StepRecord:
+    def step(self, n: int, k: int, teacher=None, lattice: str = "A", sample=None) -> StepRecord:
         """One decode step; `teacher` overrides the fed tokens (teacher forcing)."""
         fed = self.pending if teacher is None else np.asarray(teacher, dtype=np.int32)
         self.feed(fed)
-        logits, lse, logp32, ids, vals, path, margin = self.select(n, k, lattice)
+        logits, lse, logp32, ids, vals, path, margin = self.select(n, k, lattice, sample)
         a, done = accept_all(path, self.cfg.eos_id, self.remaining)
         self.pending = path[:a].astype(np.int32)
         self.generated.extend(int(t) for t in self.pending)
@@ -131,18 +154,22 @@ class MTPOracle:
                           a, done, margin)
 
     # ---- VERIFY_GREEDY ----
-    def propose(self, n: int, k: int):
-        """Heads at h_last with position 1 forced to head 1's top-1 (the greedy token)."""
+    def propose(self, n: int, k: int, sample=None):
+        """Heads at h_last with position 1 forced to head 1's top-1 (the greedy token);
+        the drafts are the Viterbi path, or a drawn path with sample = (seed, slot)."""
         logits = head_logits(self.h_last, self.w, n, self.cfg.ln_eps)
         logp, lse = log_softmax(logits)
         logp32 = logp.astype(np.float32)
         ids, vals = top_k_rows(logp32, k)
         vals = vals.copy()
         vals[0, 1:] = -np.inf  # position 1: the greedy token only
+        if sample is not None:
+            path, self.last_margin = sample_path(ids, vals, self.log_q, self.uniforms(sample, n))
+            return logits, lse, logp32, ids, vals, path
         path, _, _ = viterbi(ids[None], vals[None], self.log_q)
         return logits, lse, logp32, ids, vals, path[0]
 
-    def step_verify(self, n: int, k: int) -> "VerifyRecord":
+    def step_verify(self, n: int, k: int, sample=None) -> "VerifyRecord":
         """One VERIFY_GREEDY step (see the module docstring)."""
         fed = self.pending
         m = max(0, len(fed) - 1)  # drafts fed
@@ -159,7 +186,7 @@ class MTPOracle:
             self.h_last = h[a]
         else:
             a = 0
-        logits, lse, logp32, ids, vals, path = self.propose(n, k)
+        logits, lse, logp32, ids, vals, path = self.propose(n, k, sample)
         emit = [int(t) for t in fed[1:a + 1]] + [int(path[0])]
         e, done = accept_all(np.asarray(emit, np.int32), self.cfg.eos_id, self.remaining)
         emitted = np.asarray(emit[:e], np.int32)

@@ -194,3 +194,83 @@ def accept_all(path: np.ndarray, eos_id: int, remaining: int) -> tuple[int, bool
     a = min(a, remaining)
     done = bool(hits.size and hits[0] < a) or remaining - a <= 0
     return a, done
+
+
+# ---- path sampling (top-k sampling over the lattice, the diversity option of Fig. 2) ----
+_M64 = (1 << 64) - 1
+
+
+def splitmix64(x: int) -> int:
+    """SplitMix64 output function (Steele, Lea, Flood 2014) of a 64-bit counter."""
+    z = (x + 0x9E3779B97F4A7C15) & _M64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _M64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _M64
+    return z ^ (z >> 31)
+
+
+def path_uniform(seed: int, slot: int, generated: int, t: int) -> float:
+    """The uniform in [0, 1) (24 bits) drawn for position t of a sampling step of
+    `slot` when it has generated `generated` tokens: SplitMix64 of the counter
+    ((seed * P + slot) * P + generated) * P + t, P = 0x100000001B3, top 24 bits."""
+    p = 0x100000001B3
+    x = (((((seed & _M64) * p + slot) & _M64) * p + generated) & _M64) * p + t
+    return (splitmix64(x & _M64) >> 40) * (1.0 / (1 << 24))
+
+
+def _categorical(logw: np.ndarray, u: float) -> tuple[int, float]:
+    """(index, margin) of one draw with probabilities proportional to exp(logw):
+    the first index whose cumulative weight (index order, float64) exceeds
+    u times the total, clamped to the last index of positive weight.  margin
+    is the distance of u * total from the nearest boundary that separates the
+    drawn index from another index of positive weight, over the total (1 when
+    only one index has positive weight)."""
+    m = logw.max()
+    w = np.where(np.isfinite(logw), np.exp(logw - m), 0.0)
+    c = np.cumsum(w)
+    total = c[-1]
+    target = u * total
+    pos = np.flatnonzero(w > 0)
+    i = int(np.searchsorted(c, target, side="right"))
+    i = min(i, int(pos[-1]))
+    margin = 1.0
+    if pos[0] < i:       # a positive-weight index below: the lower boundary counts
+        margin = min(margin, (target - (c[i - 1] if i > 0 else 0.0)) / total)
+    if pos[-1] > i:      # one above: the upper boundary counts
+        margin = min(margin, (c[i] - target) / total)
+    return i, max(margin, 0.0)
+
+
+def sample_path(cand_ids: np.ndarray, cand_logp: np.ndarray, log_q: np.ndarray, uniforms):
+    """(path [n], margin) of one lattice drawn from P(path) proportional to
+    prod_t Q(c_{t-1}, c_t) S_t(c_t) (the quantity Viterbi maximises), by forward
+    filtering (log-sum-exp, float64) and backward sampling: the last state with
+    uniforms[n-1], then each earlier state given its successor with uniforms[t].
+    margin: the smallest draw margin (see _categorical) along the way."""
+    ids = np.asarray(cand_ids)
+    s = np.asarray(cand_logp, dtype=np.float64)
+    lq = np.asarray(log_q, dtype=np.float64)
+    n, k = s.shape
+    alpha = np.zeros((n, k))
+    alpha[0] = s[0]
+    for t in range(1, n):
+        x = alpha[t - 1][:, None] + lq[ids[t - 1][:, None], ids[t][None, :]]   # [k_prev, k]
+        mx = x.max(axis=0)
+        safe = np.where(np.isfinite(mx), mx, 0.0)
+        with np.errstate(divide="ignore"):
+            lse = np.where(np.isfinite(mx), safe + np.log(np.exp(x - safe).sum(axis=0)), -np.inf)
+        alpha[t] = lse + s[t]
+    state = np.zeros(n, dtype=np.int64)
+    state[n - 1], margin = _categorical(alpha[n - 1], uniforms[n - 1])
+    for t in range(n - 2, -1, -1):
+        state[t], mg = _categorical(alpha[t] + lq[ids[t], ids[t + 1][state[t + 1]]], uniforms[t])
+        margin = min(margin, mg)
+    return ids[np.arange(n), state].astype(np.int32), float(margin)
+
+
+def sample_path_union(cand_ids: np.ndarray, logp32: np.ndarray, log_q: np.ndarray, uniforms):
+    """sample_path over the union lattice (reading B): the states of every
+    position are the distinct ids of all heads' top-k, ascending, each scored
+    at position t by head t's float32 log-softmax."""
+    states = np.unique(np.asarray(cand_ids).reshape(-1))
+    n = logp32.shape[0]
+    return sample_path(np.tile(states, (n, 1)), np.asarray(logp32)[:, states], log_q, uniforms)

@@ -80,3 +80,16 @@ def test_verify_with_a_perfect_drafter_keeps_every_draft(tiny):
     r = o.step_verify(4, 4)
     assert r.kept == 3 and r.rollback == 0
     assert list(r.emitted) == ref[1:5]
+
+
+@pytest.mark.parametrize("n,k", [(4, 4), (6, 3)])
+def test_verify_with_sampled_drafts_is_still_greedy(tiny, n, k):
+    """Drawn drafts (path sampling) change which drafts are kept, never the output."""
+    w, ph, ac = tiny
+    budget = 40
+    ref = _greedy(synth.TINY, w, ph, ac, budget)
+    o = MTPOracle(synth.TINY, w)
+    o.prefill(ph, ac, budget)
+    while not o.done:
+        o.step_verify(n, k, sample=(12345, 0))
+    assert o.generated == ref
