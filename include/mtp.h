@@ -196,10 +196,20 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        split adds its partial tile with fp32 atomics; default 16)
  *   MTP_OPT_LATTICE      states of the Viterbi search (Sec. III-C): 0 = each position's own head
  *                        top-k (default); 1 = the union of all heads' top-k at every position,
- *                        each scored by that position's head (the paper's reduced m x m matrix) */
+ *                        each scored by that position's head (the paper's reduced m x m matrix)
+ *   MTP_OPT_SAMPLING     0 = select the lattice's best path (Viterbi, default); 1 = draw one path
+ *                        from the lattice's posterior P(path) ~ prod_t Q(c_{t-1}, c_t) S_t(c_t)
+ *                        (the top-k sampling that keeps diversity, Fig. 2 caption), by forward
+ *                        filtering and backward sampling in fp32.  Under MTP_VERIFY_GREEDY only
+ *                        the drafts are drawn; the output stays greedy.
+ *   MTP_OPT_SEED         seed of the path draws (any 32-bit value, zero-extended; default 0).
+ *                        Position t of a draw of slot b that has generated g tokens uses the
+ *                        uniform (SplitMix64(x) >> 40) / 2^24, x = ((seed * P + b) * P + g) * P + t
+ *                        mod 2^64, P = 0x100000001B3, so runs are reproducible.  Changing either
+ *                        option recaptures the step graphs. */
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
-    MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6
+    MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);

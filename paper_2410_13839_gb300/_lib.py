@@ -28,6 +28,8 @@ MTP_OPT_MLP_CLUSTERS = 3
 MTP_OPT_BATCHED = 4
 MTP_OPT_GEMM_SPLITS = 5
 MTP_OPT_LATTICE = 6
+MTP_OPT_SAMPLING = 7
+MTP_OPT_SEED = 8
 KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save", "pack", "gemm", "qkv", "attn")
 
 

@@ -160,6 +160,8 @@ struct SelectArgs {
     int policy;               // mtp_accept
     const int* kept;          // [B] VERIFY_GREEDY: drafts kept this step (verify_kernel)
     int lattice;              // 0: per-head top-k states (reading A); 1: union of all heads' top-k (reading B)
+    int sampling;             // 0: the lattice's best path (Viterbi); 1: a path drawn from its posterior
+    unsigned long long seed;  // path draws: counter-based uniforms of (seed, slot, tokens generated, position)
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
 

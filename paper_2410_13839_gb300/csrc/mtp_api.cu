@@ -113,6 +113,8 @@ struct mtp_ctx {
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
     int gemm_max_splits = 16;
     int lattice = 0;  // MTP_OPT_LATTICE
+    int sampling = 0;          // MTP_OPT_SAMPLING
+    uint32_t sample_seed = 0;  // MTP_OPT_SEED
     __nv_bfloat16 *d_ahi = nullptr, *d_alo = nullptr, *d_uhi = nullptr, *d_ulo = nullptr;
     struct LayerMaps {
         CUtensorMap wqkv, wo, w1, w2;
@@ -465,6 +467,7 @@ SelectArgs select_base(mtp_ctx* c, int n, int k) {
     a.out_tokens = c->d_out_tokens; a.out_accepted = c->d_out_accepted;
     a.err = c->d_err;
     a.policy = c->cfg.accept_policy; a.kept = c->d_kept; a.lattice = c->lattice;
+    a.sampling = c->sampling; a.seed = c->sample_seed;
     return a;
 }
 
@@ -921,6 +924,13 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
         if (value != 0 && value != 1) return fail(MTP_ERR_INVALID, "lattice %d: need 0 or 1", value);
         changed = c->lattice != value;
         c->lattice = value;
+    } else if (option == MTP_OPT_SAMPLING) {
+        if (value != 0 && value != 1) return fail(MTP_ERR_INVALID, "sampling %d: need 0 or 1", value);
+        changed = c->sampling != value;
+        c->sampling = value;
+    } else if (option == MTP_OPT_SEED) {
+        changed = c->sample_seed != (uint32_t)value;
+        c->sample_seed = (uint32_t)value;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -959,6 +969,8 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_BATCHED: *value = c->use_batched && c->batched_ok; break;
         case MTP_OPT_GEMM_SPLITS: *value = c->gemm_max_splits; break;
         case MTP_OPT_LATTICE: *value = c->lattice; break;
+        case MTP_OPT_SAMPLING: *value = c->sampling; break;
+        case MTP_OPT_SEED: *value = (int32_t)c->sample_seed; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;

@@ -19,6 +19,9 @@
 // head t's full fp32 log-softmax; the same recursion, add order and lowest-index
 // tie-breaks, one thread per state, transitions read from the L2-resident
 // log Q.
+// Path sampling (option): instead of the best path, one path drawn from the
+// lattice's posterior (forward filtering, backward sampling) with SplitMix64
+// uniforms of (seed, slot, tokens generated, position); either lattice.
 // VERIFY_GREEDY: verify_kernel finds the drafts kept (head 1's top-1 at each
 // fed row against the next fed token); select_kernel forces position 1 of
 // the lattice to its top-1 candidate, emits the kept drafts and path[0],
@@ -166,16 +169,19 @@ __device__ __forceinline__ void accept_all(const int* path, int n, int eos, int 
     done = (eos_in && a >= 1 && path[a - 1] == eos) || remaining - a <= 0;
 }
 
-// Reading B over one sequence's lattice; `scratch` >= 20 KB of shared memory.
-// VERIFY_GREEDY forces position 1 to head 1's top-1 (other states -inf).
-__device__ void union_viterbi(const SelectArgs& a, int bl, int n, int k, const int* s_ids, unsigned char* scratch,
-                              int* s_path) {
-    constexpr int MS = MAX_NHEADS * MAX_TOPK;  // most states
+constexpr int MS = MAX_NHEADS * MAX_TOPK;  // most states of a union lattice
+constexpr int LQ_FLOATS = (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK;  // select_kernel's scratch
+static_assert((2 + MAX_NHEADS + 2 + MAX_NHEADS) * MS <= LQ_FLOATS, "union Viterbi scratch");
+static_assert((2 + MAX_NHEADS + MAX_NHEADS + 1) * MS <= LQ_FLOATS, "union sampling scratch");
+
+// Union lattice (reading B) of one sequence in `scratch` (>= 20 KB of shared
+// memory): states [MS] (the distinct ids of all heads' top-k, ascending) and
+// emissions em [MAX_NHEADS][MS] (head t's fp32 logp of every state; position 1
+// forced to head 1's top-1 under VERIFY_GREEDY).  Returns the state count m.
+__device__ int union_states(const SelectArgs& a, int bl, int n, int k, const int* s_ids, unsigned char* scratch) {
     int* states = reinterpret_cast<int*>(scratch);            // [MS]
     int* first = states + MS;                                 // [MS]
     float* em = reinterpret_cast<float*>(first + MS);         // [MAX_NHEADS][MS]
-    float* delta = em + MAX_NHEADS * MS;                      // [2][MS]
-    int* psi = reinterpret_cast<int*>(delta + 2 * MS);        // [MAX_NHEADS][MS]
     __shared__ int s_m;
     const int tid = threadIdx.x, N = n * k;
     for (int t = tid; t < N; t += blockDim.x) {  // first occurrence of each id
@@ -206,6 +212,16 @@ __device__ void union_viterbi(const SelectArgs& a, int bl, int n, int k, const i
         em[t * MS + r] = v;
     }
     __syncthreads();
+    return m;
+}
+
+// Viterbi (reading B) over the union lattice union_states built in `scratch`.
+__device__ void union_viterbi(const SelectArgs& a, int n, int m, unsigned char* scratch, int* s_path) {
+    const int* states = reinterpret_cast<const int*>(scratch);
+    const float* em = reinterpret_cast<const float*>(states + 2 * MS);
+    float* delta = const_cast<float*>(em) + MAX_NHEADS * MS;  // [2][MS]
+    int* psi = reinterpret_cast<int*>(delta + 2 * MS);        // [MAX_NHEADS][MS]
+    const int tid = threadIdx.x;
     for (int r = tid; r < m; r += blockDim.x) delta[r] = em[r];
     __syncthreads();
     for (int t = 1; t < n; ++t) {
@@ -239,10 +255,103 @@ __device__ void union_viterbi(const SelectArgs& a, int bl, int n, int k, const i
     }
 }
 
+// SplitMix64 (Steele, Lea, Flood 2014): the output function of a 64-bit counter.
+__device__ __forceinline__ unsigned long long splitmix64(unsigned long long x) {
+    unsigned long long z = x + 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// The uniform of position t of one path draw: 24 bits of SplitMix64 of the
+// counter ((seed * P + slot) * P + generated) * P + t, P = 0x100000001B3,
+// so it is exact in fp32.
+__device__ __forceinline__ float path_uniform(unsigned long long seed, int slot, int generated, int t) {
+    constexpr unsigned long long P = 0x100000001B3ull;
+    const unsigned long long x = ((seed * P + (unsigned long long)slot) * P + (unsigned long long)generated) * P +
+                                 (unsigned long long)t;
+    return (float)(splitmix64(x) >> 40) * (1.0f / 16777216.0f);
+}
+
+// Path sampling (top-k sampling, Fig. 2): one path of a lattice of S <= MS
+// states per position (ids[t * ids_t + r], emissions em[t * em_t + r]) drawn
+// from P(path) ~ prod_t Q(c_{t-1}, c_t) S_t(c_t).  Forward filtering, one
+// thread per state: alpha_t(r) = logsumexp_i(alpha_{t-1}(i) + log Q) + s_t(r)
+// (fp32, running-max form); backward sampling by warp 0: the last state from
+// alpha_{n-1}, each earlier one from alpha_t(r) + log Q(c_{t,r}, next), by the
+// first index whose inclusive prefix sum of exp(w - max) exceeds u * total
+// (clamped to the last index of positive weight).  alpha [MAX_NHEADS][MS] and
+// cum [MS] are shared memory.
+__device__ void sample_lattice(const SelectArgs& a, int b, const int* ids, int ids_t, const float* em, int em_t,
+                               int S, int n, float* alpha, float* cum, int* s_path) {
+    const int tid = threadIdx.x, lane = tid & 31;
+    for (int r = tid; r < S; r += blockDim.x) alpha[r] = em[r];
+    __syncthreads();
+    for (int t = 1; t < n; ++t) {
+        for (int r = tid; r < S; r += blockDim.x) {
+            const float* lq_col = a.log_q + ids[t * ids_t + r];
+            float mx = -INFINITY, sum = 0.f;
+            for (int i = 0; i < S; ++i) {
+                const float x = __fadd_rn(alpha[(t - 1) * MS + i], lq_col[(size_t)ids[(t - 1) * ids_t + i] * a.V]);
+                if (x == -INFINITY) continue;
+                if (x > mx) {
+                    sum = sum * expf(mx - x) + 1.f;
+                    mx = x;
+                } else {
+                    sum += expf(x - mx);
+                }
+            }
+            alpha[t * MS + r] = mx == -INFINITY ? -INFINITY : __fadd_rn(__fadd_rn(mx, logf(sum)), em[t * em_t + r]);
+        }
+        __syncthreads();
+    }
+    if (tid >= 32) return;
+    const int gen = a.gen_count[b];
+    int next = -1;
+    for (int t = n - 1; t >= 0; --t) {
+        auto weight = [&](int r) {
+            const float al = alpha[t * MS + r];
+            return next < 0 ? al : __fadd_rn(al, a.log_q[(size_t)ids[t * ids_t + r] * a.V + next]);
+        };
+        float mx = -INFINITY;
+        for (int r = lane; r < S; r += 32) mx = fmaxf(mx, weight(r));
+        mx = warp_max(mx);
+        float carry = 0.f;
+        int last_pos = 0;
+        for (int r0 = 0; r0 < S; r0 += 32) {
+            const int r = r0 + lane;
+            const float x = r < S ? weight(r) : -INFINITY;
+            const float w = x == -INFINITY ? 0.f : expf(x - mx);
+            float c = w;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const float y = __shfl_up_sync(FULL_MASK, c, o);
+                if (lane >= o) c += y;
+            }
+            if (r < S) cum[r] = carry + c;
+            carry += __shfl_sync(FULL_MASK, c, 31);
+            const unsigned pos = __ballot_sync(FULL_MASK, w > 0.f);
+            if (pos) last_pos = r0 + 31 - __clz(pos);
+        }
+        __syncwarp();
+        const float target = path_uniform(a.seed, b, gen, t) * carry;
+        int pick = -1;
+        for (int r0 = 0; r0 < S && pick < 0; r0 += 32) {
+            const int r = r0 + lane;
+            const unsigned hit = __ballot_sync(FULL_MASK, r < S && cum[r] > target);
+            if (hit) pick = r0 + __ffs(hit) - 1;
+        }
+        if (pick < 0 || pick > last_pos) pick = last_pos;
+        next = ids[t * ids_t + pick];
+        if (lane == 0) s_path[t] = next;
+        __syncwarp();
+    }
+}
+
 __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_accept) {
     __shared__ int s_ids[MAX_NHEADS * MAX_TOPK];
     __shared__ float s_lp[MAX_NHEADS * MAX_TOPK];
-    __shared__ float s_lq[(MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK];
+    __shared__ float s_lq[LQ_FLOATS];
     __shared__ int s_path[MAX_NHEADS];
     __shared__ float s_score;
     const int bl = blockIdx.x, b = a.seq_base + bl;
@@ -270,7 +379,19 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     }
     if (!do_accept) return;
     if (a.lattice == 1) {
-        union_viterbi(a, bl, n, k, s_ids, reinterpret_cast<unsigned char*>(s_lq), s_path);
+        unsigned char* scratch = reinterpret_cast<unsigned char*>(s_lq);
+        const int m = union_states(a, bl, n, k, s_ids, scratch);
+        if (a.sampling) {
+            const int* states = reinterpret_cast<const int*>(scratch);
+            float* alpha = reinterpret_cast<float*>(scratch) + (2 + MAX_NHEADS) * MS;  // past states, first, em
+            sample_lattice(a, b, states, 0, reinterpret_cast<const float*>(states + 2 * MS), MS, m, n, alpha,
+                           alpha + MAX_NHEADS * MS, s_path);
+        } else {
+            union_viterbi(a, n, m, scratch, s_path);
+        }
+    } else if (a.sampling) {
+        float* alpha = s_lq;
+        sample_lattice(a, b, s_ids, k, s_lp, k, k, n, alpha, alpha + MAX_NHEADS * MS, s_path);
     } else {
         gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
         __syncthreads();
