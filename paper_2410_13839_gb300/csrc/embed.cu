@@ -18,11 +18,15 @@ __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
         int seq = -1, pos = 0, tok = 0, phone = 0, last = 0;
         if (a.mode == 0) {  // decode: row r is fed token j of slot seq_base + r / n
             const int b = a.seq_base + r / a.n_heads, j = r % a.n_heads;
-            if (r < a.rows && b < a.slots && a.active[b] && !a.done[b] && j < a.n_pending[b]) {
-                seq = b;
-                pos = a.seq_len[b] + j;
-                tok = a.pending[b * a.n_max + j];
-                last = (j == a.n_pending[b] - 1);
+            if (r < a.rows && b < a.slots) {  // the slot's state in one round of independent loads
+                const int act = a.active[b], dn = a.done[b], np = a.n_pending[b], len = a.seq_len[b];
+                const int t = a.pending[b * a.n_max + j];
+                if (act && !dn && j < np) {
+                    seq = b;
+                    pos = len + j;
+                    tok = t;
+                    last = (j == np - 1);
+                }
             }
         } else {  // prefill chunk: positions p0 .. p0 + rows - 1 of one slot
             pos = a.p0 + r;

@@ -71,8 +71,9 @@ __global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
     if (tid == 0 && wbytes > 0) {
         mbar_arrive_expect_tx(&bar, (uint32_t)wbytes);
         const char* src = reinterpret_cast<const char*>(a.W) + (size_t)r0 * K * sizeof(WT);
+        const uint64_t pol = l2_evict_first_policy();
         for (size_t off = 0; off < wbytes; off += BULK_CHUNK)
-            bulk_copy_g2s(smem + off, src + off, (uint32_t)min((size_t)BULK_CHUNK, wbytes - off), &bar);
+            bulk_copy_g2s_hint(smem + off, src + off, (uint32_t)min((size_t)BULK_CHUNK, wbytes - off), &bar, pol);
     }
 
     // ---- parameters (weights): read before the wait ----

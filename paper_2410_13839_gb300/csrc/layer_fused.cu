@@ -487,9 +487,12 @@ __device__ __forceinline__ void plan_row(const LayerArgs& a, int r, int& seq, in
     if (a.plan == PLAN_DEVICE) {
         const int g = r / a.rows_per_group, j = r % a.rows_per_group;
         const int b = a.seq_base + g;
-        if (b < a.slots && a.active[b] && !a.done[b] && j < a.seq_new[b]) {
-            seq = b;
-            pos = a.seq_len[b] + j;
+        if (b < a.slots) {  // one round of independent loads
+            const int act = a.active[b], dn = a.done[b], nw = a.seq_new[b], len = a.seq_len[b];
+            if (act && !dn && j < nw) {
+                seq = b;
+                pos = len + j;
+            }
         }
     } else if (r < a.val_new) {
         seq = a.val_seq;
@@ -622,8 +625,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         }
         mbar_arrive_expect_tx(&bar, wq + kvb);
         const char* srcq = reinterpret_cast<const char*>(a.wqkv) + ((size_t)h * 3 * HEAD_DIM + s * QROWS) * d * sizeof(WT);
+        const uint64_t pol = l2_evict_first_policy();
         for (uint32_t off = 0; off < wq; off += 32768)
-            bulk_copy_g2s(smem + L.wqkv + off, srcq + off, min(32768u, wq - off), &bar);
+            bulk_copy_g2s_hint(smem + L.wqkv + off, srcq + off, min(32768u, wq - off), &bar, pol);
         for (int i = 0; i < n_pre; ++i) {
             const int phys = a.block_table[(size_t)seq * a.bt_stride + pg0 + i];
             const __nv_bfloat16* base = a.kv_pool + (long long)phys * a.page_elems + a.layer_off + kv_head;
@@ -729,9 +733,9 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
         fence_proxy_async();  // the spaces were last written and read by this CTA's threads
         const uint32_t wob = (uint32_t)orows * HEAD_DIM * sizeof(WT);
         mbar_arrive_expect_tx(&bar_o, wob);
-        bulk_copy_g2s(smem + L.wo,
-                      reinterpret_cast<const char*>(a.wo) + ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT),
-                      wob, &bar_o);
+        bulk_copy_g2s_hint(smem + L.wo,
+                           reinterpret_cast<const char*>(a.wo) + ((size_t)h * d + s * orows) * HEAD_DIM * sizeof(WT),
+                           wob, &bar_o, l2_evict_first_policy());
         s_armed = 0;
         const int seq = s_gseq[0];
         if (seq >= 0) {
@@ -1066,9 +1070,10 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
         const size_t off0 = (size_t)f0 * d * sizeof(WT);
         const char* s1 = reinterpret_cast<const char*>(a.w1) + off0;
         const char* s2 = reinterpret_cast<const char*>(a.w2t) + off0;
+        const uint64_t pol = l2_evict_first_policy();
         for (uint32_t off = 0; off < wb; off += 32768) {
-            bulk_copy_g2s(smem + L.w1 + off, s1 + off, min(32768u, wb - off), &bar);
-            bulk_copy_g2s(smem + L.w2 + off, s2 + off, min(32768u, wb - off), &bar);
+            bulk_copy_g2s_hint(smem + L.w1 + off, s1 + off, min(32768u, wb - off), &bar, pol);
+            bulk_copy_g2s_hint(smem + L.w2 + off, s2 + off, min(32768u, wb - off), &bar, pol);
         }
     } else if (tid == 32 && R > 0 && a.next_w_a) {  // the next layer's slices, into L2
         const uint32_t wb = (uint32_t)R * d * sizeof(WT);

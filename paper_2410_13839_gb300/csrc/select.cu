@@ -107,50 +107,43 @@ __device__ __forceinline__ void gather_transitions(const int* ids, int n, int k,
     }
 }
 
-// Viterbi over ids/lp [n][k] with transitions lq [n-1][k][k] (all shared
-// memory); lane 0 receives the results.
-__device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, int n, int k, int* path,
+// Viterbi over ids/lp [n][k] with transitions lq [n-1][k][k] and backpointers
+// bp [MAX_NHEADS][32] (all shared memory); lane 0 writes the results.  The
+// loops stay rolled: the kernel runs once per step with a cold instruction
+// cache, so its time follows the instructions it fetches.
+__device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, int n, int k, int* bp, int* path,
                              float* score) {
     const int lane = threadIdx.x & 31;
     const bool on = lane < k;
     float delta = on ? lp[lane] : -INFINITY;
-    int bp[MAX_NHEADS];
-#pragma unroll
-    for (int t = 1; t < MAX_NHEADS; ++t) {
-        bp[t] = 0;
-        if (t < n) {
-            const float* lqt = lq + (size_t)(t - 1) * k * k + (on ? lane : 0);
-            float best = 0.f;
-            int arg = 0;
-            for (int i = 0; i < k; ++i) {
-                const float di = __shfl_sync(FULL_MASK, delta, i);
-                const float val = __fadd_rn(di, lqt[i * k]);
-                if (i == 0 || val > best) {
-                    best = val;
-                    arg = i;
-                }
+#pragma unroll 1
+    for (int t = 1; t < n; ++t) {
+        const float* lqt = lq + (size_t)(t - 1) * k * k + (on ? lane : 0);
+        float best = 0.f;
+        int arg = 0;
+#pragma unroll 1
+        for (int i = 0; i < k; ++i) {
+            const float di = __shfl_sync(FULL_MASK, delta, i);
+            const float val = __fadd_rn(di, lqt[i * k]);
+            if (i == 0 || val > best) {
+                best = val;
+                arg = i;
             }
-            delta = on ? __fadd_rn(best, lp[t * k + lane]) : -INFINITY;
-            bp[t] = arg;
         }
+        delta = on ? __fadd_rn(best, lp[t * k + lane]) : -INFINITY;
+        bp[t * 32 + lane] = arg;
     }
     float bv = delta;
     int bj = on ? lane : 0x7fffffff;
     warp_argmax(bv, bj);
-    int state = bj;
-    int st[MAX_NHEADS];
-#pragma unroll
-    for (int t = MAX_NHEADS - 1; t >= 0; --t) {
-        st[t] = 0;
-        if (t < n) {
-            st[t] = state;
-            if (t > 0) state = __shfl_sync(FULL_MASK, bp[t], state);
-        }
-    }
+    __syncwarp();
     if (lane == 0) {
-#pragma unroll
-        for (int t = 0; t < MAX_NHEADS; ++t)
-            if (t < n) path[t] = ids[t * k + st[t]];
+        int state = bj;
+#pragma unroll 1
+        for (int t = n - 1; t >= 0; --t) {
+            path[t] = ids[t * k + state];
+            if (t > 0) state = bp[t * 32 + state];
+        }
         *score = bv;
     }
 }
@@ -280,10 +273,10 @@ __device__ __forceinline__ float path_uniform(unsigned long long seed, int slot,
 // (fp32, running-max form); backward sampling by warp 0: the last state from
 // alpha_{n-1}, each earlier one from alpha_t(r) + log Q(c_{t,r}, next), by the
 // first index whose inclusive prefix sum of exp(w - max) exceeds u * total
-// (clamped to the last index of positive weight).  alpha [MAX_NHEADS][MS] and
-// cum [MS] are shared memory.
-__device__ void sample_lattice(const SelectArgs& a, int b, const int* ids, int ids_t, const float* em, int em_t,
-                               int S, int n, float* alpha, float* cum, int* s_path) {
+// (clamped to the last index of positive weight); gen = tokens the slot has
+// generated.  alpha [MAX_NHEADS][MS] and cum [MS] are shared memory.
+__device__ void sample_lattice(const SelectArgs& a, int b, int gen, const int* ids, int ids_t, const float* em,
+                               int em_t, int S, int n, float* alpha, float* cum, int* s_path) {
     const int tid = threadIdx.x, lane = tid & 31;
     for (int r = tid; r < S; r += blockDim.x) alpha[r] = em[r];
     __syncthreads();
@@ -306,7 +299,6 @@ __device__ void sample_lattice(const SelectArgs& a, int b, const int* ids, int i
         __syncthreads();
     }
     if (tid >= 32) return;
-    const int gen = a.gen_count[b];
     int next = -1;
     for (int t = n - 1; t >= 0; --t) {
         auto weight = [&](int r) {
@@ -353,15 +345,26 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     __shared__ float s_lp[MAX_NHEADS * MAX_TOPK];
     __shared__ float s_lq[LQ_FLOATS];
     __shared__ int s_path[MAX_NHEADS];
+    __shared__ int s_bp[MAX_NHEADS * 32];
+    __shared__ int s_emit[MAX_NHEADS + 1];
     __shared__ float s_score;
     const int bl = blockIdx.x, b = a.seq_base + bl;
     const int warp = threadIdx.x >> 5;
     const int n = a.n, k = a.k;
+    __shared__ int s_st[6];  // active, done, remaining, generated, fed rows, cached length
     TraceEnd trace_guard(a.trace);
     pdl_launch_dependents();
+    // The slot's state, read before the wait: the kernels of a step before
+    // this one do not change it.
+    if (do_accept && threadIdx.x < 6) {
+        const int* src = threadIdx.x == 0 ? a.active : threadIdx.x == 1 ? a.done : threadIdx.x == 2 ? a.remaining
+                         : threadIdx.x == 3 ? a.gen_count : threadIdx.x == 4 ? a.n_pending : a.seq_len;
+        s_st[threadIdx.x] = src[b];
+    }
+    __syncthreads();
     pdl_wait();
     trace_wait(a.trace);
-    if (do_accept && (!a.active[b] || a.done[b])) {
+    if (do_accept && (!s_st[0] || s_st[1])) {
         if (threadIdx.x < a.n_max) a.out_tokens[(size_t)b * a.n_max + threadIdx.x] = -1;
         if (threadIdx.x == 0) a.out_accepted[b] = 0;
         return;
@@ -371,6 +374,7 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         head_topk_warp(a.logits + row * a.V, a.V, k, s_ids + warp * k, s_lp + warp * k, a.lse + row);
     }
     __syncthreads();
+    trace_mark(a.trace, 0);  // candidates
     if (do_accept && a.policy == 1 && threadIdx.x > 0 && threadIdx.x < k) s_lp[threadIdx.x] = -INFINITY;  // force
     __syncthreads();
     for (int i = threadIdx.x; i < n * k; i += blockDim.x) {
@@ -384,54 +388,63 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         if (a.sampling) {
             const int* states = reinterpret_cast<const int*>(scratch);
             float* alpha = reinterpret_cast<float*>(scratch) + (2 + MAX_NHEADS) * MS;  // past states, first, em
-            sample_lattice(a, b, states, 0, reinterpret_cast<const float*>(states + 2 * MS), MS, m, n, alpha,
+            sample_lattice(a, b, s_st[3], states, 0, reinterpret_cast<const float*>(states + 2 * MS), MS, m, n, alpha,
                            alpha + MAX_NHEADS * MS, s_path);
         } else {
             union_viterbi(a, n, m, scratch, s_path);
         }
     } else if (a.sampling) {
         float* alpha = s_lq;
-        sample_lattice(a, b, s_ids, k, s_lp, k, k, n, alpha, alpha + MAX_NHEADS * MS, s_path);
+        sample_lattice(a, b, s_st[3], s_ids, k, s_lp, k, k, n, alpha, alpha + MAX_NHEADS * MS, s_path);
     } else {
         gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
         __syncthreads();
-        if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_path, &s_score);
+        if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_bp, s_path, &s_score);
     }
     __syncthreads();
-    if (threadIdx.x != 0) return;
+    trace_mark(a.trace, 1);  // path
+    if (warp != 0) return;
 
-    int acc, done;
-    const int rem = a.remaining[b];
-    const int gc = a.gen_count[b];
-    int emit[MAX_NHEADS];  // tokens this step emits (before the EOS / budget cut)
-    int n_emit;
+    // Acceptance and the slot's bookkeeping, one lane per token (short code:
+    // see viterbi_warp).
+    const int lane = threadIdx.x & 31;
+    const int rem = s_st[2], gc = s_st[3];
+    int n_emit;  // tokens this step emits (before the EOS / budget cut), s_emit
     if (a.policy == 1) {  // kept drafts, then head 1's argmax at the last kept row
-        const int fed = a.n_pending[b];
+        const int fed = s_st[4];
         const int kept = fed > 0 ? a.kept[b] : 0;
-        for (int t = 0; t < kept; ++t) emit[t] = a.pending[(size_t)b * a.n_max + 1 + t];
-        emit[kept] = s_path[0];
+        if (lane < kept) s_emit[lane] = a.pending[(size_t)b * a.n_max + 1 + lane];
+        if (lane == kept) s_emit[kept] = s_path[0];
         n_emit = kept + 1;
-        a.seq_len[b] += fed > 0 ? kept + 1 : 0;  // the confirmed token and the kept drafts stay cached
+        if (lane == 0) a.seq_len[b] = s_st[5] + (fed > 0 ? kept + 1 : 0);  // confirmed token + kept drafts stay
     } else {
-        for (int t = 0; t < n; ++t) emit[t] = s_path[t];
+        if (lane < n) s_emit[lane] = s_path[lane];
         n_emit = n;
-        a.seq_len[b] += a.n_pending[b];  // the tokens fed this step are now cached
+        if (lane == 0) a.seq_len[b] = s_st[5] + s_st[4];  // the tokens fed this step are now cached
     }
-    accept_all(emit, n_emit, a.eos_id, rem, acc, done);
+    __syncwarp();
+    // ACCEPT_ALL on the emitted list: cut after the first EOS and at the budget
+    const int e = lane < n_emit ? s_emit[lane] : -1;
+    const unsigned eos_at = __ballot_sync(FULL_MASK, lane < n_emit && e == a.eos_id);
+    int acc = eos_at ? __ffs(eos_at) : n_emit;
+    acc = min(acc, max(rem, 0));
+    const bool done = (eos_at != 0 && acc >= 1 && s_emit[acc - 1] == a.eos_id) || rem - acc <= 0;
     if (gc + acc > a.gen_stride) {
-        atomicOr(a.err, ERR_BOUNDS);
+        if (lane == 0) atomicOr(a.err, ERR_BOUNDS);
         acc = max(0, a.gen_stride - gc);
     }
-    for (int t = 0; t < a.n_max; ++t) a.out_tokens[(size_t)b * a.n_max + t] = t < acc ? emit[t] : -1;
-    for (int t = 0; t < n; ++t) a.path[(size_t)b * n + t] = s_path[t];
-    for (int t = 0; t < acc; ++t) a.gen_tokens[(size_t)b * a.gen_stride + gc + t] = emit[t];
     const int n_next = a.policy == 1 ? n : acc;  // VERIFY_GREEDY feeds the path: confirmed token + drafts
-    for (int t = 0; t < n_next; ++t) a.pending[(size_t)b * a.n_max + t] = s_path[t];
-    a.gen_count[b] = gc + acc;
-    a.remaining[b] = rem - acc;
-    a.n_pending[b] = done ? 0 : n_next;
-    a.done[b] = done;
-    a.out_accepted[b] = acc;
+    if (lane < a.n_max) a.out_tokens[(size_t)b * a.n_max + lane] = lane < acc ? e : -1;
+    if (lane < n) a.path[(size_t)b * n + lane] = s_path[lane];
+    if (lane < acc) a.gen_tokens[(size_t)b * a.gen_stride + gc + lane] = e;
+    if (lane < n_next) a.pending[(size_t)b * a.n_max + lane] = s_path[lane];
+    if (lane == 0) {
+        a.gen_count[b] = gc + acc;
+        a.remaining[b] = rem - acc;
+        a.n_pending[b] = done ? 0 : n_next;
+        a.done[b] = done;
+        a.out_accepted[b] = acc;
+    }
 }
 
 __global__ void __launch_bounds__(256) verify_kernel(const VerifyArgs a) {
@@ -473,6 +486,7 @@ __global__ void __launch_bounds__(VIT_WARPS * 32) viterbi_kernel(const ViterbiAr
     __shared__ int s_ids[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
     __shared__ float s_lp[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
     __shared__ int s_path[VIT_WARPS][MAX_NHEADS];
+    __shared__ int s_bp[VIT_WARPS][MAX_NHEADS * 32];
     __shared__ float s_score[VIT_WARPS];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x * VIT_WARPS + warp;
@@ -486,7 +500,7 @@ __global__ void __launch_bounds__(VIT_WARPS * 32) viterbi_kernel(const ViterbiAr
     float* lq = vit_lq + (size_t)warp * (a.n - 1) * a.k * a.k;
     gather_transitions(s_ids[warp], a.n, a.k, a.log_q, a.vocab, lq, lane, 32);
     __syncwarp();
-    viterbi_warp(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_path[warp], &s_score[warp]);
+    viterbi_warp(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_bp[warp], s_path[warp], &s_score[warp]);
     __syncwarp();
     if (lane != 0) return;
     int acc, done;
