@@ -447,7 +447,10 @@ def run_ours(args):
     step_roof = {"decode_bytes": dec_bytes, "decode_ms": decode_ms,
                  "achieved_gbs": dec_bytes / (decode_ms / 1e3) / 1e9,
                  "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak}
-    launches_per_step = 3 + ((N_PH + N_AC + 7) // 8) * (1 + 2 * L) + decode_steps // args.steps * (3 + 2 * L)
+    # prefill: two slot updates, then per 128-position chunk the embedding, 8 batched-path kernels per
+    # layer and the last-row save; decode: embedding, 2 block kernels per layer, heads, selection
+    launches_per_step = (2 + ((N_PH + N_AC + 127) // 128) * (2 + 8 * L)
+                         + decode_steps // args.steps * (3 + 2 * L))
 
     line = {"metric": METRIC, "value": value, "unit": "codec tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",

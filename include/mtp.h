@@ -186,7 +186,8 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
 /* Options:
  *   MTP_OPT_GRAPHS       1 = capture each (n_heads, top_k) step into a CUDA graph (default)
  *   MTP_OPT_PDL          1 = programmatic dependent launch between kernels (default)
- *   MTP_OPT_L2_PREFETCH  1 = each block kernel prefetches the next layer's weights into L2 (default)
+ *   MTP_OPT_L2_PREFETCH  1 = each block kernel prefetches the next layer's weights into L2; 0 = no
+ *                        prefetch (default: measured no faster, and it doubles the DRAM reads)
  *   MTP_OPT_MLP_CLUSTERS thread-block clusters of the MLP kernel (>= 1; default: as many as
  *                        the GPU holds at once)
  *   MTP_OPT_BATCHED      1 = decode steps whose fed rows (max_batch * n_heads) exceed one fused

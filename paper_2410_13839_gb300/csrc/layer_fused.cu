@@ -41,8 +41,11 @@ constexpr int CA = 8;                    // CTAs per head (cluster of kernel A)
 constexpr int QROWS = 3 * HEAD_DIM / CA;  // projection rows per CTA (24)
 constexpr int MAX_PRE_KEYS = 192;         // cached keys per CTA staged before the dependency wait
 // dynamic shared memory of kernel A: small enough for two CTAs per SM (16
-// clusters of 8 fit at once only so)
-constexpr size_t A_SMEM_CAP = 113664;
+// clusters of 8 fit at once only so), and for one CTA beside one CTA of kernel B
+// (at d = 1024, 4 fed rows: 88.75 + 133.25 KB of the SM's 228), so that under
+// programmatic launch each kernel's CTAs start, and copy their weights, while
+// the previous kernel still runs
+constexpr size_t A_SMEM_CAP = 91136;
 constexpr int PARTW = 2 + HEAD_DIM;       // (max, sum, out[64])
 constexpr int NTHREADS = 256;
 constexpr int NWARPS = NTHREADS / 32;
@@ -1217,7 +1220,11 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
 
 template <typename T>
 cudaError_t set_smem(T kern, size_t bytes) {
-    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e != cudaSuccess) return e;
+    // the whole unified L1 as shared memory, so CTAs of the two block kernels can share an SM
+    return cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                (int)cudaSharedmemCarveoutMaxShared);
 }
 
 template <typename WT, int MT>

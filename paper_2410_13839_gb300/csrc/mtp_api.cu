@@ -95,7 +95,7 @@ struct mtp_ctx {
     cudaStream_t cap_stream = nullptr;
     int device = 0, num_sms = 0, wbytes = 2;
     int mlp_clusters = 1;  // MLP clusters co-resident in one wave
-    bool use_graphs = true, use_pdl = true, use_l2_prefetch = true;
+    bool use_graphs = true, use_pdl = true, use_l2_prefetch = false;
     std::vector<void*> allocs;
     // weights
     void* d_weights = nullptr;

