@@ -187,8 +187,29 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
     }
     __syncthreads();
     const int seq = s_seq, K_tot = s_ktot, n_pre = s_pre;
+    // output pair (2 lane, 2 lane + 1) of head h in row row_j of the group
+    auto put = [&](int row_j, float v0, float v1) {
+        const size_t r = (size_t)(g * rpg + row_j);
+        if (a.out) {
+            float* o = a.out + r * a.ldo + h * HEAD_DIM + 2 * lane;
+            o[0] = v0;
+            o[1] = v1;
+        }
+        if (a.out_hi) {
+            uint32_t hi, lo;
+            split2(v0, v1, hi, lo);
+            *reinterpret_cast<uint32_t*>(a.out_hi + r * a.ldb + h * HEAD_DIM + 2 * lane) = hi;
+            *reinterpret_cast<uint32_t*>(a.out_lo + r * a.ldb + h * HEAD_DIM + 2 * lane) = lo;
+        }
+    };
     if (seq < 0) {  // nothing to do for this group (no split of it counts)
         if (n_pre > 0) mbar_wait(&bar, 0, a.err);
+        if (a.out_hi && sp == 0)
+            for (int row_j = warp; row_j < rpg; row_j += ATT_THREADS / 32) {
+                const size_t o = (size_t)(g * rpg + row_j) * a.ldb + h * HEAD_DIM + 2 * lane;
+                *reinterpret_cast<uint32_t*>(a.out_hi + o) = 0u;
+                *reinterpret_cast<uint32_t*>(a.out_lo + o) = 0u;
+            }
         return;
     }
 
@@ -360,15 +381,14 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
             acc1[q] = fmaf(sc, ws[3 + 2 * lane], acc1[q]);
         }
     }
-    auto out_row = [&](int row_j) { return a.out + (size_t)(g * rpg + row_j) * a.ldo + h * HEAD_DIM + 2 * lane; };
     if (S == 1) {
 #pragma unroll
         for (int q = 0; q < RPW; ++q) {
             const int row_j = warp + q * NW;
             if (row_j < RPG && s_act[row_j]) {
-                float* o = out_row(row_j);
-                o[0] = acc0[q] / l_run[q];
-                o[1] = acc1[q] / l_run[q];
+                put(row_j, acc0[q] / l_run[q], acc1[q] / l_run[q]);
+            } else if (row_j < rpg && a.out_hi) {
+                put(row_j, 0.f, 0.f);
             }
         }
         return;
@@ -396,7 +416,10 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
 
 #pragma unroll 1
     for (int row_j = warp; row_j < RPG; row_j += NW) {
-        if (!s_act[row_j]) continue;
+        if (!s_act[row_j]) {
+            if (row_j < rpg && a.out_hi) put(row_j, 0.f, 0.f);
+            continue;
+        }
         // lane s holds split s's (max, sum); every split's output pair is
         // loaded before any is used, so the merge costs one L2 round trip
         const float* base = a.ws_part + ((size_t)(g * H + h) * S * RPG) * PART + row_j * PART;
@@ -422,9 +445,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
             r0 = fmaf(ws, o0[sx], r0);
             r1 = fmaf(ws, o1[sx], r1);
         }
-        float* o = out_row(row_j);
-        o[0] = r0 / L;
-        o[1] = r1 / L;
+        put(row_j, r0 / L, r1 / L);
     }
     if (tid == 0) a.ws_count[g * H + h] = 0;
 }

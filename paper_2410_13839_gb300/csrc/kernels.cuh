@@ -66,7 +66,9 @@ struct AttnArgs {
     const __nv_bfloat16* kv_pool; long long page_elems; long long layer_off;
     const int* block_table; int bt_stride;
     const int* row_seq; const int* row_pos;
-    float* out; int ldo;
+    float* out; int ldo;                       // fp32 output rows, or null
+    __nv_bfloat16* out_hi; __nv_bfloat16* out_lo; int ldb;  // or null: output rows as bf16 hi + lo (the
+                                               // W_o GEMM's operand; rows of no sequence written as zeros)
     float* ws_part; int* ws_count;             // split partials and per-(group, head) counters
     int rows_per_group, n_heads, page_size, n_splits;
     int plan;

@@ -107,7 +107,7 @@ struct mtp_ctx {
     bool use_batched = true, batched_ok = false;
     int bm_max = 0;  // rows of the batched buffers: max_batch * n_heads_max
     uint16_t* d_w2p = nullptr;  // W2 [layers][d][F] as stored in the blob (the fused kernels keep it transposed)
-    float *d_bx = nullptr, *d_bqkv = nullptr, *d_bq = nullptr, *d_batt = nullptr, *d_bh = nullptr;
+    float *d_bx = nullptr, *d_bqkv = nullptr, *d_bq = nullptr, *d_bh = nullptr;
     float* d_bws = nullptr;  // attention split partials
     int* d_bwc = nullptr;    // attention split counters
     int battn_ws_units = 1;  // (group, split) pairs the attention workspace holds
@@ -349,7 +349,7 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         at.layer_off = layer_off;
         at.block_table = c->d_block_table; at.bt_stride = c->pages_per_seq;
         at.row_seq = c->d_row_seq; at.row_pos = c->d_row_pos;
-        at.out = c->d_batt; at.ldo = d;
+        at.out_hi = c->d_ahi; at.out_lo = c->d_alo; at.ldb = d;  // straight into W_o's operand
         at.ws_part = c->d_bws; at.ws_count = c->d_bwc;
         at.rows_per_group = rpg; at.n_heads = H; at.page_size = P;
         at.n_splits = std::min(attn_splits_for(groups, H, P, cf.max_ctx, c->num_sms),
@@ -360,7 +360,6 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         at.trace = tslot(c, MTP_K_ATTN);
         LAUNCH(MTP_K_ATTN, launch_attention(at, groups, s, pdl));
         // x += attention W_o^T + b_o (the per-head W_o blocks are the k-chunks)
-        MTP_TRY(pack(PACK_COPY, c->d_batt, d, nullptr, nullptr, nullptr, c->d_ahi, c->d_alo));
         MTP_TRY(gemm(W.wo, d, d, false, TC_ACCUM, c->d_bx, d, L.bo, d));
         // x += GELU(LN2(x) W1^T + b1) W2^T + b2 (W1's epilogue writes the GELU rows as bf16 hi + lo)
         MTP_TRY(pack(PACK_LN, c->d_bx, d, L.ln2_g, L.ln2_b, nullptr, c->d_ahi, c->d_alo));
@@ -380,7 +379,6 @@ int setup_batched(mtp_ctx* c) {
     MTP_TRY(c->alloc(&c->d_bx, M * d));
     MTP_TRY(c->alloc(&c->d_bqkv, M * 3 * d));
     MTP_TRY(c->alloc(&c->d_bq, M * d));
-    MTP_TRY(c->alloc(&c->d_batt, M * d));
     MTP_TRY(c->alloc(&c->d_bh, M * F));
     uint16_t *ahi, *alo, *uhi, *ulo;
     MTP_TRY(c->alloc(&ahi, M * d));
