@@ -210,15 +210,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
         if (c < chunks) s_ok = 0;
         tc_commit(&done);  // every MMA issued above has completed
-    }
-    if (warp < 2) __syncwarp();
-
-    // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
-    const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
-    tc_fence_after();
-    if (fin && s_ok) {
-        if (tid < NT && (a.epilogue == TC_QKV || a.epilogue == TC_GELU_PACK)) {  // per-row facts, once
-            const int n = arow + tid;
+    } else if (warp >= 2 && (a.epilogue == TC_QKV || a.epilogue == TC_GELU_PACK)) {
+        // per-row facts of the epilogue, gathered by the two idle warps while the ring runs
+        for (int j = tid - 64; j < NT; j += TC_THREADS - 64) {
+            const int n = arow + j;
             const int seq = n < a.m ? a.row_seq[n] : -1;
             long long base = -1;
             int t = 0;
@@ -231,9 +226,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 else
                     base = (long long)page * a.page_elems + a.layer_off + (long long)t * HEAD_DIM;
             }
-            s_rowbase[tid] = seq >= 0 ? base : -2;  // -2: no sequence
-            s_rowt[tid] = a.epilogue == TC_QKV ? t : (seq >= 0);
+            s_rowbase[j] = seq >= 0 ? base : -2;  // -2: no sequence
+            s_rowt[j] = a.epilogue == TC_QKV ? t : (seq >= 0);
         }
+    }
+    if (warp < 2) __syncwarp();
+
+    // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
+    const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
+    tc_fence_after();
+    if (fin && s_ok) {
         // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them),
         // then float4 rows of T -> out, coalesced
         constexpr int TP = TC_M + 4;  // row pitch (floats)
