@@ -34,6 +34,8 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
     return t;
 }
 
+// ALL: every row is packed (no row_seq) and zero_buf is zeroed first.
+template <bool ALL>
 __global__ void __launch_bounds__(PK_THREADS) pack_rows_kernel(const PackArgs a) {
     __shared__ float red[PK_THREADS / 32];
     constexpr int MAXV = 16;  // values per thread: K <= 4096
@@ -42,7 +44,10 @@ __global__ void __launch_bounds__(PK_THREADS) pack_rows_kernel(const PackArgs a)
     pdl_launch_dependents();
     pdl_wait();
     trace_wait(a.trace);
-    const bool on = a.row_seq[r] >= 0;
+    if constexpr (ALL)
+        for (long long i = (long long)r * PK_THREADS + tid; i < a.zero_n; i += (long long)a.m * PK_THREADS)
+            a.zero_buf[i] = 0.f;
+    const bool on = ALL || a.row_seq[r] >= 0;
     const int K = a.k;
     float v[MAXV];
 #pragma unroll
@@ -155,7 +160,12 @@ cudaError_t launch_rows(K kern, const A& args, int rows, cudaStream_t s, bool pd
 
 cudaError_t launch_pack_rows(const PackArgs& a, cudaStream_t s, bool pdl) {
     if (a.k < 1 || a.k > 16 * PK_THREADS || a.m < 1) return cudaErrorInvalidValue;
-    return launch_rows(pack_rows_kernel, a, a.m, s, pdl);
+    if (a.row_seq == nullptr) {
+        if (a.zero_n > 0 && a.zero_buf == nullptr) return cudaErrorInvalidValue;
+        return launch_rows(pack_rows_kernel<true>, a, a.m, s, pdl);
+    }
+    if (a.zero_buf) return cudaErrorInvalidValue;  // zeroing comes with the every-row variant
+    return launch_rows(pack_rows_kernel<false>, a, a.m, s, pdl);
 }
 
 cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl) {

@@ -211,9 +211,11 @@ struct PackArgs {
     const float* x; int ldx;      // input rows [m][ldx], k columns used
     float* zero_after;            // PACK_GELU: rows zeroed after reading (may be x), or null
     const float* gamma; const float* beta; float eps;   // PACK_LN
-    const int* row_seq;           // rows with row_seq < 0 are packed as zeros
+    const int* row_seq;           // rows with row_seq < 0 are packed as zeros (null: every row is packed,
+                                  // and zero_buf [zero_n] is zeroed first)
     __nv_bfloat16* hi; __nv_bfloat16* lo;  // [m][k] bf16 parts: hi + lo = the fp32 row
     int k, m;                     // k <= 4096
+    float* zero_buf; long long zero_n;  // or null: zeroed (an accumulation target of the next kernel)
     unsigned long long* trace;
 };
 struct QkvFinishArgs {
@@ -249,6 +251,7 @@ struct TcGemmArgs {
     __nv_bfloat16* kv_pool; long long page_elems; long long layer_off; int page_size, n_heads;
     const int* block_table; int bt_stride;
     __nv_bfloat16* pack_hi; __nv_bfloat16* pack_lo;  // TC_GELU_PACK: [m][n_w]
+    int n_valid;                  // TC_ACCUM: 0, or only features < n_valid are added (element atomics, any ldo)
     int* err;
     unsigned long long* trace;
 };

@@ -120,6 +120,7 @@ struct mtp_ctx {
         CUtensorMap wqkv, wo, w1, w2;
     };
     std::vector<LayerMaps> lmaps;
+    CUtensorMap heads_map;  // the heads [n_heads_max * V][d] as GEMM weights (batched decode)
     CUtensorMap amap_hi[3], amap_lo[3], umap_hi[3], umap_lo[3];  // activation tiles of 32, 64, 128 rows
     float* d_pe = nullptr;
     // KV cache
@@ -413,6 +414,8 @@ int setup_batched(mtp_ctx* c) {
         bad |= tc_encode_2d(&c->umap_hi[t], c->d_uhi, (uint64_t)F, M, (uint32_t)nts[t], false);
         bad |= tc_encode_2d(&c->umap_lo[t], c->d_ulo, (uint64_t)F, M, (uint32_t)nts[t], false);
     }
+    bad |= tc_encode_2d(&c->heads_map, c->w_heads, (uint64_t)d, (uint64_t)cf.n_heads_max * cf.codec_vocab, 128,
+                        false);
     c->batched_ok = bad == 0;  // without tensor maps the fused path serves every batch
     return MTP_OK;
 }
@@ -434,6 +437,39 @@ EmbedArgs embed_base(mtp_ctx* c) {
 
 // Heads on the hidden states of slots [b0, b0 + m): rows of A, or, with
 // `gather`, the slot's last row fed this step in the single pass `gather`.
+// The heads over the slots' last hidden rows h_last [B][d] on the tensor cores
+// (batched decode): LN_f rows as bf16 hi + lo (the same kernel zeroes the
+// logits), then one split-K GEMM over the first n heads' n V rows, added into
+// logits [B][n V].
+int launch_heads_batched(mtp_ctx* c, int B, int n, cudaStream_t s, bool pdl, Prof* prof) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, V = cf.codec_vocab;
+    PackArgs pa;
+    std::memset(&pa, 0, sizeof(pa));
+    pa.mode = PACK_LN; pa.x = c->d_h_last; pa.ldx = d; pa.gamma = c->lnf_g; pa.beta = c->lnf_b;
+    pa.eps = cf.ln_eps; pa.row_seq = nullptr; pa.hi = c->d_ahi; pa.lo = c->d_alo; pa.k = d; pa.m = B;
+    pa.zero_buf = c->d_logits; pa.zero_n = (long long)B * n * V;
+    pa.trace = tslot(c, MTP_K_PACK);
+    LAUNCH(MTP_K_PACK, launch_pack_rows(pa, s, pdl));
+    const int nt = tc_tile_rows(B), ntiles = (B + nt - 1) / nt;
+    const int n_w = (n * V + 127) / 128 * 128, tiles = n_w / 128, chunks = d / 64;
+    int splits = 1;
+    while (2 * splits <= c->gemm_max_splits && chunks % (2 * splits) == 0 && tiles * ntiles * 2 * splits <= c->num_sms)
+        splits *= 2;
+    TcGemm g;
+    std::memset(&g, 0, sizeof(g));
+    g.w = c->heads_map;
+    g.a_hi = c->amap_hi[tile_index(nt)];
+    g.a_lo = c->amap_lo[tile_index(nt)];
+    g.n_w = n_w; g.nt = nt; g.splits = splits;
+    TcGemmArgs& ga = g.args;
+    ga.out = c->d_logits; ga.ldo = n * V; ga.bias = c->b_heads; ga.m = B;
+    ga.k_chunks = chunks / splits; ga.epilogue = TC_ACCUM; ga.n_valid = n * V; ga.err = c->d_err;
+    ga.trace = tslot(c, MTP_K_HEADS);
+    LAUNCH(MTP_K_HEADS, launch_tc_gemm(g, s, pdl));
+    return MTP_OK;
+}
+
 int launch_heads(mtp_ctx* c, const float* A, int m, int n, float* logits, const float* gather, int b0,
                  cudaStream_t s, bool pdl, Prof* prof) {
     const int d = c->cfg.d_model, V = c->cfg.codec_vocab;
@@ -508,11 +544,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
             LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
         }
-        for (int b0 = 0; b0 < B; b0 += MAX_ROWS) {
-            const int m = std::min(MAX_ROWS, B - b0);
-            MTP_TRY(launch_heads(c, c->d_h_last + (size_t)b0 * d, m, n, c->d_logits + (size_t)b0 * n * V, nullptr,
-                                 b0, s, pdl, prof));
-        }
+        MTP_TRY(launch_heads_batched(c, B, n, s, pdl, prof));
         SelectArgs sa = select_base(c, n, k);
         sa.trace = tslot(c, MTP_K_SELECT);
         LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));

@@ -107,7 +107,7 @@ __host__ __device__ constexpr uint32_t tc_idesc(int nt) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(nt >> 3) << 17) | ((uint32_t)(TC_M >> 4) << 24);
 }
 
-template <int NT>
+template <int NT, bool PART>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tw, const __grid_constant__ CUtensorMap tah,
                    const __grid_constant__ CUtensorMap tal, const TcGemmArgs a) {
@@ -250,6 +250,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         __syncthreads();
         const int rows = min(NT, a.m - arow);
         const int P = a.page_size, H = a.n_heads, d = H * HEAD_DIM;
+        if constexpr (PART) {  // TC_ACCUM of features < n_valid only, element atomics (rows of any pitch)
+            for (int i = tid; i < rows * TC_M; i += TC_THREADS) {
+                const int j = i / TC_M, fl = i % TC_M, f = tile * TC_M + fl;
+                if (f < a.n_valid)
+                    atomicAdd(a.out + (size_t)(arow + j) * a.ldo + f,
+                              T[j * TP + fl] + (a.bias && split == 0 ? a.bias[f] : 0.f));
+            }
+        } else
         for (int i = tid; i < rows * (TC_M / 4); i += TC_THREADS) {
             const int j = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
             const int f = tile * TC_M + f4, n = arow + j;
@@ -330,10 +338,8 @@ size_t tc_smem() {
     return (size_t)tc_stages(NT) * (TC_W_BYTES + 2u * NT * TC_K * 2) + 1024;
 }
 
-template <int NT>
-cudaError_t launch_nt(const TcGemm& g, cudaStream_t s, bool pdl) {
-    auto kern = tc_gemm_kernel<NT>;
-    static size_t configured = 0;
+template <int NT, typename K>
+cudaError_t launch_kern(K kern, size_t& configured, const TcGemm& g, cudaStream_t s, bool pdl) {
     const size_t smem = tc_smem<NT>();
     if (configured < smem) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -351,6 +357,13 @@ cudaError_t launch_nt(const TcGemm& g, cudaStream_t s, bool pdl) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, g.w, g.a_hi, g.a_lo, g.args);
+}
+
+template <int NT>
+cudaError_t launch_nt(const TcGemm& g, cudaStream_t s, bool pdl) {
+    static size_t configured[2] = {0, 0};
+    if (g.args.n_valid) return launch_kern<NT>(tc_gemm_kernel<NT, true>, configured[1], g, s, pdl);
+    return launch_kern<NT>(tc_gemm_kernel<NT, false>, configured[0], g, s, pdl);
 }
 
 }  // namespace
