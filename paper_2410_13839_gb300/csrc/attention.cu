@@ -30,7 +30,7 @@ namespace mtp {
 namespace {
 
 constexpr int ATT_THREADS = 128;  // four warps: four CTAs per SM
-constexpr int ATT_KEYS = 256;    // most keys staged at once (two halves; pages of 128 keys need 128 per half)
+constexpr int ATT_STAGES = 3;    // staging slots of the key/value ring (three 64-key slots keep ~48 KB in flight)
 constexpr int RPG = MAX_ROWS;    // rows per group, upper bound
 constexpr int PART = 2 + HEAD_DIM;  // (max, sum, out[64]) per row and split
 constexpr int MAX_SPLITS = 32;     // one warp lane per split in the merge
@@ -72,17 +72,22 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_
 // One thread calls it; returns whether anything was requested.
 __device__ __forceinline__ bool stage_pages(const AttnArgs& a, int seq, int p_from, int p_to, int slot0,
                                             __nv_bfloat16* Ks, __nv_bfloat16* Vs, long long kv_head_off,
-                                            long long v_off, uint64_t* bar) {
+                                            long long v_off, uint64_t* bar, const int* ids = nullptr,
+                                            int id0 = 0, int n_ids = 0) {
     const int P = a.page_size;
     const uint32_t blk = (uint32_t)P * HEAD_DIM * 2;
+    // page p's id: from the shared copy ids[p - id0] when it holds it, else from the block table
+    auto page_id = [&](int p) {
+        return (ids && p - id0 >= 0 && p - id0 < n_ids) ? ids[p - id0] : a.block_table[(size_t)seq * a.bt_stride + p];
+    };
     uint32_t bytes = 0;
     for (int p = p_from; p < p_to; ++p)
-        if (a.block_table[(size_t)seq * a.bt_stride + p] >= 0) bytes += 2 * blk;
+        if (page_id(p) >= 0) bytes += 2 * blk;
     if (!bytes) return false;
     fence_proxy_async();  // the half was last read by this CTA's threads
     mbar_arrive_expect_tx(bar, bytes);
     for (int p = p_from; p < p_to; ++p) {
-        const int phys = a.block_table[(size_t)seq * a.bt_stride + p];
+        const int phys = page_id(p);
         if (phys < 0) {  // unreserved page: report, never read
             if (a.err) atomicOr(a.err, ERR_BOUNDS);
             continue;
@@ -98,13 +103,15 @@ __device__ __forceinline__ bool stage_pages(const AttnArgs& a, int seq, int p_fr
 __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;         // pages staged before the dependency wait
-    __shared__ uint64_t hbar[2];     // the two staging halves
-    __shared__ int s_armed[2];
+    __shared__ uint64_t hbar[ATT_STAGES];  // the staging slots
+    __shared__ int s_armed[ATT_STAGES];
     __shared__ float s_scale[ATT_THREADS / 32][RPG];
     __shared__ int s_pos[RPG];
     __shared__ int s_act[RPG];
     __shared__ int s_rseq[RPG];
     __shared__ int s_seq, s_ktot, s_pre, s_last;
+    constexpr int ID_CAP = 128;
+    __shared__ int s_ids[ID_CAP];  // this split's page ids (the first ID_CAP), read once
 
     const int sp = blockIdx.x, h = blockIdx.y, g = blockIdx.z;
     TraceEnd trace_guard(a.trace);
@@ -112,16 +119,15 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int HALF_KEYS = half_keys(P);  // keys per staging half
     __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(smem);
-    __nv_bfloat16* Vs = Ks + 2 * HALF_KEYS * HEAD_DIM;
-    float* qs = reinterpret_cast<float*>(Vs + 2 * HALF_KEYS * HEAD_DIM);  // [RPG][64], pre-scaled
+    __nv_bfloat16* Vs = Ks + ATT_STAGES * HALF_KEYS * HEAD_DIM;
+    float* qs = reinterpret_cast<float*>(Vs + ATT_STAGES * HALF_KEYS * HEAD_DIM);  // [RPG][64], pre-scaled
     const int pages_per_batch = HALF_KEYS / P;  // pages per staging half
     const long long kv_head_off = (long long)h * P * HEAD_DIM;
     const long long v_off = (long long)H * P * HEAD_DIM;
 
     if (tid == 0) {
         mbar_init(&bar, 1);
-        mbar_init(&hbar[0], 1);
-        mbar_init(&hbar[1], 1);
+        for (int i = 0; i < ATT_STAGES; ++i) mbar_init(&hbar[i], 1);
         fence_barrier_init();
         s_pre = 0;
     }
@@ -221,15 +227,18 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
         const int j = i / HEAD_DIM, dd = i % HEAD_DIM;
         qs[i] = s_act[j] ? a.q[(size_t)(g * rpg + j) * a.ldq + h * HEAD_DIM + dd] * 0.125f : 0.f;  // 1/sqrt(64)
     }
-    // batches of one staging half each: batch i = pages pg0 + i*ppb .. in half i & 1
+    const int n_ids = min(ID_CAP, max(0, pg1 - pg0));
+    for (int i = tid; i < n_ids; i += ATT_THREADS) s_ids[i] = a.block_table[(size_t)seq * a.bt_stride + pg0 + i];
+    __syncthreads();
+    // batches of one staging slot each: batch i = pages pg0 + i*ppb .. in slot i % ATT_STAGES
     const int n_batches = (pg1 - pg0 + pages_per_batch - 1) / pages_per_batch;
     if (tid == 0) {
-        s_armed[0] = s_armed[1] = 0;
-        for (int i = 0; i < 2 && i < n_batches; ++i) {
+        for (int i = 0; i < ATT_STAGES; ++i) s_armed[i] = 0;
+        for (int i = 0; i < ATT_STAGES && i < n_batches; ++i) {
             const int b0 = pg0 + i * pages_per_batch, b1 = min(pg1, b0 + pages_per_batch);
             const int from = i == 0 ? b0 + n_pre : b0;  // batch 0's first pages came before the wait
             s_armed[i] = stage_pages(a, seq, from, b1, i * pages_per_batch + (from - b0), Ks, Vs, kv_head_off,
-                                     v_off, &hbar[i]);
+                                     v_off, &hbar[i], s_ids, pg0, n_ids);
         }
     }
     __syncthreads();
@@ -255,9 +264,9 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
         for (int i = 0; i < 4; ++i) o[j][i] = 0.f;
     const int swz = a.kv_swizzled ? 7 : 0;
     bool ok = true;
-    uint32_t hphase[2] = {0u, 0u};
+    uint32_t hphase[ATT_STAGES] = {};
     for (int i = 0; i < n_batches; ++i) {
-        const int half = i & 1;
+        const int half = i % ATT_STAGES;
         const int bp = pg0 + i * pages_per_batch;
         const int nk = min(pages_per_batch, pg1 - bp) * P;
         if (i == 0 && n_pre > 0) ok = mbar_wait(&bar, 0, a.err) && ok;
@@ -323,17 +332,17 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
                 mma_bf16(o[2 * dp + 1], pl, v1);
             }
         }
-        __syncthreads();  // every warp is done with this half
-        if (tid == 0 && i + 2 < n_batches) {
-            const int b0 = pg0 + (i + 2) * pages_per_batch, b1 = min(pg1, b0 + pages_per_batch);
+        __syncthreads();  // every warp is done with this slot
+        if (tid == 0 && i + ATT_STAGES < n_batches) {
+            const int b0 = pg0 + (i + ATT_STAGES) * pages_per_batch, b1 = min(pg1, b0 + pages_per_batch);
             s_armed[half] = stage_pages(a, seq, b0, b1, half * pages_per_batch, Ks, Vs, kv_head_off, v_off,
-                                        &hbar[half]);
+                                        &hbar[half], s_ids, pg0, n_ids);
         }
         __syncthreads();
     }
     if (!__syncthreads_and(ok)) {  // error word set; let copies in flight land before leaving
         if (n_pre > 0) mbar_wait(&bar, 0, nullptr);
-        for (int hb = 0; hb < 2; ++hb)
+        for (int hb = 0; hb < ATT_STAGES; ++hb)
             if (s_armed[hb]) mbar_wait(&hbar[hb], hphase[hb], nullptr);
         return;
     }
@@ -457,7 +466,7 @@ size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int /*rows_p
 }
 
 size_t attn_smem_bytes(int page_size) {
-    return (size_t)4 * half_keys(page_size) * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4;
+    return (size_t)2 * ATT_STAGES * half_keys(page_size) * HEAD_DIM * 2 + (size_t)RPG * HEAD_DIM * 4;
 }
 
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms) {
