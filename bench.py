@@ -471,6 +471,31 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_profile_b32():
+    """A small batch-32 decode for kernel captures (not a measurement): 32 slots with
+    40-position prompts (one prefill chunk each), then PROFILE_B32_STEPS decode steps.
+    Per prefill chunk the batched path launches 48 GEMMs and 12 attention kernels;
+    per decode step 49 GEMMs (the heads' included) and 12 attention kernels."""
+    import torch
+    from paper_2410_13839_gb300 import build
+    build.build()
+    from paper_2410_13839_gb300 import mtp
+    w = synth.make_weights(MODEL)
+    stream = torch.cuda.Stream()
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, B32, 512, stream=stream)
+    for b in range(B32):
+        ph, ac = synth.make_prompt(100 + b, 10, 30, MODEL.phone_vocab)
+        dec.prefill(b, ph, ac, 400)
+    for _ in range(PROFILE_B32_STEPS):
+        mtp.mtp_decode_step(dec.ctx, N_HEADS, TOP_K)
+    torch.cuda.synchronize()
+    dec.close()
+    print(json.dumps({"profile_b32": "done", "slots": B32, "decode_steps": PROFILE_B32_STEPS}), flush=True)
+
+
+PROFILE_B32_STEPS = 12
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -480,8 +505,12 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b32", action="store_true", help="skip the batch-32 serving measurement")
     ap.add_argument("--no-sweep", action="store_true", help="skip the head/beam sweep")
+    ap.add_argument("--profile-b32", action="store_true",
+                    help="only run a small batch-32 decode for kernel captures (prints no measurement)")
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.profile_b32:
+        run_profile_b32()
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
