@@ -7,11 +7,6 @@
 //               into them), then the fp32 row as bf16 hi + lo parts, the
 //               activation operand of the tensor-core GEMM.  Rows of no
 //               sequence are written as zeros.
-//   qkv_finish  one CTA per row: the projected q|k|v row (bias included,
-//               head-major features h*192 + {0,64,128} + dd) -> the query row
-//               for the attention, keys and values -> the paged cache (bf16,
-//               16-byte chunks of key row t at chunk ^ (t & 7)); the row is
-//               zeroed for the next layer's split-K accumulation.
 #include <math.h>
 
 #include "common.cuh"
@@ -94,59 +89,11 @@ __global__ void __launch_bounds__(PK_THREADS) pack_rows_kernel(const PackArgs a)
     }
 }
 
-constexpr int QF_THREADS = 128;
-
-// One CTA per row; each thread takes 8 consecutive features (one 16-byte
-// chunk of a key/value row): two float4 loads, then the query as two float4
-// stores or the key/value chunk as one 16-byte store at its swizzled place.
-__global__ void __launch_bounds__(QF_THREADS) qkv_finish_kernel(const QkvFinishArgs a) {
-    const int r = blockIdx.x, tid = threadIdx.x;
-    TraceEnd trace_guard(a.trace);
-    pdl_launch_dependents();
-    pdl_wait();
-    trace_wait(a.trace);
-    const int seq = a.row_seq[r], pos = a.row_pos[r];
-    const int H = a.n_heads, P = a.page_size, d = H * HEAD_DIM;
-    float* row = a.qkv + (size_t)r * 3 * d;
-    int page = -1;
-    if (seq >= 0) {
-        page = a.block_table[(size_t)seq * a.bt_stride + pos / P];
-        if (page < 0 && tid == 0) atomicOr(a.err, ERR_BOUNDS);
-    }
-    const int t = pos % P;
-    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c = tid; c < 3 * d / 8; c += QF_THREADS) {
-        float4* src = reinterpret_cast<float4*>(row + c * 8);
-        const float4 y0 = src[0], y1 = src[1];
-        src[0] = zero;
-        src[1] = zero;
-        if (seq < 0) continue;
-        const int i = c * 8, h = i / (3 * HEAD_DIM), sec = (i / HEAD_DIM) % 3, dd = i % HEAD_DIM;
-        if (sec == 0) {
-            float4* q = reinterpret_cast<float4*>(a.q + (size_t)r * d + h * HEAD_DIM + dd);
-            q[0] = y0;
-            q[1] = y1;
-        } else if (page >= 0) {
-            uint4 pk;
-            auto pair = [](float lo, float hi) {
-                return (uint32_t)f32_to_bf16_bits(lo) | ((uint32_t)f32_to_bf16_bits(hi) << 16);
-            };
-            pk.x = pair(y0.x, y0.y);
-            pk.y = pair(y0.z, y0.w);
-            pk.z = pair(y1.x, y1.y);
-            pk.w = pair(y1.z, y1.w);
-            const long long idx = (long long)page * a.page_elems + a.layer_off + (long long)(sec - 1) * H * P * HEAD_DIM +
-                                  (long long)h * P * HEAD_DIM + (long long)t * HEAD_DIM + (((dd >> 3) ^ (t & 7)) << 3);
-            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(a.kv_pool) + idx) = pk;
-        }
-    }
-}
-
 template <typename K, typename A>
-cudaError_t launch_rows(K kern, const A& args, int rows, cudaStream_t s, bool pdl, int threads = PK_THREADS) {
+cudaError_t launch_rows(K kern, const A& args, int rows, cudaStream_t s, bool pdl) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(rows);
-    cfg.blockDim = dim3(threads);
+    cfg.blockDim = dim3(PK_THREADS);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -166,11 +113,6 @@ cudaError_t launch_pack_rows(const PackArgs& a, cudaStream_t s, bool pdl) {
     }
     if (a.zero_buf) return cudaErrorInvalidValue;  // zeroing comes with the every-row variant
     return launch_rows(pack_rows_kernel<false>, a, a.m, s, pdl);
-}
-
-cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl) {
-    if (a.m < 1) return cudaErrorInvalidValue;
-    return launch_rows(qkv_finish_kernel, a, a.m, s, pdl, QF_THREADS);
 }
 
 }  // namespace mtp

@@ -218,18 +218,7 @@ struct PackArgs {
     float* zero_buf; long long zero_n;  // or null: zeroed (an accumulation target of the next kernel)
     unsigned long long* trace;
 };
-struct QkvFinishArgs {
-    float* qkv;                   // [m][3d], features h*192 + {q,k,v}*64 + dd (bias included); zeroed after use
-    float* q;                     // [m][d] query rows, head h at columns 64h..64h+63
-    __nv_bfloat16* kv_pool; long long page_elems; long long layer_off; int page_size, n_heads;
-    const int* block_table; int bt_stride;
-    const int* row_seq; const int* row_pos;
-    int m;
-    int* err;
-    unsigned long long* trace;
-};
 cudaError_t launch_pack_rows(const PackArgs& a, cudaStream_t s, bool pdl);
-cudaError_t launch_qkv_finish(const QkvFinishArgs& a, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------ tensor-core GEMM ----
 // out[n][f] (+)= sum_k (a_hi[n][k] + a_lo[n][k]) w[f][k] with tcgen05 (tc_gemm.cu).
