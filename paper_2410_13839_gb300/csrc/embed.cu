@@ -11,8 +11,11 @@ __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
     __shared__ int s_tok, s_pos, s_act, s_phone;
     const int r = blockIdx.x, tid = threadIdx.x;
     TraceEnd trace_guard(a.trace);
-    pdl_launch_dependents();
+    // The next kernels read the slot state before their own dependency wait, so
+    // they may start only once this launch is past its wait (the kernel that
+    // updates the slot state is then complete).
     pdl_wait();
+    pdl_launch_dependents();
     trace_wait(a.trace);
     if (tid == 0) {
         int seq = -1, pos = 0, tok = 0, phone = 0, last = 0;

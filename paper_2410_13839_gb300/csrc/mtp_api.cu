@@ -524,7 +524,10 @@ int enqueue_verify(mtp_ctx* c, const float* x, int slots, int n, int b0, cudaStr
     return MTP_OK;
 }
 
-int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof) {
+// chain: the step follows another step in the same stream or graph; its first
+// kernel then starts under programmatic launch (it waits for the previous
+// step's selection before it lets the next kernels start).
+int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof, bool chain = false) {
     const int B = c->cfg.max_batch, d = c->cfg.d_model, V = c->cfg.codec_vocab;
     const int spc = std::max(1, MAX_ROWS / n);
     const bool verify = c->cfg.accept_policy == MTP_VERIFY_GREEDY;
@@ -536,7 +539,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
         e.trace = tslot(c, MTP_K_EMBED);
-        LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
+        LAUNCH(MTP_K_EMBED, launch_embed(e, s, chain && pdl));
         MTP_TRY(run_layers_batched(c, M, n, B, PLAN_DEVICE, s, pdl, prof));
         if (verify) {
             MTP_TRY(enqueue_verify(c, c->d_bx, B, n, 0, s, pdl, prof));
@@ -555,7 +558,8 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof)
         EmbedArgs e = embed_base(c);
         e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
         e.trace = tslot(c, MTP_K_EMBED);
-        LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));  // full dependency on the previous pass
+        // full dependency on the previous pass; the step's first pass may chain to the previous step
+        LAUNCH(MTP_K_EMBED, launch_embed(e, s, b0 == 0 && chain && pdl));
         MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
         if (verify) {
             MTP_TRY(enqueue_verify(c, final_x, G, n, b0, s, pdl, prof));
@@ -605,6 +609,45 @@ int run_step(mtp_ctx* c, int n, int k) {
     }
     c->trace_kinds = c->graph_kinds[key];
     CUDA_TRY(cudaGraphLaunch(it->second, c->stream));
+    return MTP_OK;
+}
+
+// `count` decode steps: graphs of STEPS_PER_GRAPH chained steps, then single steps.
+constexpr int STEPS_PER_GRAPH = 4;
+int run_steps(mtp_ctx* c, int n, int k, int count) {
+    if (!c->use_graphs || c->tracing) {
+        for (int i = 0; i < count; ++i) MTP_TRY(run_step(c, n, k));
+        return MTP_OK;
+    }
+    int done = 0;
+    if (count >= STEPS_PER_GRAPH) {
+        const auto key = std::make_tuple(n, k, 2);  // 2: the chained multi-step graph
+        auto it = c->graphs.find(key);
+        if (it == c->graphs.end()) {
+            cudaGraph_t graph = nullptr;
+            cudaGraphExec_t exec = nullptr;
+            c->trace_kinds.clear();
+            CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
+            int r = MTP_OK;
+            for (int i = 0; i < STEPS_PER_GRAPH && r == MTP_OK; ++i)
+                r = enqueue_step(c, n, k, c->cap_stream, c->use_pdl, nullptr, i > 0);
+            const cudaError_t ec = cudaStreamEndCapture(c->cap_stream, &graph);
+            if (r != MTP_OK) {
+                if (graph) cudaGraphDestroy(graph);
+                return r;
+            }
+            CUDA_TRY(ec);
+            const cudaError_t ei = cudaGraphInstantiate(&exec, graph, 0);
+            cudaGraphDestroy(graph);
+            CUDA_TRY(ei);
+            it = c->graphs.emplace(key, exec).first;
+            c->graph_kinds[key] = c->trace_kinds;
+        }
+        c->last_n = n;
+        c->last_k = k;
+        for (; done + STEPS_PER_GRAPH <= count; done += STEPS_PER_GRAPH) CUDA_TRY(cudaGraphLaunch(it->second, c->stream));
+    }
+    for (; done < count; ++done) MTP_TRY(run_step(c, n, k));
     return MTP_OK;
 }
 
@@ -1127,7 +1170,7 @@ MTP_API int mtp_generate(mtp_ctx* c, int n, int k, int32_t* out_tokens, int out_
         for (int b = 0; b < c->cfg.max_batch; ++b)
             if (active[b] && !done[b]) round = std::max(round, (rem[b] + n - 1) / n);
         if (round == 0) break;
-        for (int i = 0; i < round; ++i) MTP_TRY(run_step(c, n, k));
+        MTP_TRY(run_steps(c, n, k, round));
         steps += round;
         MTP_TRY(check_device_error(c));
     }
