@@ -197,6 +197,72 @@ def run_b32(mtp, stream, warmup, steps):
 SWEEP_GEN = 1500
 
 
+C5_BATCH, C5_N, C5_K, C5_LATTICES = 256, 8, 16, 10000
+
+
+def c5_lattices(count: int, n: int, k: int, vocab: int, seed: int = 5):
+    """Seeded lattices of the microbenchmark shape: per (lattice, position) k distinct ids
+    (an arithmetic progression mod vocab with a step coprime to it) and log-uniform scores
+    sorted in descending order, as a top-k would give them."""
+    rng = np.random.default_rng(seed)
+    start = rng.integers(0, vocab, size=(count, n, 1))
+    step = rng.integers(1, vocab, size=(count, n, 1))
+    bad = np.gcd(step, vocab) != 1
+    while bad.any():
+        step[bad] = rng.integers(1, vocab, size=int(bad.sum()))
+        bad = np.gcd(step, vocab) != 1
+    ids = ((start + step * np.arange(k)) % vocab).astype(np.int32)
+    lp = -np.sort(-np.log1p(-rng.random((count, n, k))), axis=2).astype(np.float32)
+    return ids, lp
+
+
+def run_c5(mtp, ctx, stream):
+    """The isolated head + Viterbi microbenchmark: n=8 heads with log-softmax and top-16
+    on 256 bf16 hidden rows N(0,1) (the context's VALL-E-sized heads), and Viterbi with
+    acceptance over 10^4 lattices of 8 positions x 16 candidates.  CUDA events, 3 warm-up
+    calls; head bytes = the 8 heads' weights once per call."""
+    import torch
+    d, V = MODEL.d_model, MODEL.codec_vocab
+    h = torch.from_numpy(synth.make_hidden(C5_BATCH, d, seed=C5_BATCH)).cuda().to(torch.bfloat16)
+    ids = torch.zeros((C5_BATCH, C5_N, C5_K), dtype=torch.int32, device="cuda")
+    lp = torch.zeros((C5_BATCH, C5_N, C5_K), dtype=torch.float32, device="cuda")
+    lg = torch.zeros((C5_BATCH, C5_N, V), dtype=torch.float32, device="cuda")
+    lse = torch.zeros((C5_BATCH, C5_N), dtype=torch.float32, device="cuda")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    calls = 20
+    for _ in range(3):
+        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, lg, lse)
+    torch.cuda.synchronize()
+    ev[0].record(stream)
+    for _ in range(calls):
+        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, lg, lse)
+    ev[1].record(stream)
+    torch.cuda.synchronize()
+    heads_s = ev[0].elapsed_time(ev[1]) / 1e3 / calls
+    c_ids, c_lp = c5_lattices(C5_LATTICES, C5_N, C5_K, V)
+    t_ids, t_lp = torch.from_numpy(c_ids).cuda(), torch.from_numpy(c_lp).cuda()
+    t_q = torch.from_numpy(synth.transition_log_q(V)).cuda()
+    path = torch.zeros((C5_LATTICES, C5_N), dtype=torch.int32, device="cuda")
+    acc = torch.zeros(C5_LATTICES, dtype=torch.int32, device="cuda")
+    vs = torch.cuda.current_stream()
+    for _ in range(3):
+        mtp.mtp_viterbi(C5_LATTICES, C5_N, C5_K, V, MODEL.eos_id, t_ids, t_lp, t_q, None, path, None, acc, None, vs)
+    torch.cuda.synchronize()
+    ev[2].record(vs)
+    for _ in range(calls):
+        mtp.mtp_viterbi(C5_LATTICES, C5_N, C5_K, V, MODEL.eos_id, t_ids, t_lp, t_q, None, path, None, acc, None, vs)
+    ev[3].record(vs)
+    torch.cuda.synchronize()
+    vit_s = ev[2].elapsed_time(ev[3]) / 1e3 / calls
+    head_bytes = C5_N * V * d * 2
+    flops = 2.0 * C5_BATCH * C5_N * V * d
+    return {"workload": "isolated heads + Viterbi: 256 bf16 hidden rows N(0,1), n=8 heads x V=1025 with "
+                        "log-softmax and top-16; Viterbi + acceptance over 10^4 lattices of 8 x 16",
+            "heads_topk_us": heads_s * 1e6, "heads_gbs": head_bytes / heads_s / 1e9,
+            "heads_tflops": flops / heads_s / 1e12, "viterbi_us": vit_s * 1e6,
+            "viterbi_lattices_per_s": C5_LATTICES / vit_s}
+
+
 def run_sweep(mtp, stream):
     """Head/beam sweep on the VALL-E-sized model (B=1, prompt 64+225, 1500 tokens): tokens/s
     (prefill + decode) and mean accepted tokens per step for each (n, top_k); and the mean
@@ -212,7 +278,7 @@ def run_sweep(mtp, stream):
         ctx = dec.ctx
         ph_d, ac_d = torch.from_numpy(ph).cuda(), torch.from_numpy(ac).cuda()
         lens = torch.zeros(1, dtype=torch.int32, device="cuda")
-        grid = [(n, k) for n in (1, 2, 4, 8) for k in (1, 4, 8)] if policy == 0 else [(4, 4)]
+        grid = [(n, k) for n in (1, 2, 4, 8) for k in (1, 4, 8, 25)] if policy == 0 else [(4, 4)]
         for n, k in grid:
             for rep in range(2):  # the first run captures the step graph
                 ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
@@ -446,7 +512,8 @@ def run_ours(args):
     dec_bytes = _decode_bytes_total(d, F, V, L, N_HEADS, 2, N_PH + N_AC, GEN)
     step_roof = {"decode_bytes": dec_bytes, "decode_ms": decode_ms,
                  "achieved_gbs": dec_bytes / (decode_ms / 1e3) / 1e9,
-                 "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak}
+                 "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak,
+                 "frac_of_nominal_8tbs": dec_bytes / (decode_ms / 1e3) / 1e9 / 8000.0}
     # prefill: two slot updates, then per 128-position chunk the embedding, 8 batched-path kernels per
     # layer and the last-row save; decode: embedding, 2 block kernels per layer, heads, selection
     launches_per_step = (2 + ((N_PH + N_AC + 127) // 128) * (2 + 8 * L)
@@ -460,6 +527,8 @@ def run_ours(args):
             "decode_tokens_per_s": GEN / (decode_ms / 1e3),
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
             "clocks": clk.summary(), "kernel_ms": {k: v[0] for k, v in prof.items()}}
+    if not args.no_c5:
+        line["c5"] = run_c5(mtp, ctx, stream)
     dec.close()
     if not args.no_b32:
         line["b32"] = run_b32(mtp, stream, max(1, min(args.warmup, 2)), max(1, min(args.steps, 3)))
@@ -505,6 +574,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b32", action="store_true", help="skip the batch-32 serving measurement")
     ap.add_argument("--no-sweep", action="store_true", help="skip the head/beam sweep")
+    ap.add_argument("--no-c5", action="store_true", help="skip the isolated heads + Viterbi microbenchmark")
     ap.add_argument("--profile-b32", action="store_true",
                     help="only run a small batch-32 decode for kernel captures (prints no measurement)")
     args = ap.parse_args()

@@ -282,6 +282,9 @@ MTP_API int mtp_viterbi(int batch, int n, int k, int vocab, int eos_id,
  *   out_ids    int32 [batch][n_heads][top_k]; out_logp float, same shape
  *   out_logits float [batch][n_heads][codec_vocab] or NULL
  *   out_lse    float [batch][n_heads] or NULL
+ * More than 8 rows with bf16 weights run on the tensor cores (LN_f rows packed
+ * as bf16 hi + lo, one GEMM over the n_heads * codec_vocab weight rows, head
+ * weights streamed once per chunk of rows); otherwise passes of 8 rows.
  * Uses the context's stream.  Errors: MTP_ERR_INVALID, MTP_ERR_CUDA. */
 MTP_API int mtp_heads_topk(mtp_ctx* ctx, int batch, const void* hidden, int hidden_dtype,
                            int n_heads, int top_k, int32_t* out_ids, float* out_logp,

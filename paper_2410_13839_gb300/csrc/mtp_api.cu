@@ -437,18 +437,19 @@ EmbedArgs embed_base(mtp_ctx* c) {
 
 // Heads on the hidden states of slots [b0, b0 + m): rows of A, or, with
 // `gather`, the slot's last row fed this step in the single pass `gather`.
-// The heads over the slots' last hidden rows h_last [B][d] on the tensor cores
-// (batched decode): LN_f rows as bf16 hi + lo (the same kernel zeroes the
-// logits), then one split-K GEMM over the first n heads' n V rows, added into
+// The heads over B hidden rows x [B][d] (B <= the batched buffers' rows) on the
+// tensor cores: LN_f rows as bf16 hi + lo (the same kernel zeroes the logits),
+// then one split-K GEMM over the first n heads' n V rows, added into
 // logits [B][n V].
-int launch_heads_batched(mtp_ctx* c, int B, int n, cudaStream_t s, bool pdl, Prof* prof) {
+int launch_heads_batched(mtp_ctx* c, const float* x, int B, int n, float* logits, cudaStream_t s, bool pdl,
+                         Prof* prof) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, V = cf.codec_vocab;
     PackArgs pa;
     std::memset(&pa, 0, sizeof(pa));
-    pa.mode = PACK_LN; pa.x = c->d_h_last; pa.ldx = d; pa.gamma = c->lnf_g; pa.beta = c->lnf_b;
+    pa.mode = PACK_LN; pa.x = x; pa.ldx = d; pa.gamma = c->lnf_g; pa.beta = c->lnf_b;
     pa.eps = cf.ln_eps; pa.row_seq = nullptr; pa.hi = c->d_ahi; pa.lo = c->d_alo; pa.k = d; pa.m = B;
-    pa.zero_buf = c->d_logits; pa.zero_n = (long long)B * n * V;
+    pa.zero_buf = logits; pa.zero_n = (long long)B * n * V;
     pa.trace = tslot(c, MTP_K_PACK);
     LAUNCH(MTP_K_PACK, launch_pack_rows(pa, s, pdl));
     const int nt = tc_tile_rows(B), ntiles = (B + nt - 1) / nt;
@@ -463,7 +464,7 @@ int launch_heads_batched(mtp_ctx* c, int B, int n, cudaStream_t s, bool pdl, Pro
     g.a_lo = c->amap_lo[tile_index(nt)];
     g.n_w = n_w; g.nt = nt; g.splits = splits;
     TcGemmArgs& ga = g.args;
-    ga.out = c->d_logits; ga.ldo = n * V; ga.bias = c->b_heads; ga.m = B;
+    ga.out = logits; ga.ldo = n * V; ga.bias = c->b_heads; ga.m = B;
     ga.k_chunks = chunks / splits; ga.epilogue = TC_ACCUM; ga.n_valid = n * V; ga.err = c->d_err;
     ga.trace = tslot(c, MTP_K_HEADS);
     LAUNCH(MTP_K_HEADS, launch_tc_gemm(g, s, pdl));
@@ -547,7 +548,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
             LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
         }
-        MTP_TRY(launch_heads_batched(c, B, n, s, pdl, prof));
+        MTP_TRY(launch_heads_batched(c, c->d_h_last, B, n, c->d_logits, s, pdl, prof));
         SelectArgs sa = select_base(c, n, k);
         sa.trace = tslot(c, MTP_K_SELECT);
         LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
@@ -1349,8 +1350,28 @@ MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden
     const int d = c->cfg.d_model, V = c->cfg.codec_vocab;
     cudaStream_t s = c->stream;
     Prof* prof = nullptr;
-    for (int b0 = 0; b0 < batch; b0 += MAX_ROWS) {
-        const int m = std::min(MAX_ROWS, batch - b0);
+    // more rows than one fused pass: tensor-core heads over chunks of the batched buffers' rows
+    // (of the context's logits rows when the caller passes no logits / lse buffers)
+    const int lrows = std::max(c->cfg.max_batch, MAX_ROWS);
+    const int tc_rows = out_logits && out_lse ? c->bm_max : std::min(c->bm_max, lrows);
+    const bool tc = c->use_batched && c->batched_ok && batch > MAX_ROWS && tc_rows > MAX_ROWS;
+    const int chunk = tc ? tc_rows : MAX_ROWS;
+    for (int b0 = 0; b0 < batch; b0 += chunk) {
+        const int m = std::min(chunk, batch - b0);
+        if (tc) {
+            const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
+            CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,
+                                         hidden_dtype == MTP_BF16, c->d_bx, m, d, s));
+            float* logits = out_logits ? out_logits + (size_t)b0 * n * V : c->d_logits;
+            MTP_TRY(launch_heads_batched(c, c->d_bx, m, n, logits, s, false, prof));
+            SelectArgs sa = select_base(c, n, k);
+            sa.logits = logits;
+            sa.lse = out_lse ? out_lse + (size_t)b0 * n : c->d_lse;
+            sa.cand_ids = out_ids + (size_t)b0 * n * k;
+            sa.cand_logp = out_logp + (size_t)b0 * n * k;
+            CUDA_TRY(launch_select(sa, m, false, s, false));
+            continue;
+        }
         const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
         CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,
                                      hidden_dtype == MTP_BF16, xbuf(c, 0), m, d, s));
