@@ -142,16 +142,16 @@ def _batched_decode_bytes(prompt_lens, gens, d, F, V, L, n, wb):
     return total
 
 
-def run_b32(mtp, stream, warmup, steps):
+def run_b32(mtp, stream, warmup, steps, batch=B32):
     """Whole-job codec tokens/s of the batched-serving workload on this GPU (prefill + decode)."""
     import torch
-    seqs = b32_sequences()
+    seqs = b32_sequences(batch)
     max_ctx = max(len(p) + len(a) + g for p, a, g in seqs) + MODEL.n_heads_max + 8
     w = synth.make_weights(MODEL)
-    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, B32, max_ctx, stream=stream)
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, batch, max_ctx, stream=stream)
     ctx = dec.ctx
     dev = [(torch.from_numpy(p).cuda(), torch.from_numpy(a).cuda(), g) for p, a, g in seqs]
-    lens = torch.zeros(B32, dtype=torch.int32, device="cuda")
+    lens = torch.zeros(batch, dtype=torch.int32, device="cuda")
     torch.cuda.synchronize()
 
     def job(ev=None):
@@ -184,8 +184,8 @@ def run_b32(mtp, stream, warmup, steps):
     peak, peak_kind = _peaks()
     batched = mtp.mtp_get_option(ctx, mtp.MTP_OPT_BATCHED)
     dec.close()
-    return {"value": tokens * steps / (total_ms / 1e3), "unit": "codec tokens/s", "batch": B32,
-            "workload": B32_WORKLOAD, "tokens_per_job": tokens, "jobs": steps, "warmup_jobs": warmup,
+    return {"value": tokens * steps / (total_ms / 1e3), "unit": "codec tokens/s", "batch": batch,
+            "workload": B32_WORKLOAD.replace("B=32", "B=%d" % batch), "tokens_per_job": tokens, "jobs": steps, "warmup_jobs": warmup,
             "ms_per_job": total_ms / steps, "prefill_ms": prefill_ms, "decode_ms": decode_ms,
             "decode_steps_per_job": dsteps // steps, "decode_tokens_per_s": tokens / (decode_ms / 1e3),
             "path": "batched (tensor-core projections)" if batched else "fused 8-row passes",
@@ -541,6 +541,7 @@ def run_ours(args):
     dec.close()
     if not args.no_b32:
         line["b32"] = run_b32(mtp, stream, max(1, min(args.warmup, 2)), max(1, min(args.steps, 3)))
+        line["b128"] = run_b32(mtp, stream, 1, 1, batch=128)
     if not args.no_sweep:
         line["sweep"] = run_sweep(mtp, stream)
     if rank == 0:

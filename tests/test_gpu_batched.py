@@ -84,3 +84,9 @@ def test_batched_equals_fused_passes():
 
 def test_batched_valle_b32():
     batched_teacher_forced(synth.VALLE, batch=32, n=4, k=4, max_new=16, max_steps=2, seed0=500)
+
+
+def test_batched_tiny_bf16_b128():
+    """The batch-128 serving shape: 512 fed rows per step (several activation tiles per
+    projection, 128 attention groups)."""
+    batched_teacher_forced(synth.TINY_BF16, batch=128, n=4, k=4, max_new=16, max_steps=3, seed0=700)
