@@ -614,7 +614,7 @@ int run_step(mtp_ctx* c, int n, int k) {
 }
 
 // `count` decode steps: graphs of STEPS_PER_GRAPH chained steps, then single steps.
-constexpr int STEPS_PER_GRAPH = 4;
+constexpr int STEPS_PER_GRAPH = 8;
 int run_steps(mtp_ctx* c, int n, int k, int count) {
     if (!c->use_graphs || c->tracing) {
         for (int i = 0; i < count; ++i) MTP_TRY(run_step(c, n, k));
