@@ -113,3 +113,16 @@ def test_forced_position_is_kept():
         assert path[0] == ids[0, 0]
         seen.add(tuple(path))
     assert len(seen) > 10   # the drafts after it still vary
+
+
+def test_hand_worked_draws():
+    import json
+    import os
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "sampling_hand.json")))
+    lq = np.log(np.array(g["log_q_probs"])).astype(np.float32)
+    ids = np.array(g["cand_ids"], dtype=np.int32)
+    lp = np.log(np.array(g["cand_probs"])).astype(np.float32)
+    for case in g["cases"]:
+        path, margin = S.sample_path(ids, lp, lq, case["uniforms"])
+        assert path.tolist() == case["path"], case["note"]
+        assert margin > 0.05
