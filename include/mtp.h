@@ -255,6 +255,16 @@ MTP_API int mtp_trace_step(mtp_ctx* ctx, int n_heads, int top_k, int64_t* out, i
  * slot, from the current slot state (host uint64 out). */
 MTP_API int mtp_step_bytes(mtp_ctx* ctx, int n_heads, uint64_t* out_bytes);
 
+/* Self-test of the bounded waits (failure detection without a GPU fault): one
+ * block waits on a shared-memory barrier that nothing completes.  The wait
+ * gives up after its poll limit (the same bounded wait every kernel's barrier
+ * waits use; well under a few seconds), ORs MTP_DEVICE_ERR_WAIT (1) into
+ * *err_word and the kernel returns, leaving the CUDA context usable.
+ *   err_word  int32, device memory
+ * Errors: MTP_ERR_INVALID (null), MTP_ERR_CUDA. */
+#define MTP_DEVICE_ERR_WAIT 1
+MTP_API int mtp_selftest_bounded_wait(int32_t* err_word, void* cuda_stream);
+
 /* ---- stand-alone operators (device pointers, caller's stream) ---------- */
 
 /* Viterbi selection over candidate lattices (Sec. III-C, reading A: the

@@ -1339,6 +1339,27 @@ MTP_API int mtp_viterbi(int batch, int n, int k, int vocab, int eos_id, const in
     return MTP_OK;
 }
 
+namespace {
+// A barrier with one expected arrival that never comes: the bounded wait runs out.
+__global__ void selftest_wait_kernel(int* err) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait(&bar, 0, err);
+}
+}  // namespace
+
+MTP_API int mtp_selftest_bounded_wait(int32_t* err_word, void* cuda_stream) {
+    g_err.clear();
+    if (!err_word) return fail(MTP_ERR_INVALID, "selftest: null error word");
+    selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(cuda_stream)>>>(err_word);
+    CUDA_TRY(cudaGetLastError());
+    return MTP_OK;
+}
+
 MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden_dtype, int n, int k,
                            int32_t* out_ids, float* out_logp, float* out_logits, float* out_lse) {
     g_err.clear();

@@ -180,6 +180,10 @@ def mtp_viterbi(batch, n, k, vocab, eos_id, cand_ids, cand_logp, log_q, remainin
                           _ptr(out_rollback), _stream_handle(stream)))
 
 
+def mtp_selftest_bounded_wait(err_word, stream=None) -> None:
+    check(lib.mtp_selftest_bounded_wait(_ptr(err_word), _stream_handle(stream)))
+
+
 def mtp_heads_topk(ctx, batch, hidden, hidden_dtype, n_heads, top_k, out_ids, out_logp,
                    out_logits=None, out_lse=None) -> None:
     check(lib.mtp_heads_topk(ctx, batch, _ptr(hidden), hidden_dtype, n_heads, top_k, _ptr(out_ids),
