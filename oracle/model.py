@@ -18,7 +18,9 @@ angle-addition identity; LayerNorm moments; GELU against printed normal-CDF
 values; attention special cases (one key returns v, zero query averages,
 future keys have no effect); the block with zeroed weights is the identity
 plus biases; a one-token block against its closed form; cached chunked decode
-against a cache-free full recompute.  Beyond these, the composition of the
+against a cache-free full recompute; invariance to permutations of the
+attention heads, of the FFN units and of the dimensions within a head (which
+a transposed operand or a wrong head layout breaks).  Beyond these, the composition of the
 block is "parity unpinned" against any printed value: the paper prints no
 activation, logit or worked example of the model.
 """

@@ -159,3 +159,99 @@ def test_rollback_then_append_equals_append(tiny_weights):
     dec.forward(prompt, is_phone, c2)
     y2 = dec.forward(np.array([9, 10]), np.zeros(2, bool), c2)
     assert np.array_equal(y1, y2)
+
+
+# ---- permutation invariances of the block: a transposed operand or a wrong head /
+# feature layout in the oracle breaks at least one of them ----
+
+def _forward(cfg, w, seed=11):
+    dec = M.ARDecoder(cfg, w)
+    ph, ac = synth.make_prompt(seed, 6, 14, cfg.phone_vocab)
+    tokens = np.concatenate([ph, ac])
+    return dec.forward(tokens, np.arange(20) < 6, dec.new_cache())
+
+
+def _permute_heads(cfg, w, perm, fix_wo=True):
+    """Heads reordered: q, k and v row blocks of W_qkv (and b_qkv) and W_o's column blocks."""
+    d, H = cfg.d_model, cfg.n_attn_heads
+    hd = d // H
+    rows = np.concatenate([np.arange(p * hd, (p + 1) * hd) for p in perm])
+    out = {k: v.copy() for k, v in w.items()}
+    for layer in range(cfg.layers):
+        p = f"layers.{layer}."
+        idx = np.concatenate([sec * d + rows for sec in range(3)])
+        out[p + "wqkv"] = w[p + "wqkv"][idx]
+        out[p + "bqkv"] = w[p + "bqkv"][idx]
+        if fix_wo:
+            out[p + "wo"] = w[p + "wo"][:, rows]
+    return out
+
+
+def test_block_is_invariant_to_a_head_permutation(tiny_weights):
+    cfg = synth.TINY
+    perm = np.array([2, 0, 3, 1])
+    base = _forward(cfg, tiny_weights)
+    assert np.allclose(_forward(cfg, _permute_heads(cfg, tiny_weights, perm)), base, atol=1e-10)
+    # the same reordering without W_o's columns is a different model
+    assert not np.allclose(_forward(cfg, _permute_heads(cfg, tiny_weights, perm, fix_wo=False)), base, atol=1e-3)
+
+
+def test_block_is_invariant_to_an_ffn_unit_permutation(tiny_weights):
+    cfg = synth.TINY
+    sigma = np.random.default_rng(3).permutation(cfg.d_ffn)
+    w = {k: v.copy() for k, v in tiny_weights.items()}
+    broken = {k: v.copy() for k, v in tiny_weights.items()}
+    for layer in range(cfg.layers):
+        p = f"layers.{layer}."
+        w[p + "w1"] = tiny_weights[p + "w1"][sigma]
+        w[p + "b1"] = tiny_weights[p + "b1"][sigma]
+        w[p + "w2"] = tiny_weights[p + "w2"][:, sigma]
+        broken[p + "w1"] = w[p + "w1"]
+        broken[p + "b1"] = w[p + "b1"]
+    base = _forward(cfg, tiny_weights)
+    assert np.allclose(_forward(cfg, w), base, atol=1e-10)
+    assert not np.allclose(_forward(cfg, broken), base, atol=1e-3)
+
+
+def test_block_is_invariant_to_a_dimension_permutation_within_heads(tiny_weights):
+    """q and k dimensions of every head reordered alike (scores unchanged); v dimensions
+    reordered with W_o's matching columns (outputs unchanged)."""
+    cfg = synth.TINY
+    d, H = cfg.d_model, cfg.n_attn_heads
+    hd = d // H
+    rng = np.random.default_rng(4)
+    tau, rho = rng.permutation(hd), rng.permutation(hd)
+    qk = np.concatenate([h * hd + tau for h in range(H)])
+    vv = np.concatenate([h * hd + rho for h in range(H)])
+    w = {k: v.copy() for k, v in tiny_weights.items()}
+    for layer in range(cfg.layers):
+        p = f"layers.{layer}."
+        idx = np.concatenate([qk, d + qk, 2 * d + vv])
+        w[p + "wqkv"] = tiny_weights[p + "wqkv"][idx]
+        w[p + "bqkv"] = tiny_weights[p + "bqkv"][idx]
+        w[p + "wo"] = tiny_weights[p + "wo"][:, vv]
+    assert np.allclose(_forward(cfg, w), _forward(cfg, tiny_weights), atol=1e-10)
+
+
+def test_a_transposed_output_projection_breaks_the_head_pin(tiny_weights):
+    """Planted mistake: an oracle that applies W_o untransposed (x += att W_o instead of
+    att W_o^T).  It still runs, but the head-permutation invariance fails."""
+    cfg = synth.TINY
+
+    class Planted(M.ARDecoder):
+        def block(self, layer, x, positions, cache):
+            key = f"layers.{layer}.wo"
+            wo = self.w[key]
+            self.w[key] = wo.T
+            try:
+                return super().block(layer, x, positions, cache)
+            finally:
+                self.w[key] = wo
+
+    def fwd(w):
+        dec = Planted(cfg, w)
+        ph, ac = synth.make_prompt(11, 6, 14, cfg.phone_vocab)
+        return dec.forward(np.concatenate([ph, ac]), np.arange(20) < 6, dec.new_cache())
+
+    perm = np.array([2, 0, 3, 1])
+    assert not np.allclose(fwd(_permute_heads(cfg, tiny_weights, perm)), fwd(tiny_weights), atol=1e-3)
