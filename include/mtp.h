@@ -134,7 +134,7 @@ MTP_API int mtp_prefill(mtp_ctx* ctx, int seq_slot, const int32_t* phonemes, int
                         const int32_t* acoustic, int n_ac, int max_new_tokens);
 
 /* Return the slot's pages to the pool and mark it inactive. */
-MTP_API int mtp_release(mtp_ctx* ctx, int seq_slot);
+MTP_API int mtp_release(mtp_ctx* ctx, int seq_slot);  /* Errors: MTP_ERR_INVALID (slot), MTP_ERR_CUDA. */
 
 /* One decode step for every active, unfinished slot (Fig. 1 caption,
  * Sec. III-B/C): feed the tokens accepted by the previous step (appending
@@ -156,31 +156,37 @@ MTP_API int mtp_decode_step(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_t
  * ceil(remaining / n) steps with one state read between rounds).  out_tokens (host or device, may be NULL)
  * receives each slot's generated tokens in row b at stride `out_stride`
  * (>= the slot's max_new_tokens); out_lens (may be NULL) their counts.
- * Returns the number of steps run (>= 0) or an error. */
+ * Steps run as CUDA graphs of eight chained steps where possible.
+ * Returns the number of steps run (>= 0) or an error: MTP_ERR_INVALID
+ * (n_heads, top_k, out_stride), MTP_ERR_CUDA, MTP_ERR_DEVICE. */
 MTP_API int mtp_generate(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_tokens,
                          int out_stride, int32_t* out_lens);
 
 /* Remove the last `n_tokens` cached positions of a slot (rejected tokens).
- * The pages stay reserved for the slot and are reused by later appends. */
+ * The pages stay reserved for the slot and are reused by later appends.
+ * Errors: MTP_ERR_INVALID (slot, n_tokens < 0 or > the cached length), MTP_ERR_CUDA. */
 MTP_API int mtp_rollback(mtp_ctx* ctx, int seq_slot, int n_tokens);
 
 /* Replace the tokens the next step feeds for a slot (teacher forcing for
- * parity tests): `tokens` (host, int32) of length 1..n_heads_max. */
+ * parity tests): `tokens` (host, int32) of length 1..n_heads_max.
+ * Errors: MTP_ERR_INVALID (slot, n, ids out of range), MTP_ERR_CUDA. */
 MTP_API int mtp_set_teacher_tokens(mtp_ctx* ctx, int seq_slot, const int32_t* tokens, int n);
 
 /* Slot state (host int32[6]): cached length, tokens pending to be fed,
- * remaining budget, done flag, active flag, tokens generated so far. */
+ * remaining budget, done flag, active flag, tokens generated so far.
+ * Errors: MTP_ERR_INVALID (slot, null), MTP_ERR_CUDA. */
 MTP_API int mtp_seq_state(mtp_ctx* ctx, int seq_slot, int32_t* out6);
 
 /* Logits and log-sum-exp of the last decode step (host or device):
  * out_logits float [max_batch][n_heads][codec_vocab] and out_lse float
  * [max_batch][n_heads] (either may be NULL), for the n_heads of that step.
- * The kernels rank candidates by logp = logits - lse rounded to fp32. */
+ * The kernels rank candidates by logp = logits - lse rounded to fp32.
+ * Errors: MTP_ERR_INVALID (no step run yet), MTP_ERR_CUDA. */
 MTP_API int mtp_debug_logits(mtp_ctx* ctx, float* out_logits, float* out_lse);
 
 /* Candidate lattice and selected path of the last decode step (host or
  * device, may be NULL): out_ids int32 and out_logp float [max_batch][n][k],
- * out_path int32 [max_batch][n]. */
+ * out_path int32 [max_batch][n].  Errors: MTP_ERR_INVALID (no step run yet), MTP_ERR_CUDA. */
 MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, int32_t* out_path);
 
 /* Options:
