@@ -512,6 +512,20 @@ def run_ours(args):
     tr = mtp.mtp_trace_step(ctx, N_HEADS, TOP_K)
     spans = [(r[3] - r[2]) / 1e3 for r in tr if KERNEL_KINDS[int(r[0])] == dom and r[3] > r[2]]
     pipelined_us = statistics.mean(spans) if spans else None
+    # the traced step by kernel kind: launches, mean time from the last CTA past the dependency wait
+    # to the last CTA's end, and mean time from the previous launch's end to this one's wait
+    timeline = {}
+    for i, r in enumerate(tr):
+        kind = KERNEL_KINDS[int(r[0])]
+        t = timeline.setdefault(kind, {"launches": 0, "post_wait_us": 0.0, "gap_us": 0.0})
+        t["launches"] += 1
+        t["post_wait_us"] += max(0, int(r[3]) - int(r[2])) / 1e3
+        if i > 0:
+            t["gap_us"] += max(0, int(r[2]) - int(tr[i - 1][3])) / 1e3
+    for t in timeline.values():
+        t["post_wait_us"] /= t["launches"]
+        t["gap_us"] /= t["launches"]
+    step_span_us = (int(tr[-1][3]) - int(tr[0][1])) / 1e3 if len(tr) else None
     roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic, "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": kb[dom], "avg_launch_us": per_launch_ms * 1e3,
@@ -535,7 +549,9 @@ def run_ours(args):
             "prefill_ms": prefill_ms, "decode_ms": decode_ms,
             "decode_tokens_per_s": GEN / (decode_ms / 1e3),
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
-            "clocks": clk.summary(), "kernel_ms": {k: v[0] for k, v in prof.items()}}
+            "clocks": clk.summary(), "kernel_ms": {k: v[0] for k, v in prof.items()},
+            "step_timeline": {"span_us": step_span_us, "kinds": timeline,
+                              "timing": "one graph-launched decode step, %globaltimer (mtp_trace_step)"}}
     if not args.no_c5:
         line["c5"] = run_c5(mtp, ctx, stream)
     dec.close()
