@@ -20,7 +20,11 @@ future keys have no effect); the block with zeroed weights is the identity
 plus biases; a one-token block against its closed form; cached chunked decode
 against a cache-free full recompute; invariance to permutations of the
 attention heads, of the FFN units and of the dimensions within a head (which
-a transposed operand or a wrong head layout breaks).  Beyond these, the composition of the
+a transposed operand or a wrong head layout breaks); with every block matrix
+and bias zero the decoder returns tok_phone[id] + PE(p) on the phoneme span
+and tok_codec[id] + PE(p) on the codec span, the sinusoid written out in
+scalar form (tests/test_oracle_heads_embed.py; swapped or shared tables
+rejected).  Beyond these, the composition of the
 block is "parity unpinned" against any printed value: the paper prints no
 activation, logit or worked example of the model.
 """

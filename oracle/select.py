@@ -33,7 +33,10 @@ Parity pins (tests/test_oracle_select.py): brute-force enumeration of all
 k^n paths, scored left to right with the same float32 adds (bit-exact), hand-worked lattices
 in tests/golden/, k = 1 and uniform-Q reductions to per-head argmax, the
 sticky-diagonal case, sum(exp(logp)) = 1, shift invariance, and top-k against
-a stable lexicographic sort.
+a stable lexicographic sort.  head_logits (tests/test_oracle_heads_embed.py):
+the closed form of LN_f on an alternating hidden state through heads whose
+rows select one coordinate each, with planted mistakes (LN_f or its affine
+part skipped, head i reading head i + 1, bias dropped) rejected.
 """
 from __future__ import annotations
 
