@@ -107,15 +107,19 @@ typedef struct mtp_config {
 
 typedef struct mtp_ctx mtp_ctx;
 
-/* Create a context on the current CUDA device: validates config and blob,
- * copies the weights to the device (the caller keeps the blob), allocates
- * the KV page pool and all step buffers.  `cuda_stream` is a cudaStream_t
+/* Create a context on the current CUDA device for the model of Sec. III-A
+ * (the AR decoder theta_AR of Eq. 1) with the n MTP heads of Sec. III-B and
+ * the transition matrix Q of Sec. III-C: validates config and blob, copies
+ * the weights to the device (the caller keeps the blob), allocates the KV
+ * page pool and all step buffers.  `cuda_stream` is a cudaStream_t
  * (NULL = legacy default stream) used by every later call on the context.
  * Errors: MTP_ERR_INVALID (config), MTP_ERR_WEIGHTS (blob), MTP_ERR_CUDA. */
 MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_t blob_bytes,
                        void* cuda_stream, mtp_ctx** out);
 
-/* Free every device resource of the context (NULL is ignored). */
+/* Free every device resource of the context made by mtp_create (the model of
+ * Sec. III-A/B/C and its KV cache); NULL is ignored.  Synchronises the
+ * context's stream first. */
 MTP_API void mtp_destroy(mtp_ctx* ctx);
 
 /* Message of the last failed call on this thread ("" if none). */
@@ -162,13 +166,19 @@ MTP_API int mtp_decode_step(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_t
 MTP_API int mtp_generate(mtp_ctx* ctx, int n_heads, int top_k, int32_t* out_tokens,
                          int out_stride, int32_t* out_lens);
 
-/* Remove the last `n_tokens` cached positions of a slot (rejected tokens).
- * The pages stay reserved for the slot and are reused by later appends.
+/* Remove the last `n_tokens` cached positions of a slot: the rejected
+ * tokens of a step, whose keys/values were appended when they were fed but
+ * which the selection did not accept (the speculative-decoding framing of
+ * Sec. I-II and the acceptance of Sec. III-C; MTP_VERIFY_GREEDY rolls back
+ * on the device in the same way).  The pages stay reserved for the slot and
+ * are reused by later appends.
  * Errors: MTP_ERR_INVALID (slot, n_tokens < 0 or > the cached length), MTP_ERR_CUDA. */
 MTP_API int mtp_rollback(mtp_ctx* ctx, int seq_slot, int n_tokens);
 
-/* Replace the tokens the next step feeds for a slot (teacher forcing for
- * parity tests): `tokens` (host, int32) of length 1..n_heads_max.
+/* Replace the tokens the next step feeds for a slot: the codec tokens that
+ * extend the concatenated sequence of Sec. III-A (teacher forcing, for parity
+ * tests; under MTP_VERIFY_GREEDY tokens[0] is the confirmed token and the
+ * rest the drafts).  `tokens` (host, int32) of length 1..n_heads_max.
  * Errors: MTP_ERR_INVALID (slot, n, ids out of range), MTP_ERR_CUDA. */
 MTP_API int mtp_set_teacher_tokens(mtp_ctx* ctx, int seq_slot, const int32_t* tokens, int n);
 
@@ -344,10 +354,12 @@ MTP_API int mtp_attention(const mtp_attention_args* args, void* workspace, size_
  * MTP_ATTENTION_NOALLOC_SCRATCH_BYTES per GPU, held from library load until
  * process exit and shared by every call on that GPU.  A call whose scratch
  * need (mtp_attention_workspace_bytes) exceeds it fails with MTP_ERR_INVALID
- * before launching anything.  The first call on a device looks up the
- * array's device address; make that first call before any stream capture.
- * Each call clears the merge counters it uses (an asynchronous memset on the
- * stream); the partial results keep the last call's contents.  Calls that
+ * before launching anything, as does any invalid argument: nothing is queued
+ * then.  Every call looks up the array's device address (which allocates
+ * nothing); the first call on a device may also load the library's device
+ * code, so make that first call before any stream capture.  Each call clears
+ * the merge counters it uses (an asynchronous memset on the stream); the
+ * partial results keep the last call's contents.  Calls that
  * overlap on the GPU (other streams or threads) race on the array: order
  * them on one stream.  Arguments, outputs and errors as mtp_attention.  No
  * cudaMalloc, cudaFree or allocating library call is made. */

@@ -20,7 +20,6 @@
 #include <math.h>
 
 #include <cstdio>
-#include <mutex>
 
 #include "common.cuh"
 #include "kernels.cuh"
@@ -480,13 +479,9 @@ cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool
     if (a.rows_per_group < 1 || a.rows_per_group > RPG || half_keys(a.page_size) % a.page_size != 0 ||
         a.n_splits < 1)
         return cudaErrorInvalidValue;
-    static size_t configured = 0;
     const size_t smem = attn_smem_bytes(a.page_size);
-    if (configured < smem) {
-        cudaError_t e = cudaFuncSetAttribute(attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = smem;
-    }
+    cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(attn_kernel), smem);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.n_splits, a.n_heads, groups);
     cfg.blockDim = dim3(ATT_THREADS);
@@ -510,62 +505,30 @@ cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool
 // held until the process exits and shared by every call on that GPU.
 static __device__ __align__(256) unsigned char g_attention_scratch[MTP_ATTENTION_NOALLOC_SCRATCH_BYTES];
 
-namespace {
-
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device.  The array's
-// name is only a host-side stand-in, so the address is looked up once per
-// device (with that device current) and remembered.
-int scratch_address(void** out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices) return mtp::report_error(MTP_ERR_INVALID, "device index out of range");
-    std::lock_guard<std::mutex> lock(g_scratch_mutex);
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_attention_scratch);
-        if (e != cudaSuccess || !p) {
-            char msg[256];
-            std::snprintf(msg, sizeof(msg), "attention scratch address lookup failed: %s", cudaGetErrorString(e));
-            return mtp::report_error(MTP_ERR_CUDA, msg);
-        }
-        g_scratch_addr[dev] = p;
-    }
-    *out = g_scratch_addr[dev];
-    return MTP_OK;
-}
-
-}  // namespace
-
 extern "C" MTP_API int mtp_attention_noalloc(const mtp_attention_args* args, void* cuda_stream) {
     mtp::clear_error();
-    if (!args) return mtp::report_error(MTP_ERR_INVALID, "attention: null arguments");
-    const size_t need = mtp_attention_workspace_bytes(args);
-    if (need == 0) return mtp::report_error(MTP_ERR_INVALID, "attention: invalid sizes");
-    if (need > MTP_ATTENTION_NOALLOC_SCRATCH_BYTES) {
+    mtp::AttnStandalonePlan p;
+    const int r = mtp::attention_standalone_plan(args, true, &p);  // checked before anything is queued
+    if (r != MTP_OK) return r;
+    if (p.need > MTP_ATTENTION_NOALLOC_SCRATCH_BYTES) {
         char msg[256];
         std::snprintf(msg, sizeof(msg),
-                      "attention: this call needs %zu bytes of scratch, the fixed scratch array holds %u", need,
+                      "attention: this call needs %zu bytes of scratch, the fixed scratch array holds %u", p.need,
                       (unsigned)MTP_ATTENTION_NOALLOC_SCRATCH_BYTES);
         return mtp::report_error(MTP_ERR_INVALID, msg);
     }
+    // The array's name is only a host-side stand-in for it; its device address
+    // is looked up on every call (no allocation), so it stays right after the
+    // context of the device is torn down and made again.
     void* scratch = nullptr;
-    const int r = scratch_address(&scratch);
-    if (r != MTP_OK) return r;
-    // the merge counters follow the 256-byte-aligned partials and must start at zero
-    int dev = 0, sms = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaError_t e = cudaGetSymbolAddress(&scratch, g_attention_scratch);
+    if (e != cudaSuccess || !scratch) {
+        char msg[256];
+        std::snprintf(msg, sizeof(msg), "attention scratch address lookup failed: %s", cudaGetErrorString(e));
+        return mtp::report_error(MTP_ERR_CUDA, msg);
+    }
+    const cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+    e = cudaMemsetAsync(static_cast<char*>(scratch) + p.part_bytes, 0, p.count_bytes, s);  // merge counters
     if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
-    const int groups = (args->rows + args->rows_per_group - 1) / args->rows_per_group;
-    const int splits = mtp::attn_splits_for(groups, args->n_heads, args->page_size, args->max_keys, sms);
-    const size_t part = (mtp::attn_workspace_floats(groups, args->n_heads, splits, args->rows_per_group) * 4 + 255) &
-                        ~(size_t)255;
-    e = cudaMemsetAsync(static_cast<char*>(scratch) + part, 0, need - part, static_cast<cudaStream_t>(cuda_stream));
-    if (e != cudaSuccess) return mtp::report_error(MTP_ERR_CUDA, cudaGetErrorString(e));
-    return mtp_attention(args, scratch, MTP_ATTENTION_NOALLOC_SCRATCH_BYTES, cuda_stream);
+    return mtp::attention_standalone_launch(args, p, scratch, s);
 }

@@ -313,12 +313,8 @@ __global__ void __launch_bounds__(WARPS * 32, 2) gemv_kernel(const GemvArgs a) {
 template <typename WT, int MT, int WARPS, int NSUB, int EPI, bool LN>
 cudaError_t launch_one(const GemvArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl) {
     auto kern = gemv_kernel<WT, MT, WARPS, NSUB, EPI, LN>;
-    static bool configured = false;  // one attribute call per instantiation
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(kern), 200 * 1024);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(WARPS * 32);

@@ -11,6 +11,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+struct mtp_attention_args;  // include/mtp.h
+
 namespace mtp {
 
 constexpr int HEAD_DIM = 64;     // attention head width (fixed by the kernels)
@@ -255,6 +257,28 @@ int tc_encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t ro
                  bool pre_swizzled);
 int tc_tile_rows(int m);          // activation rows per tile for m rows: 32, 64 or 128
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl);
+
+// Raise `kernel`'s dynamic shared-memory limit to at least `bytes` on the
+// current device (and, with max_shared_carveout, prefer the whole unified L1
+// as shared memory).  The attribute is per device: the call is made once per
+// (kernel, device, size) and is safe from several threads.
+cudaError_t ensure_kernel_smem(const void* kernel, size_t bytes, bool max_shared_carveout = false);
+
+// The stand-alone attention operator (mtp_attention*): its arguments checked
+// and its workspace laid out once, for every entry point that runs it.  The
+// workspace holds the split partials (part_bytes, a multiple of 256) and then
+// the per-(group, head) merge counters (count_bytes), which must be zero when
+// a launch starts and are left zero by it.
+struct AttnStandalonePlan {
+    int groups, splits;
+    size_t part_bytes, count_bytes, need;
+};
+// MTP_OK or MTP_ERR_INVALID / MTP_ERR_CUDA (message set); with check_pointers
+// the device pointers must be non-null too.
+int attention_standalone_plan(const struct ::mtp_attention_args* a, bool check_pointers, AttnStandalonePlan* p);
+// Enqueue the kernel on `stream` with `workspace` laid out as `p` describes.
+int attention_standalone_launch(const struct ::mtp_attention_args* a, const AttnStandalonePlan& p, void* workspace,
+                                cudaStream_t stream);
 
 // C-ABI error reporting shared by the translation units (message for mtp_last_error)
 int report_error(int code, const char* msg);

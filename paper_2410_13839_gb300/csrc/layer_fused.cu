@@ -1218,25 +1218,18 @@ __global__ void __launch_bounds__(NTHREADS, 2) mlp_kernel(const LayerArgs a) {
     cluster_wait();            // peers may still read this CTA's shared memory
 }
 
+// the whole unified L1 as shared memory, so CTAs of the two block kernels can share an SM
 template <typename T>
 cudaError_t set_smem(T kern, size_t bytes) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-    if (e != cudaSuccess) return e;
-    // the whole unified L1 as shared memory, so CTAs of the two block kernels can share an SM
-    return cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                (int)cudaSharedmemCarveoutMaxShared);
+    return ensure_kernel_smem(reinterpret_cast<const void*>(kern), bytes, true);
 }
 
 template <typename WT, int MT>
 cudaError_t launch_attn_block_t(const LayerArgs& a, cudaStream_t s, bool pdl) {
     const ALayout L(a.d, sizeof(WT), MT, a.page_size);
     auto kern = attn_block_kernel<WT, MT>;
-    static size_t configured = 0;
-    if (configured < L.total) {
-        cudaError_t e = set_smem(kern, L.total);
-        if (e != cudaSuccess) return e;
-        configured = L.total;
-    }
+    cudaError_t e = set_smem(kern, L.total);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(CA, a.n_heads);
     cfg.blockDim = dim3(NTHREADS);
@@ -1254,12 +1247,8 @@ template <typename WT, int MT>
 cudaError_t launch_mlp_t(const LayerArgs& a, int grid, cudaStream_t s, bool pdl) {
     const BLayout L(a.d, a.ffn_rows_per_cta, sizeof(WT), MT, MLP_CLUSTER);
     auto kern = mlp_kernel<WT, MT, MLP_CLUSTER>;
-    static size_t configured = 0;
-    if (configured < L.total) {
-        cudaError_t e = set_smem(kern, L.total);
-        if (e != cudaSuccess) return e;
-        configured = L.total;
-    }
+    cudaError_t e = set_smem(kern, L.total);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(NTHREADS);

@@ -17,6 +17,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <tuple>
 #include <string>
 #include <utility>
@@ -43,6 +44,23 @@ int fail(int code, const char* fmt, ...) {
 }
 
 }  // namespace
+
+cudaError_t mtp::ensure_kernel_smem(const void* kernel, size_t bytes, bool max_shared_carveout) {
+    static std::mutex mu;
+    static std::map<std::pair<const void*, int>, size_t> done;  // (kernel, device) -> configured bytes
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    size_t& have = done[{kernel, dev}];
+    if (have >= bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess && max_shared_carveout)
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
+    if (e == cudaSuccess) have = bytes;
+    return e;
+}
 
 // error reporting for C-ABI functions defined in other translation units
 int mtp::report_error(int code, const char* msg) {
@@ -885,6 +903,45 @@ void destroy(mtp_ctx* c) {
 
 }  // namespace
 
+int mtp::attention_standalone_plan(const mtp_attention_args* a, bool check_pointers, AttnStandalonePlan* p) {
+    if (!a || a->rows < 1 || a->rows_per_group < 1 || a->rows_per_group > MAX_ROWS || a->n_heads < 1 ||
+        (a->page_size != 16 && a->page_size != 32 && a->page_size != 64 && a->page_size != 128) || a->layers < 1 ||
+        a->layer < 0 || a->layer >= a->layers || a->bt_stride < 1 || a->max_keys < 1)
+        return fail(MTP_ERR_INVALID, "attention: invalid sizes");
+    if (check_pointers && (!a->q || !a->kv_pool || !a->block_table || !a->row_seq || !a->row_pos || !a->out))
+        return fail(MTP_ERR_INVALID, "attention: null pointer");
+    int dev = 0, sms = 0;
+    CUDA_TRY(cudaGetDevice(&dev));
+    CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    p->groups = (a->rows + a->rows_per_group - 1) / a->rows_per_group;
+    p->splits = attn_splits_for(p->groups, a->n_heads, a->page_size, a->max_keys, sms);
+    p->part_bytes = align256(attn_workspace_floats(p->groups, a->n_heads, p->splits, a->rows_per_group) * sizeof(float));
+    p->count_bytes = align256((size_t)p->groups * a->n_heads * sizeof(int));
+    p->need = p->part_bytes + p->count_bytes;
+    return MTP_OK;
+}
+
+int mtp::attention_standalone_launch(const mtp_attention_args* a, const AttnStandalonePlan& p, void* workspace,
+                                     cudaStream_t stream) {
+    AttnArgs at;
+    std::memset(&at, 0, sizeof(at));
+    const int d = a->n_heads * HEAD_DIM;
+    at.q = a->q; at.ldq = d;
+    at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(a->kv_pool);
+    at.page_elems = (long long)a->layers * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.layer_off = (long long)a->layer * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.block_table = a->block_table; at.bt_stride = a->bt_stride;
+    at.row_seq = a->row_seq; at.row_pos = a->row_pos;
+    at.out = a->out; at.ldo = d;
+    at.ws_part = static_cast<float*>(workspace);
+    at.ws_count = reinterpret_cast<int*>(static_cast<char*>(workspace) + p.part_bytes);
+    at.rows_per_group = a->rows_per_group; at.n_heads = a->n_heads; at.page_size = a->page_size;
+    at.n_splits = p.splits; at.plan = PLAN_ROWS;
+    at.err = nullptr;
+    CUDA_TRY(launch_attention(at, p.groups, stream, false));
+    return MTP_OK;
+}
+
 // ================================================================ C ABI ====
 
 extern "C" {
@@ -1409,53 +1466,21 @@ MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden
 }
 
 MTP_API size_t mtp_attention_workspace_bytes(const mtp_attention_args* a) {
-    if (!a || a->rows < 1 || a->rows_per_group < 1 || a->n_heads < 1 || a->page_size < 1) return 0;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) {
-        cudaGetLastError();
-        return 0;
-    }
-    const int groups = (a->rows + a->rows_per_group - 1) / a->rows_per_group;
-    const int S = attn_splits_for(groups, a->n_heads, a->page_size, a->max_keys, sms);
-    return align256(attn_workspace_floats(groups, a->n_heads, S, a->rows_per_group) * sizeof(float)) +
-           align256((size_t)groups * a->n_heads * sizeof(int));
+    AttnStandalonePlan p;
+    const std::string keep = g_err;  // a size query leaves the last error alone
+    const int r = attention_standalone_plan(a, false, &p);
+    g_err = keep;
+    return r == MTP_OK ? p.need : 0;
 }
 
 MTP_API int mtp_attention(const mtp_attention_args* a, void* workspace, size_t workspace_bytes, void* cuda_stream) {
     g_err.clear();
-    if (!a || a->rows < 1 || a->rows_per_group < 1 || a->rows_per_group > MAX_ROWS || a->n_heads < 1 ||
-        (a->page_size != 16 && a->page_size != 32 && a->page_size != 64 && a->page_size != 128) || a->layers < 1 ||
-        a->layer < 0 || a->layer >= a->layers || a->bt_stride < 1 || a->max_keys < 1)
-        return fail(MTP_ERR_INVALID, "attention: invalid sizes");
-    if (!a->q || !a->kv_pool || !a->block_table || !a->row_seq || !a->row_pos || !a->out || !workspace)
-        return fail(MTP_ERR_INVALID, "attention: null pointer");
-    const size_t need = mtp_attention_workspace_bytes(a);
-    if (need == 0 || workspace_bytes < need)
-        return fail(MTP_ERR_INVALID, "attention: workspace %zu bytes, need %zu", workspace_bytes, need);
-    int dev = 0, sms = 0;
-    CUDA_TRY(cudaGetDevice(&dev));
-    CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    const int groups = (a->rows + a->rows_per_group - 1) / a->rows_per_group;
-    const int S = attn_splits_for(groups, a->n_heads, a->page_size, a->max_keys, sms);
-    AttnArgs at;
-    std::memset(&at, 0, sizeof(at));
-    const int d = a->n_heads * HEAD_DIM;
-    at.q = a->q; at.ldq = d;
-    at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(a->kv_pool);
-    at.page_elems = (long long)a->layers * 2 * a->n_heads * a->page_size * HEAD_DIM;
-    at.layer_off = (long long)a->layer * 2 * a->n_heads * a->page_size * HEAD_DIM;
-    at.block_table = a->block_table; at.bt_stride = a->bt_stride;
-    at.row_seq = a->row_seq; at.row_pos = a->row_pos;
-    at.out = a->out; at.ldo = d;
-    at.ws_part = static_cast<float*>(workspace);
-    at.ws_count = reinterpret_cast<int*>(static_cast<char*>(workspace) +
-                                         align256(attn_workspace_floats(groups, a->n_heads, S, a->rows_per_group) *
-                                                  sizeof(float)));
-    at.rows_per_group = a->rows_per_group; at.n_heads = a->n_heads; at.page_size = a->page_size;
-    at.n_splits = S; at.plan = PLAN_ROWS;
-    at.err = nullptr;
-    CUDA_TRY(launch_attention(at, groups, static_cast<cudaStream_t>(cuda_stream), false));
-    return MTP_OK;
+    AttnStandalonePlan p;
+    MTP_TRY(attention_standalone_plan(a, true, &p));
+    if (!workspace) return fail(MTP_ERR_INVALID, "attention: null workspace");
+    if (workspace_bytes < p.need)
+        return fail(MTP_ERR_INVALID, "attention: workspace %zu bytes, need %zu", workspace_bytes, p.need);
+    return attention_standalone_launch(a, p, workspace, static_cast<cudaStream_t>(cuda_stream));
 }
 
 }  // extern "C"

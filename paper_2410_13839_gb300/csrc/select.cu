@@ -547,13 +547,9 @@ cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s) {
     if (a.n < 1 || a.n > MAX_NHEADS || a.k < 1 || a.k > MAX_TOPK || a.batch < 0) return cudaErrorInvalidValue;
     if (a.batch == 0) return cudaSuccess;
     const size_t smem = (size_t)VIT_WARPS * (a.n - 1) * a.k * a.k * sizeof(float);
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(viterbi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             VIT_WARPS * (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK * (int)sizeof(float));
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(viterbi_kernel),
+                                       (size_t)VIT_WARPS * (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK * sizeof(float));
+    if (e != cudaSuccess) return e;
     viterbi_kernel<<<(a.batch + VIT_WARPS - 1) / VIT_WARPS, VIT_WARPS * 32, smem, s>>>(a);
     return cudaGetLastError();
 }

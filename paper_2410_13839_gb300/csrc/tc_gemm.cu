@@ -339,13 +339,10 @@ size_t tc_smem() {
 }
 
 template <int NT, typename K>
-cudaError_t launch_kern(K kern, size_t& configured, const TcGemm& g, cudaStream_t s, bool pdl) {
+cudaError_t launch_kern(K kern, const TcGemm& g, cudaStream_t s, bool pdl) {
     const size_t smem = tc_smem<NT>();
-    if (configured < smem) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = smem;
-    }
+    cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(kern), smem);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.n_w / TC_M, g.splits, (g.args.m + NT - 1) / NT);
     cfg.blockDim = dim3(TC_THREADS);
@@ -361,9 +358,8 @@ cudaError_t launch_kern(K kern, size_t& configured, const TcGemm& g, cudaStream_
 
 template <int NT>
 cudaError_t launch_nt(const TcGemm& g, cudaStream_t s, bool pdl) {
-    static size_t configured[2] = {0, 0};
-    if (g.args.n_valid) return launch_kern<NT>(tc_gemm_kernel<NT, true>, configured[1], g, s, pdl);
-    return launch_kern<NT>(tc_gemm_kernel<NT, false>, configured[0], g, s, pdl);
+    if (g.args.n_valid) return launch_kern<NT>(tc_gemm_kernel<NT, true>, g, s, pdl);
+    return launch_kern<NT>(tc_gemm_kernel<NT, false>, g, s, pdl);
 }
 
 }  // namespace
