@@ -152,13 +152,15 @@ def clear_prefix(margins):
     return low[0] if low else len(margins)
 
 
-def _run_verify(model, batch, n, k, budget, seed0, batched=1):
+def _run_verify(model, batch, n, k, budget, seed0, batched=1, options=()):
     mtp = lib_module()
     prompts = _prompts(model, batch, seed0)
     max_ctx = max(len(p) + len(a) for p, a in prompts) + budget + model.n_heads_max + 4
     dec, w = decoder(model, max_batch=batch, max_ctx=max_ctx, accept_policy=1)
     try:
         mtp.mtp_set_option(dec.ctx, 4, batched)
+        for opt, val in options:
+            mtp.mtp_set_option(dec.ctx, opt, val)
         for b, (ph, ac) in enumerate(prompts):
             dec.prefill(b, ph, ac, budget)
         out, steps = dec.generate(n, k, budget)
