@@ -81,6 +81,9 @@ def _kernel_bytes(d, F, V, L, n, wb, ctx_keys, fed):
         "attn_block": (4 * d * d) * wb + (3 * d + d + 2 * d) * 4 + ctx_keys * d * 2 * 2 + fed * d * 2 * 2,
         "mlp": 2 * F * d * wb + (F + d + 2 * d) * 4,
         "heads": n * V * d * wb + n * V * 4 + 2 * d * 4,
+        # the persistent kernel: the fed rows' embedding and all L blocks of one pass
+        "step": L * ((4 * d * d + 2 * F * d) * wb + (3 * d + d + F + d + 4 * d) * 4
+                     + ctx_keys * d * 2 * 2 + fed * d * 2 * 2) + fed * d * (wb + 4),
     }
 
 
@@ -538,9 +541,11 @@ def run_ours(args):
                  "frac": dec_bytes / (decode_ms / 1e3) / 1e9 / peak,
                  "frac_of_nominal_8tbs": dec_bytes / (decode_ms / 1e3) / 1e9 / 8000.0}
     # prefill: two slot updates, then per 128-position chunk the embedding, 8 batched-path kernels per
-    # layer and the last-row save; decode: embedding, 2 block kernels per layer, heads, selection
+    # layer and the last-row save; decode: the persistent step kernel (or the embedding and 2 block
+    # kernels per layer), heads, selection
+    per_decode_step = 3 if mtp.mtp_get_option(ctx, 9) else 3 + 2 * L
     launches_per_step = (2 + ((N_PH + N_AC + 127) // 128) * (2 + 8 * L)
-                         + decode_steps // args.steps * (3 + 2 * L))
+                         + decode_steps // args.steps * per_decode_step)
 
     line = {"metric": METRIC, "value": value, "unit": "codec tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",

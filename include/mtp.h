@@ -219,6 +219,11 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        (the top-k sampling that keeps diversity, Fig. 2 caption), by forward
  *                        filtering and backward sampling in fp32.  Under MTP_VERIFY_GREEDY only
  *                        the drafts are drawn; the output stays greedy.
+ *   MTP_OPT_PERSISTENT   1 = a pass of <= 8 fed rows with bf16 weights runs its embedding and all
+ *                        blocks as one persistent kernel (one CTA per SM in clusters of 4, weights
+ *                        and cached keys streamed into shared-memory rings ahead of use, bounded grid
+ *                        barriers between the attention and MLP phases), where the model and GPU
+ *                        allow it; 0 = two block kernels per layer (default: faster on GB300 at B = 1)
  *   MTP_OPT_SEED         seed of the path draws (any 32-bit value, zero-extended; default 0).
  *                        Position t of a draw of slot b that has generated g tokens uses the
  *                        uniform (SplitMix64(x) >> 40) / 2^24, x = ((seed * P + b) * P + g) * P + t
@@ -226,7 +231,8 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        option recaptures the step graphs. */
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
-    MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8
+    MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8,
+    MTP_OPT_PERSISTENT = 9
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
@@ -242,10 +248,17 @@ MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
  *   PACK        LN / copy / GELU of the rows into bf16 hi + lo GEMM operands
  *   GEMM        a tensor-core projection (q|k|v, W_o, W1 or W2)
  *   QKV         query rows out, keys and values appended to the cache
- *   ATTN        split-KV attention of the fed rows over the cache */
+ *   ATTN        split-KV attention of the fed rows over the cache
+ * and of the persistent path (bf16 weights, <= 8 fed rows per pass):
+ *   STEP        one persistent kernel: the fed rows' embedding and every block
+ *   STEP_ATTN   (trace only) one attention phase of a layer inside STEP
+ *   STEP_MLP    (trace only) one MLP phase of a layer inside STEP
+ *   STEP_CTA    (trace only) one CTA's attention or MLP phase of the middle layer */
 typedef enum mtp_kernel_kind {
     MTP_K_EMBED = 0, MTP_K_ATTN_BLOCK = 1, MTP_K_MLP = 2, MTP_K_HEADS = 3, MTP_K_SELECT = 4,
-    MTP_K_SAVE = 5, MTP_K_PACK = 6, MTP_K_GEMM = 7, MTP_K_QKV = 8, MTP_K_ATTN = 9, MTP_K_COUNT = 10
+    MTP_K_SAVE = 5, MTP_K_PACK = 6, MTP_K_GEMM = 7, MTP_K_QKV = 8, MTP_K_ATTN = 9, MTP_K_STEP = 10,
+    MTP_K_STEP_ATTN = 11, MTP_K_STEP_MLP = 12,
+    MTP_K_STEP_CTA = 13, MTP_K_COUNT = 14
 } mtp_kernel_kind;
 
 /* Run one decode step with each kernel launched alone (no graph, no PDL)
@@ -260,7 +273,11 @@ MTP_API int mtp_profile_step(mtp_ctx* ctx, int n_heads, int top_k, float* out_ms
  * record per kernel launch: out int64 [cap][MTP_TRACE_COLS] rows of
  * {mtp_kernel_kind, earliest CTA start, latest CTA past its dependency wait,
  * latest CTA end, then 8 phase marks (latest CTA past each, 0 if unused)},
- * times in ns of the GPU's global timer.  Returns the number of launches
+ * times in ns of the GPU's global timer.  A STEP launch is followed by one
+ * row per phase of each layer (STEP_ATTN, STEP_MLP): earliest CTA start of the
+ * phase, latest CTA start, latest CTA end, marks; then two rows per CTA
+ * (STEP_CTA, attention then MLP phase of the middle layer): that CTA's start,
+ * its index, its end and marks.  Returns the number of launches
  * recorded (<= cap).  The step's effect on the slots is that of
  * mtp_decode_step. */
 #define MTP_TRACE_COLS 12

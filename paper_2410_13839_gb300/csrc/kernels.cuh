@@ -126,6 +126,52 @@ cudaError_t launch_mlp(const LayerArgs& a, bool w_bf16, int grid, cudaStream_t s
 // clusters of the MLP kernel that can be resident at once (rows per CTA chosen for that count)
 cudaError_t mlp_max_clusters(int d, int num_sms, int wbytes, int d_ffn, int* clusters);
 
+// ------------------------------------------------ persistent step ----
+// The embedding and every block of one decode pass (<= MAX_ROWS fed rows,
+// bf16 weights) as one persistent kernel of clusters of SK_CLUSTER CTAs, one
+// CTA per SM, each fed by a ring of SK_STAGE_BYTES shared-memory stages
+// (step_kernel.cu).
+constexpr int SK_CLUSTER = 4;
+constexpr int SK_STAGE_BYTES = 16384;
+constexpr int SK_MAX_STAGES = 12;
+
+struct StepArgs {
+    int L, d, F, H;                  // layers, model width, FFN width, attention heads (d = 64 H)
+    int rows, rpg, seq_base, slots;  // fed rows, rows per slot (n), first slot, slots in the context
+    int n_max, page_size, codec_vocab, max_pos;
+    float ln_eps;
+    // layer 0's tensors in their device layouts; layer l's is at + l * layer_stride bytes
+    const float *ln1_g, *ln1_b, *bqkv, *bo, *ln2_g, *ln2_b, *b1, *b2;
+    const __nv_bfloat16* wqkv;       // [H][q|k|v 64 rows][d]
+    const __nv_bfloat16* wo;         // [H][d][64]
+    const __nv_bfloat16* w1;         // [F][d]
+    const __nv_bfloat16* w2t;        // [F][d] (W2 transposed)
+    long long layer_stride;
+    const __nv_bfloat16* tok_codec;  // [codec_vocab][d]
+    const float* pe;                 // [max_pos][d]
+    // slot state, read after the dependency wait
+    const int *active, *done, *n_pending, *pending, *seq_len;
+    __nv_bfloat16* kv_pool; long long page_elems;
+    const int* block_table; int bt_stride;
+    // work split and ring
+    const int2* ffn_range;           // [grid]: first FFN unit and unit count of each CTA
+    int res_cluster;                 // the cluster (one with FFN units) that adds x_mid + b2
+    int ffn_unit_rows;               // FFN rows per unit = weight rows per stage (SK_STAGE_BYTES / (2 d))
+    int ring_stages;
+    // buffers: residual rows [4][MAX_ROWS][d] (buffer 3 must be zero at entry), grid-barrier words [2]
+    float* xbuf; unsigned* bar;
+    int *row_seq, *row_pos, *row_last;  // [MAX_ROWS] plan of the pass (for the kernels after it)
+    int* err;
+    unsigned long long* trace;
+};
+// The residual buffer that holds the pass's final rows.
+inline int step_final_buffer(int layers) { return (2 * layers - 2) % 3; }
+// Ring stages that fit beside the kernel's other shared memory for mt (1, 2, 4 or 8) fed rows.
+int step_ring_stages(int d, int mt);
+// Clusters of SK_CLUSTER CTAs that can be resident at once (the 8-row footprint).
+cudaError_t step_kernel_configure(int d, int* max_clusters);
+cudaError_t launch_step_kernel(const StepArgs& a, int grid, cudaStream_t s, bool pdl);
+
 // --------------------------------------------------------------- embed ----
 struct EmbedArgs {
     int mode;                  // 0 = decode rows from slot state, 1 = prefill chunk

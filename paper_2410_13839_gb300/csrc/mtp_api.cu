@@ -162,6 +162,14 @@ struct mtp_ctx {
     std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;  // (n_heads, top_k, traced)
     std::map<std::tuple<int, int, int>, std::vector<int>> graph_kinds;
     int last_n = 0, last_k = 0;
+    // persistent step kernel (bf16 weights, passes of <= 8 fed rows)
+    bool use_persistent = false, sk_ok = false;  // measured slower than the block kernels at B = 1
+    int sk_grid = 0, sk_unit_rows = 0, sk_res_cluster = 0;
+    int sk_stages[4] = {0, 0, 0, 0};  // ring stages for passes of 1, 2, 4 and 8 rows
+    long long sk_layer_stride = 0;
+    float* d_skx = nullptr;         // residual rows [4][MAX_ROWS][d]
+    unsigned* d_skbar = nullptr;    // grid-barrier words
+    int2* d_skffn = nullptr;        // FFN units of each CTA
     // launch timeline (mtp_trace_step)
     unsigned long long* d_trace = nullptr;
     int trace_cap = 0;
@@ -388,6 +396,103 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
     return MTP_OK;
 }
 
+// The persistent step kernel: ring stages, grid (clusters resident at once),
+// and the FFN units of each CTA (one ring stage of W1 rows plus the same rows of
+// W2^T each): spread evenly over every CTA, the remainder to the CTAs without
+// attention work first.  Leaves sk_ok false where the path does not apply.
+int setup_step_kernel(mtp_ctx* c) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads;
+    if (c->wbytes != 2 || (d != 256 && d != 512 && d != 1024) || cf.layers < 2 || c->layers.size() < 2)
+        return MTP_OK;
+    const long long stride = (const char*)c->layers[1].wqkv - (const char*)c->layers[0].wqkv;
+    auto same_stride = [&](const void* p0, const void* p1) { return (const char*)p1 - (const char*)p0 == stride; };
+    const Layer &L0 = c->layers[0], &L1 = c->layers[1];
+    if (!same_stride(L0.ln1_g, L1.ln1_g) || !same_stride(L0.wo, L1.wo) || !same_stride(L0.w1, L1.w1) ||
+        !same_stride(L0.w2, L1.w2) || !same_stride(L0.b2, L1.b2) || !same_stride(L0.bqkv, L1.bqkv))
+        return MTP_OK;
+    int clusters = 0;
+    if (step_kernel_configure(d, &clusters) != cudaSuccess) {
+        cudaGetLastError();
+        return MTP_OK;
+    }
+    const int nst = step_ring_stages(d, MAX_ROWS);  // the fewest (8 rows): bounds the FFN units per CTA
+    clusters = std::min(clusters, c->num_sms / SK_CLUSTER);
+    const int rps = SK_STAGE_BYTES / (2 * d);
+    const int units = F / rps;
+    const int G = clusters * SK_CLUSTER;
+    const int max_units = std::min(64 / rps, nst - 2);
+    if (clusters < H || F % rps || units > G * max_units) return MTP_OK;
+    // every CTA takes FFN units (more CTAs, shorter chains in the MLP phase); the attention
+    // CTAs, busy in the other phase, take the remainder's smaller share
+    std::vector<int> count(G, units / G);
+    int extra = units % G;
+    for (int i = SK_CLUSTER * H; i < G && extra > 0; ++i, --extra) ++count[i];
+    for (int i = 0; i < SK_CLUSTER * H && extra > 0; ++i, --extra) ++count[i];
+    for (int i = 0; i < G; ++i)
+        if (count[i] > max_units) return MTP_OK;
+    std::vector<int2> ranges(G);
+    for (int i = 0, first = 0; i < G; ++i) {
+        ranges[i] = make_int2(first, count[i]);
+        if (first == 0 && count[i] > 0) c->sk_res_cluster = i / SK_CLUSTER;
+        first += count[i];
+    }
+    MTP_TRY(c->alloc(&c->d_skx, (size_t)4 * MAX_ROWS * d));
+    MTP_TRY(c->alloc(&c->d_skbar, 2));
+    MTP_TRY(c->alloc(&c->d_skffn, (size_t)G));
+    CUDA_TRY(cudaMemcpy(c->d_skffn, ranges.data(), G * sizeof(int2), cudaMemcpyHostToDevice));
+    c->sk_grid = G;
+    for (int i = 0; i < 4; ++i) c->sk_stages[i] = step_ring_stages(d, 1 << i);
+    c->sk_unit_rows = rps;
+    c->sk_layer_stride = stride;
+    c->sk_ok = true;
+    return MTP_OK;
+}
+
+// One pass of <= MAX_ROWS fed rows (slots seq_base .., rpg rows each) through
+// the persistent kernel; returns the buffer holding the pass's final rows.
+int launch_step_pass(mtp_ctx* c, int rows, int rpg, int seq_base, cudaStream_t s, bool pdl, Prof* prof,
+                     float** final_x) {
+    const mtp_config& cf = c->cfg;
+    const Layer& L = c->layers[0];
+    StepArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.L = cf.layers; a.d = cf.d_model; a.F = cf.d_ffn; a.H = cf.n_attn_heads;
+    a.rows = rows; a.rpg = rpg; a.seq_base = seq_base; a.slots = cf.max_batch;
+    a.n_max = cf.n_heads_max; a.page_size = cf.page_size; a.codec_vocab = cf.codec_vocab; a.max_pos = cf.max_ctx;
+    a.ln_eps = cf.ln_eps;
+    a.ln1_g = L.ln1_g; a.ln1_b = L.ln1_b; a.bqkv = L.bqkv; a.bo = L.bo;
+    a.ln2_g = L.ln2_g; a.ln2_b = L.ln2_b; a.b1 = L.b1; a.b2 = L.b2;
+    a.wqkv = static_cast<const __nv_bfloat16*>(L.wqkv);
+    a.wo = static_cast<const __nv_bfloat16*>(L.wo);
+    a.w1 = static_cast<const __nv_bfloat16*>(L.w1);
+    a.w2t = static_cast<const __nv_bfloat16*>(L.w2);
+    a.layer_stride = c->sk_layer_stride;
+    a.tok_codec = static_cast<const __nv_bfloat16*>(c->tok_codec);
+    a.pe = c->d_pe;
+    a.active = c->d_active; a.done = c->d_done; a.n_pending = c->d_npend; a.pending = c->d_pending;
+    a.seq_len = c->d_len;
+    a.kv_pool = reinterpret_cast<__nv_bfloat16*>(c->d_kv); a.page_elems = c->page_elems;
+    a.block_table = c->d_block_table; a.bt_stride = c->pages_per_seq;
+    a.ffn_range = c->d_skffn; a.ffn_unit_rows = c->sk_unit_rows; a.res_cluster = c->sk_res_cluster;
+    a.ring_stages = c->sk_stages[rows <= 1 ? 0 : rows <= 2 ? 1 : rows <= 4 ? 2 : 3];
+    a.xbuf = c->d_skx; a.bar = c->d_skbar;
+    a.row_seq = c->d_row_seq; a.row_pos = c->d_row_pos; a.row_last = c->d_row_last;
+    a.err = c->d_err;
+    a.trace = nullptr;
+    if (c->tracing && (int)c->trace_kinds.size() + 1 + 2 * cf.layers + 2 * c->sk_grid <= c->trace_cap) {
+        a.trace = tslot(c, MTP_K_STEP);  // then one record per phase, then per CTA and phase of the middle layer
+        for (int l = 0; l < cf.layers; ++l) {
+            tslot(c, MTP_K_STEP_ATTN);
+            tslot(c, MTP_K_STEP_MLP);
+        }
+        for (int i = 0; i < 2 * c->sk_grid; ++i) tslot(c, MTP_K_STEP_CTA);
+    }
+    LAUNCH(MTP_K_STEP, launch_step_kernel(a, c->sk_grid, s, pdl));
+    *final_x = c->d_skx + (size_t)step_final_buffer(cf.layers) * MAX_ROWS * cf.d_model;
+    return MTP_OK;
+}
+
 // Buffers and tensor maps of the batched path (bf16 weights only).
 int setup_batched(mtp_ctx* c) {
     const mtp_config& cf = c->cfg;
@@ -574,12 +679,17 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
     }
     for (int b0 = 0; b0 < B; b0 += spc) {
         const int G = std::min(spc, B - b0), M = G * n;
-        EmbedArgs e = embed_base(c);
-        e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
-        e.trace = tslot(c, MTP_K_EMBED);
-        // full dependency on the previous pass; the step's first pass may chain to the previous step
-        LAUNCH(MTP_K_EMBED, launch_embed(e, s, b0 == 0 && chain && pdl));
-        MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
+        if (c->use_persistent && c->sk_ok) {  // the pass's embedding and blocks in one kernel
+            // it reads nothing from earlier kernels before its dependency wait: always under programmatic launch
+            MTP_TRY(launch_step_pass(c, M, n, b0, s, pdl, prof, &final_x));
+        } else {
+            EmbedArgs e = embed_base(c);
+            e.mode = 0; e.rows = M; e.seq_base = b0; e.n_heads = n;
+            e.trace = tslot(c, MTP_K_EMBED);
+            // full dependency on the previous pass; the step's first pass may chain to the previous step
+            LAUNCH(MTP_K_EMBED, launch_embed(e, s, b0 == 0 && chain && pdl));
+            MTP_TRY(run_layers(c, M, G, n, PLAN_DEVICE, b0, 0, 0, 0, s, pdl, prof, &final_x));
+        }
         if (verify) {
             MTP_TRY(enqueue_verify(c, final_x, G, n, b0, s, pdl, prof));
         } else if (!single) {
@@ -1013,7 +1123,7 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
         (r = c->alloc(&c->d_row_seq, row_cap)) || (r = c->alloc(&c->d_row_pos, row_cap)) ||
         (r = c->alloc(&c->d_row_last, row_cap)) || (r = c->alloc(&c->d_err, 1)) || (r = c->alloc(&c->d_kept, B)) ||
-        (r = setup_batched(c)))
+        (r = setup_batched(c)) || (r = setup_step_kernel(c)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
     if (cudaMemcpy(c->d_block_table, c->h_block_table.data(), c->h_block_table.size() * sizeof(int),
@@ -1062,6 +1172,9 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
     } else if (option == MTP_OPT_SEED) {
         changed = c->sample_seed != (uint32_t)value;
         c->sample_seed = (uint32_t)value;
+    } else if (option == MTP_OPT_PERSISTENT) {
+        changed = c->use_persistent != (value != 0);
+        c->use_persistent = value != 0;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -1102,6 +1215,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_LATTICE: *value = c->lattice; break;
         case MTP_OPT_SAMPLING: *value = c->sampling; break;
         case MTP_OPT_SEED: *value = (int32_t)c->sample_seed; break;
+        case MTP_OPT_PERSISTENT: *value = c->use_persistent && c->sk_ok; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;
