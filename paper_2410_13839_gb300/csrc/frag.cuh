@@ -161,71 +161,6 @@ __device__ __forceinline__ void layer_norm_rows(RowRegs<MT>& r, int K, const flo
         for (int i = 0; i < 4; ++i) r.v[m][i] = (r.v[m][i] - stat[0][m]) * stat[1][m] * gam[i] + bet[i];
 }
 
-// layer_norm_rows with shorter dependency chains (the same statistics: per
-// warp the mean and the sum of squared deviations of its K/8 columns, merged
-// with mean = average of the warp means, M2 = sum of warp M2 + Kw * sum
-// (mean_w - mean)^2): the warp reductions of all MT rows run interleaved, and
-// every thread merges the warps' partials itself (one synchronisation instead
-// of two).  part: [2 * NWARPS][MT] scratch.
-template <int MT, class Sync = CtaSync>
-__device__ __forceinline__ void layer_norm_rows_fast(RowRegs<MT>& r, int K, const float (&gam)[4],
-                                                     const float (&bet)[4], float eps, float (*part)[MT]) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int Kw = K / NWARPS;
-    const bool valid = lane * 4 < Kw;
-    float s[MT];
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-        s[m] = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) s[m] += valid ? r.v[m][i] : 0.f;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-        for (int m = 0; m < MT; ++m) s[m] += __shfl_xor_sync(FULL_MASK, s[m], o);
-    float mw[MT], q[MT];
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-        mw[m] = s[m] / (float)Kw;
-        q[m] = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float t = r.v[m][i] - mw[m];
-            q[m] += valid ? t * t : 0.f;
-        }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-        for (int m = 0; m < MT; ++m) q[m] += __shfl_xor_sync(FULL_MASK, q[m], o);
-    if (lane < MT) {  // lane m stores row m's partials (registers indexed by a constant)
-#pragma unroll
-        for (int m = 0; m < MT; ++m)
-            if (lane == m) {
-                part[warp][m] = mw[m];
-                part[NWARPS + warp][m] = q[m];
-            }
-    }
-    Sync()();
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-        float mean = 0.f;
-#pragma unroll
-        for (int w = 0; w < NWARPS; ++w) mean += part[w][m];
-        mean /= (float)NWARPS;
-        float m2 = 0.f;
-#pragma unroll
-        for (int w = 0; w < NWARPS; ++w) {
-            const float dm = part[w][m] - mean;
-            m2 += part[NWARPS + w][m] + (float)Kw * dm * dm;
-        }
-        const float rstd = 1.0f / sqrtf(m2 / (float)K + eps);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) r.v[m][i] = (r.v[m][i] - mean) * rstd * gam[i] + bet[i];
-    }
-}
-
 // Column of element dd of key/value row t inside a cached page: the row's
 // 16-byte chunks are stored in the order chunk ^ (t & 7), which keeps the
 // attention's ldmatrix reads of eight consecutive rows free of bank conflicts.

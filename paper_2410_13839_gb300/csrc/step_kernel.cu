@@ -717,6 +717,7 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(THREADS, 1) step_ke
     __shared__ int s_seq[MAX_ROWS], s_pos[MAX_ROWS], s_tok[MAX_ROWS];
     __shared__ int s_gseq[MAX_ROWS], s_gold[MAX_ROWS], s_gnew[MAX_ROWS];
     __shared__ float ln_part[2 * NWARPS][MT];
+    __shared__ float ln_stat[2][MT];
     __shared__ float s_scale[NWARPS][MT];
     __shared__ volatile int s_abort;
     __shared__ int s_issued, s_consumed;
@@ -915,7 +916,7 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(THREADS, 1) step_ke
         };
         // register rows -> LN -> bf16 hi | lo in xb
         auto ln_rows = [&](RowRegs<MT>& xr, const float (&g)[4], const float (&b)[4]) {
-            layer_norm_rows_fast<MT, ConsumerSync>(xr, d, g, b, a.ln_eps, ln_part);
+            layer_norm_rows<MT, ConsumerSync>(xr, d, g, b, a.ln_eps, ln_part, ln_stat);
             store_rows_split<MT>(xr, d, xb);
             consumer_sync();
         };
