@@ -19,6 +19,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -339,8 +340,26 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": reasons, "samples": len(rows)}
 
 
-def cpu_baseline(max_steps: int = 60):
-    """The oracle as it stands on this host: prefill + the first decode steps of the workload."""
+def cpu_model() -> str:
+    """The host CPU as /proc/cpuinfo names it (model name, or implementer/part on Arm)."""
+    try:
+        info = open("/proc/cpuinfo").read()
+    except OSError:
+        return platform.machine()
+    for line in info.splitlines():
+        if line.lower().startswith("model name"):
+            return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info.splitlines():
+        if ":" in line:
+            k, v = line.split(":", 1)
+            fields.setdefault(k.strip(), v.strip())
+    parts = [f"{k} {fields[k]}" for k in ("CPU implementer", "CPU part", "CPU variant") if k in fields]
+    return f"{platform.machine()} ({', '.join(parts)})" if parts else platform.machine()
+
+
+def _oracle_rate(max_steps: int):
+    """The oracle as it stands: prefill + the first decode steps of the workload (tokens/s, sample)."""
     from oracle.mtp import MTPOracle
     w = synth.make_weights(MODEL)
     ph, ac = synth.make_prompt(0, N_PH, N_AC, MODEL.phone_vocab)
@@ -350,10 +369,25 @@ def cpu_baseline(max_steps: int = 60):
     recs = o.generate(N_HEADS, TOP_K, max_steps=max_steps)
     dt = time.perf_counter() - t0
     toks = sum(r.accepted for r in recs)
+    return toks / dt, (f"prefill of the {N_PH + N_AC}-token prompt + first {len(recs)} decode steps "
+                       f"({toks} tokens), float64 numpy, {dt:.1f} s")
+
+
+def cpu_baseline(max_steps: int = 60, single_steps: int = 16):
+    """The oracle on this host's cores, and on one core (a child process with one BLAS thread)."""
+    value, sample = _oracle_rate(max_steps)
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
-    return {"value": toks / dt, "unit": "codec tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"prefill of the {N_PH + N_AC}-token prompt + first {len(recs)} decode steps "
-                      f"({toks} tokens), float64 numpy, {dt:.1f} s"}
+    out = {"value": value, "unit": "codec tokens/s", "cores": cores, "kind": "oracle", "sample": sample,
+           "cpu_model": cpu_model()}
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        res = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-rate-steps", str(single_steps)],
+                             env=env, capture_output=True, text=True, timeout=600)
+        one = json.loads(res.stdout.strip().splitlines()[-1])
+        out["single_thread"] = {"value": one["value"], "unit": "codec tokens/s", "cores": 1, "sample": one["sample"]}
+    except (subprocess.SubprocessError, ValueError, IndexError, KeyError, OSError) as e:
+        out["single_thread"] = {"value": None, "error": type(e).__name__}
+    return out
 
 
 KERNEL_SOURCES = ("paper_2410_13839_gb300/csrc/layer_fused.cu", "paper_2410_13839_gb300/csrc/common.cuh",
@@ -603,13 +637,17 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-rate-steps", type=int, default=0, help=argparse.SUPPRESS)  # child of cpu_baseline
     ap.add_argument("--no-b32", action="store_true", help="skip the batch-32 serving measurement")
     ap.add_argument("--no-sweep", action="store_true", help="skip the head/beam sweep")
     ap.add_argument("--no-c5", action="store_true", help="skip the isolated heads + Viterbi microbenchmark")
     ap.add_argument("--profile-b32", action="store_true",
                     help="only run a small batch-32 decode for kernel captures (prints no measurement)")
     args = ap.parse_args()
-    if args.profile_b32:
+    if args.oracle_rate_steps:
+        value, sample = _oracle_rate(args.oracle_rate_steps)
+        print(json.dumps({"value": value, "sample": sample}), flush=True)
+    elif args.profile_b32:
         run_profile_b32()
     elif args.impl == "reference":
         run_reference(args)

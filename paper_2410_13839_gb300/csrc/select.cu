@@ -95,24 +95,38 @@ __device__ void head_topk_warp(const float* row, int V, int k, int* out_ids, flo
 
 // Gather the transition scores the lattice uses, lq[t-1][i][j] = log_q[c_{t-1,i}][c_{t,j}]
 // for t = 1..n-1, into shared memory with all threads of the group at once
-// (one memory latency instead of one per recursion step).  Ids outside
-// [0, V) get -inf (never read out of range).
+// (one memory latency instead of one per recursion step).  Each pass covers
+// nthreads / kp candidate rows i (kp = k rounded up to a power of two, lane
+// j of a row slice = candidate j): no integer division per element.  Ids
+// outside [0, V) get -inf (never read out of range).
 __device__ __forceinline__ void gather_transitions(const int* ids, int n, int k, const float* log_q, int V,
                                                    float* lq, int tid, int nthreads) {
+    int kp = 1;
+    while (kp < k) kp <<= 1;
+    const int sh = __ffs(kp) - 1;
+    const int j = tid & (kp - 1), rows_per_pass = nthreads >> sh;
     const int kk = k * k;
-    for (int e = tid; e < (n - 1) * kk; e += nthreads) {
-        const int t = e / kk + 1, i = (e % kk) / k, j = e % k;
-        const int ci = ids[(t - 1) * k + i], cj = ids[t * k + j];
-        lq[e] = (ci >= 0 && ci < V && cj >= 0 && cj < V) ? __ldg(log_q + (size_t)ci * V + cj) : -INFINITY;
+    for (int t = 1; t < n; ++t) {
+        const int* prev = ids + (t - 1) * k;
+        const int cj = ids[t * k + min(j, k - 1)];
+        float* out = lq + (size_t)(t - 1) * kk;
+#pragma unroll 4
+        for (int i = tid >> sh; i < k && j < k; i += rows_per_pass) {
+            const int ci = prev[i];
+            out[i * k + j] = (ci >= 0 && ci < V && cj >= 0 && cj < V) ? __ldg(log_q + (size_t)ci * V + cj) : -INFINITY;
+        }
     }
 }
 
 // Viterbi over ids/lp [n][k] with transitions lq [n-1][k][k] and backpointers
 // bp [MAX_NHEADS][32] (all shared memory); lane 0 writes the results.  The
-// loops stay rolled: the kernel runs once per step with a cold instruction
-// cache, so its time follows the instructions it fetches.
-__device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, int n, int k, int* bp, int* path,
-                             float* score) {
+// selection kernel runs it once per step with a cold instruction cache and
+// keeps the loops rolled (UNROLL = 1: its time follows the instructions it
+// fetches); the stand-alone kernel, warm over many lattices, unrolls the
+// candidate loop (the comparisons stay in order: the lowest i keeps ties).
+template <int UNROLL>
+__device__ void viterbi_warp_t(const int* ids, const float* lp, const float* lq, int n, int k, int* bp, int* path,
+                               float* score) {
     const int lane = threadIdx.x & 31;
     const bool on = lane < k;
     float delta = on ? lp[lane] : -INFINITY;
@@ -121,7 +135,7 @@ __device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, i
         const float* lqt = lq + (size_t)(t - 1) * k * k + (on ? lane : 0);
         float best = 0.f;
         int arg = 0;
-#pragma unroll 1
+#pragma unroll (UNROLL)
         for (int i = 0; i < k; ++i) {
             const float di = __shfl_sync(FULL_MASK, delta, i);
             const float val = __fadd_rn(di, lqt[i * k]);
@@ -399,14 +413,14 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     } else {
         gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
         __syncthreads();
-        if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_bp, s_path, &s_score);
+        if (warp == 0) viterbi_warp_t<1>(s_ids, s_lp, s_lq, n, k, s_bp, s_path, &s_score);
     }
     __syncthreads();
     trace_mark(a.trace, 1);  // path
     if (warp != 0) return;
 
     // Acceptance and the slot's bookkeeping, one lane per token (short code:
-    // see viterbi_warp).
+    // see viterbi_warp_t).
     const int lane = threadIdx.x & 31;
     const int rem = s_st[2], gc = s_st[3];
     int n_emit;  // tokens this step emits (before the EOS / budget cut), s_emit
@@ -500,7 +514,7 @@ __global__ void __launch_bounds__(VIT_WARPS * 32) viterbi_kernel(const ViterbiAr
     float* lq = vit_lq + (size_t)warp * (a.n - 1) * a.k * a.k;
     gather_transitions(s_ids[warp], a.n, a.k, a.log_q, a.vocab, lq, lane, 32);
     __syncwarp();
-    viterbi_warp(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_bp[warp], s_path[warp], &s_score[warp]);
+    viterbi_warp_t<4>(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_bp[warp], s_path[warp], &s_score[warp]);
     __syncwarp();
     if (lane != 0) return;
     int acc, done;
