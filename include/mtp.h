@@ -137,6 +137,26 @@ MTP_API const char* mtp_last_error(void);
 MTP_API int mtp_prefill(mtp_ctx* ctx, int seq_slot, const int32_t* phonemes, int n_ph,
                         const int32_t* acoustic, int n_ac, int max_new_tokens);
 
+/* Admit a sequence into slot `seq_slot` without running its prompt: the same
+ * checks, page reservation and prompt copy as mtp_prefill, then the prompt
+ * [phonemes ; acoustic prompt] (Sec. III-A) is prefilled by the following
+ * decode steps, inside their batched pass beside the other slots' fed rows:
+ * each step's prefill lane takes up to 128 prompt positions (a multiple of
+ * n_heads) from the admitted slots in slot order, and a slot selects its
+ * first tokens in the step after its last prompt row ran.  mtp_generate runs
+ * such steps first; mtp_prefill_pending runs all admitted prompts at once.
+ * Needs the batched path (bf16 weights) and MTP_ACCEPT_ALL; otherwise the
+ * call is mtp_prefill.  Errors: as mtp_prefill. */
+MTP_API int mtp_admit(mtp_ctx* ctx, int seq_slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic,
+                      int n_ac, int max_new_tokens);
+
+/* Run every admitted prompt now (Sec. III-A prefill, many sequences per
+ * pass): passes of up to all the batched rows, filled with the admitted
+ * slots' remaining prompt positions in slot order, in attention groups of 8
+ * positions of one slot.  Returns the number of passes (0: none pending).
+ * Errors: MTP_ERR_INVALID (no batched path), MTP_ERR_CUDA, MTP_ERR_DEVICE. */
+MTP_API int mtp_prefill_pending(mtp_ctx* ctx);
+
 /* Return the slot's pages to the pool and mark it inactive. */
 MTP_API int mtp_release(mtp_ctx* ctx, int seq_slot);  /* Errors: MTP_ERR_INVALID (slot), MTP_ERR_CUDA. */
 

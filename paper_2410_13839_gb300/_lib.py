@@ -66,6 +66,8 @@ def _load() -> ctypes.CDLL:
         "mtp_last_error": (ctypes.c_char_p, []),
         "mtp_prefill": (i32, [vp, i32, vp, i32, vp, i32, i32]),
         "mtp_release": (i32, [vp, i32]),
+        "mtp_admit": (i32, [vp, i32, vp, i32, vp, i32, i32]),
+        "mtp_prefill_pending": (i32, [vp]),
         "mtp_decode_step": (i32, [vp, i32, i32, vp, vp, vp]),
         "mtp_generate": (i32, [vp, i32, i32, vp, i32, vp]),
         "mtp_rollback": (i32, [vp, i32, i32]),

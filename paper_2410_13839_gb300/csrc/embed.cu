@@ -31,6 +31,15 @@ __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
                     last = (j == np - 1);
                 }
             }
+        } else if (a.mode == 2) {  // prefill lane: the plan kernel chose slot and position
+            if (r < a.rows) {
+                seq = a.row_seq[a.row0 + r];
+                if (seq >= 0) {
+                    pos = a.row_pos[a.row0 + r];
+                    tok = a.prompt[(size_t)seq * a.prompt_stride + pos];
+                    phone = pos < a.prompt_nph[seq];
+                }
+            }
         } else {  // prefill chunk: positions p0 .. p0 + rows - 1 of one slot
             pos = a.p0 + r;
             if (r < a.rows && pos < a.total) {
@@ -44,9 +53,11 @@ __global__ void __launch_bounds__(256) embed_kernel(const EmbedArgs a) {
             atomicOr(a.err, ERR_BOUNDS);
             seq = -1;
         }
-        a.row_seq[r] = seq;
-        a.row_pos[r] = seq >= 0 ? pos : -1;
-        a.row_last[r] = seq >= 0 ? last : 0;
+        if (a.mode != 2) {  // the lane's plan is already written
+            a.row_seq[r] = seq;
+            a.row_pos[r] = seq >= 0 ? pos : -1;
+            a.row_last[r] = seq >= 0 ? last : 0;
+        }
         s_act = seq >= 0;
         s_tok = tok;
         s_pos = pos;
@@ -92,6 +103,46 @@ __global__ void convert_rows_kernel(const void* src, int src_bf16, float* dst, l
                       : reinterpret_cast<const float*>(src)[i];
 }
 
+__global__ void __launch_bounds__(1024) lane_plan_kernel(const LanePlanArgs a) {
+    __shared__ int s_scan[1024];
+    pdl_wait();  // the previous step's selection moved the slots' state
+    pdl_launch_dependents();
+    const int b = threadIdx.x;
+    for (int i = threadIdx.x; i < a.capacity; i += blockDim.x) {
+        a.row_seq[a.row0 + i] = -1;
+        a.row_pos[a.row0 + i] = -1;
+        a.row_last[a.row0 + i] = 0;
+    }
+    int left = 0, len = 0;
+    if (b < a.slots && a.active[b] && !a.done[b]) {
+        left = max(0, a.prompt_left[b]);
+        len = a.seq_len[b];
+    }
+    const int demand = (left + a.rpg - 1) / a.rpg * a.rpg;
+    s_scan[b] = demand;  // inclusive scan of the padded demands (Hillis-Steele)
+    __syncthreads();
+    for (int o = 1; o < (int)blockDim.x; o <<= 1) {
+        const int add = b >= o ? s_scan[b - o] : 0;
+        __syncthreads();
+        s_scan[b] += add;
+        __syncthreads();
+    }
+    const int start = s_scan[b] - demand;
+    int take = 0;
+    if (left > 0 && start < a.capacity) {
+        take = min(left, a.capacity - start);
+        for (int i = 0; i < take; ++i) {
+            const int row = a.row0 + start + i;
+            a.row_seq[row] = b;
+            a.row_pos[row] = len + i;
+            a.row_last[row] = (i == take - 1 && take == left) ? 1 : 0;
+        }
+        a.prompt_left[b] = left - take;
+        a.seq_len[b] = len + take;
+    }
+    if (b < a.slots) a.lane_take[b] = take;
+}
+
 __global__ void slot_set_kernel(SlotSet s) {
     if (threadIdx.x != 0) return;
     pdl_wait();
@@ -102,6 +153,8 @@ __global__ void slot_set_kernel(SlotSet s) {
     if (s.set_done >= 0) s.done[b] = s.set_done;
     if (s.set_active >= 0) s.active[b] = s.set_active;
     if (s.set_gen >= 0) s.gen_count[b] = s.set_gen;
+    if (s.set_prompt_left >= 0 && s.prompt_left) s.prompt_left[b] = s.set_prompt_left;
+    if (s.set_prompt_nph >= 0 && s.prompt_nph) s.prompt_nph[b] = s.set_prompt_nph;
 }
 
 }  // namespace
@@ -167,6 +220,20 @@ __global__ void trace_reset_kernel(unsigned long long* tr, int records) {
 cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s) {
     trace_reset_kernel<<<(records + 255) / 256, 256, 0, s>>>(trace, records);
     return cudaGetLastError();
+}
+
+cudaError_t launch_lane_plan(const LanePlanArgs& a, cudaStream_t s, bool pdl) {
+    if (a.slots < 1 || a.slots > 1024 || a.rpg < 1 || a.capacity < 1 || a.capacity % a.rpg) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3((a.slots + 31) / 32 * 32);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, lane_plan_kernel, a);
 }
 
 cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s) {

@@ -174,7 +174,8 @@ cudaError_t launch_step_kernel(const StepArgs& a, int grid, cudaStream_t s, bool
 
 // --------------------------------------------------------------- embed ----
 struct EmbedArgs {
-    int mode;                  // 0 = decode rows from slot state, 1 = prefill chunk
+    int mode;                  // 0 = decode rows from slot state, 1 = prefill chunk, 2 = prefill lane rows
+                               // (slot and position already in row_seq / row_pos at row0 + r, token from prompt)
     const void* tok_phone; const void* tok_codec; int w_bf16;
     int phone_vocab, codec_vocab;
     const float* pe; int d; int max_pos;   // positional table [max_pos][d]
@@ -186,11 +187,28 @@ struct EmbedArgs {
     const int* active; const int* done; const int* n_pending; const int* pending; const int* seq_len;
     // prefill
     int slot, p0, n_ph, total, prompt_stride; const int* prompt;
+    // prefill lane (mode 2): rows row0.. of the plan arrays; phoneme count of each slot's prompt
+    int row0; const int* prompt_nph;
     float* zero_buf;           // [MAX_ROWS][d] zeroed (first residual accumulation target)
     int* err;
     unsigned long long* trace;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s, bool pdl);
+
+// The prefill lane of a pass: up to `capacity` rows (a multiple of rpg) from
+// row0 on, given to the slots with prompt tokens left in slot order, each
+// slot's share padded to a multiple of rpg (attention groups hold one slot).
+// Slot b gets take_b = min(left_b, capacity - start_b) rows, start_b = the
+// padded demands of the slots before it; row i of its share is prompt
+// position len_b + i, the share's last row is marked when it ends the
+// prompt.  The kernel writes the rows' plan (row_seq/row_pos/row_last, -1
+// for unused rows) and lane_take, and advances prompt_left and seq_len.
+struct LanePlanArgs {
+    int slots, rpg, capacity, row0;
+    int* prompt_left; int* seq_len; const int* active; const int* done;
+    int* row_seq; int* row_pos; int* row_last; int* lane_take;
+};
+cudaError_t launch_lane_plan(const LanePlanArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_pe_table(float* pe, int max_ctx, int d, cudaStream_t s);
 
 // -------------------------------------------------------------- select ----
@@ -212,6 +230,9 @@ struct SelectArgs {
     int lattice;              // 0: per-head top-k states (reading A); 1: union of all heads' top-k (reading B)
     int sampling;             // 0: the lattice's best path (Viterbi); 1: a path drawn from its posterior
     unsigned long long seed;  // path draws: counter-based uniforms of (seed, slot, tokens generated, position)
+    const int* prompt_left;   // slots with prompt tokens left select nothing (null: no admitted prompts)
+    const int* lane_take;     // with `lane`: slots whose prompt rows ran in this step's lane select nothing
+    int lane;
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
 
@@ -244,7 +265,9 @@ cudaError_t launch_convert_rows(const void* src, int src_bf16, float* dst, int r
 struct SlotSet {
     int slot;
     int* seq_len; int* n_pending; int* remaining; int* done; int* active; int* gen_count;
+    int* prompt_left; int* prompt_nph;
     int set_len, set_pending, set_remaining, set_done, set_active, set_gen;
+    int set_prompt_left, set_prompt_nph;
 };
 cudaError_t launch_slot_set(const SlotSet& set, cudaStream_t s);
 cudaError_t launch_trace_reset(unsigned long long* trace, int records, cudaStream_t s);

@@ -159,6 +159,9 @@ struct mtp_ctx {
         *d_out_tokens = nullptr, *d_out_accepted = nullptr;
     int* d_err = nullptr;
     int* d_kept = nullptr;  // VERIFY_GREEDY: drafts kept this step, per slot
+    // admitted prompts (mtp_admit), run in the prefill lane of the batched steps
+    int *d_prompt_left = nullptr, *d_prompt_nph = nullptr, *d_lane_take = nullptr;
+    std::vector<int> h_prompt_left;  // host copy of prompt_left, advanced by the same rule as the device
     std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;  // (n_heads, top_k, traced)
     std::map<std::tuple<int, int, int>, std::vector<int>> graph_kinds;
     int last_n = 0, last_k = 0;
@@ -497,7 +500,8 @@ int launch_step_pass(mtp_ctx* c, int rows, int rpg, int seq_base, cudaStream_t s
 int setup_batched(mtp_ctx* c) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
-    c->bm_max = std::max(cf.max_batch * cf.n_heads_max, PREFILL_ROWS);
+    // every slot's fed rows plus a prefill lane of up to PREFILL_ROWS prompt rows
+    c->bm_max = cf.max_batch * cf.n_heads_max + PREFILL_ROWS;
     if (c->wbytes != 2 || !c->d_w2p) return MTP_OK;
     const size_t M = (size_t)c->bm_max;
     MTP_TRY(c->alloc(&c->d_bx, M * d));
@@ -513,8 +517,9 @@ int setup_batched(mtp_ctx* c) {
     c->d_alo = reinterpret_cast<__nv_bfloat16*>(alo);
     c->d_uhi = reinterpret_cast<__nv_bfloat16*>(uhi);
     c->d_ulo = reinterpret_cast<__nv_bfloat16*>(ulo);
-    {  // attention workspace for the decode groups (slots) and the prefill groups (8-row runs)
-        const int gd = cf.max_batch, gp = (c->bm_max + 7) / 8;
+    {  // attention workspace for the decode groups (slots, plus the lane's groups of as few as one row)
+        // and the prefill groups (8-row runs)
+        const int gd = cf.max_batch + PREFILL_ROWS, gp = (c->bm_max + 7) / 8;
         c->battn_ws_units = std::max(gd * attn_splits_for(gd, H, P, cf.max_ctx, c->num_sms),
                                      gp * attn_splits_for(gp, H, P, cf.max_ctx, c->num_sms));
         MTP_TRY(c->alloc(&c->d_bws, attn_workspace_floats(c->battn_ws_units, H, 1, MAX_ROWS)));
@@ -626,6 +631,7 @@ SelectArgs select_base(mtp_ctx* c, int n, int k) {
     a.err = c->d_err;
     a.policy = c->cfg.accept_policy; a.kept = c->d_kept; a.lattice = c->lattice;
     a.sampling = c->sampling; a.seed = c->sample_seed;
+    a.prompt_left = c->d_prompt_left; a.lane_take = c->d_lane_take; a.lane = 0;
     return a;
 }
 
@@ -648,23 +654,66 @@ int enqueue_verify(mtp_ctx* c, const float* x, int slots, int n, int b0, cudaStr
     return MTP_OK;
 }
 
+// ---- the prefill lane (prompts admitted with mtp_admit) ----
+
+// Prompt rows the lane of a batched step takes: up to PREFILL_ROWS, whole groups of n.
+int lane_rows(int n) { return PREFILL_ROWS / n * n; }
+
+bool lane_pending(const mtp_ctx* c) {
+    for (int v : c->h_prompt_left)
+        if (v > 0) return true;
+    return false;
+}
+
+// The host's copy of the lane rule of lane_plan_kernel (slot order, padded demands).
+void lane_mirror(mtp_ctx* c, int capacity, int rpg) {
+    int start = 0;
+    for (int& left : c->h_prompt_left) {
+        if (left <= 0) continue;
+        const int demand = (left + rpg - 1) / rpg * rpg;
+        if (start < capacity) left -= std::min(left, capacity - start);
+        start += demand;
+    }
+}
+
+int enqueue_lane_plan(mtp_ctx* c, int row0, int capacity, int rpg, cudaStream_t s, bool pdl, Prof* prof) {
+    LanePlanArgs lp;
+    std::memset(&lp, 0, sizeof(lp));
+    lp.slots = c->cfg.max_batch; lp.rpg = rpg; lp.capacity = capacity; lp.row0 = row0;
+    lp.prompt_left = c->d_prompt_left; lp.seq_len = c->d_len; lp.active = c->d_active; lp.done = c->d_done;
+    lp.row_seq = c->d_row_seq; lp.row_pos = c->d_row_pos; lp.row_last = c->d_row_last; lp.lane_take = c->d_lane_take;
+    LAUNCH(MTP_K_EMBED, launch_lane_plan(lp, s, pdl));
+    EmbedArgs e = embed_base(c);
+    e.mode = 2; e.rows = capacity; e.row0 = row0; e.prompt_nph = c->d_prompt_nph;
+    e.x = c->d_bx + (size_t)row0 * c->cfg.d_model; e.zero_buf = nullptr;
+    e.trace = tslot(c, MTP_K_EMBED);
+    LAUNCH(MTP_K_EMBED, launch_embed(e, s, pdl));
+    return MTP_OK;
+}
+
 // chain: the step follows another step in the same stream or graph; its first
 // kernel then starts under programmatic launch (it waits for the previous
 // step's selection before it lets the next kernels start).
-int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof, bool chain = false) {
+// lane: the pass also runs up to lane_rows(n) prompt rows of admitted slots
+// (batched path; the caller checked that it is available).
+int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof, bool chain = false,
+                 bool lane = false) {
     const int B = c->cfg.max_batch, d = c->cfg.d_model, V = c->cfg.codec_vocab;
     const int spc = std::max(1, MAX_ROWS / n);
     const bool verify = c->cfg.accept_policy == MTP_VERIFY_GREEDY;
     // one pass feeds every slot: the heads read its rows directly (VERIFY_GREEDY: the kept row, via h_last)
     const bool single = B <= spc && !verify;
     float* final_x = nullptr;
-    if (B > spc && c->use_batched && c->batched_ok && B * n <= c->bm_max) {  // every slot's rows in one pass
-        const int M = B * n;
+    const int P = lane ? lane_rows(n) : 0;
+    if ((B > spc || lane) && c->use_batched && c->batched_ok && B * n + P <= c->bm_max) {  // every slot's rows in one pass
+        const int Md = B * n, M = Md + P;
         EmbedArgs e = embed_base(c);
-        e.mode = 0; e.rows = M; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
+        e.mode = 0; e.rows = Md; e.seq_base = 0; e.n_heads = n; e.x = c->d_bx; e.zero_buf = nullptr;
         e.trace = tslot(c, MTP_K_EMBED);
         LAUNCH(MTP_K_EMBED, launch_embed(e, s, chain && pdl));
-        MTP_TRY(run_layers_batched(c, M, n, B, PLAN_DEVICE, s, pdl, prof));
+        if (lane) MTP_TRY(enqueue_lane_plan(c, Md, P, n, s, pdl, prof));
+        // with a lane the groups are read from the rows' plan (slots of n rows, then the lane's groups)
+        MTP_TRY(run_layers_batched(c, M, n, M / n, lane ? PLAN_ROWS : PLAN_DEVICE, s, pdl, prof));
         if (verify) {
             MTP_TRY(enqueue_verify(c, c->d_bx, B, n, 0, s, pdl, prof));
         } else {
@@ -673,6 +722,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
         }
         MTP_TRY(launch_heads_batched(c, c->d_h_last, B, n, c->d_logits, s, pdl, prof));
         SelectArgs sa = select_base(c, n, k);
+        sa.lane = lane ? 1 : 0;
         sa.trace = tslot(c, MTP_K_SELECT);
         LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
         return MTP_OK;
@@ -709,21 +759,21 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
     return MTP_OK;
 }
 
-int run_step(mtp_ctx* c, int n, int k) {
+int run_step(mtp_ctx* c, int n, int k, bool lane = false) {
     c->last_n = n;
     c->last_k = k;
     if (!c->use_graphs) {
         c->trace_kinds.clear();
-        return enqueue_step(c, n, k, c->stream, c->use_pdl, nullptr);
+        return enqueue_step(c, n, k, c->stream, c->use_pdl, nullptr, false, lane);
     }
-    const auto key = std::make_tuple(n, k, c->tracing ? 1 : 0);
+    const auto key = std::make_tuple(n, k, (c->tracing ? 1 : 0) | (lane ? 4 : 0));
     auto it = c->graphs.find(key);
     if (it == c->graphs.end()) {
         cudaGraph_t graph = nullptr;
         cudaGraphExec_t exec = nullptr;
         c->trace_kinds.clear();
         CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
-        const int r = enqueue_step(c, n, k, c->cap_stream, c->use_pdl, nullptr);
+        const int r = enqueue_step(c, n, k, c->cap_stream, c->use_pdl, nullptr, false, lane);
         const cudaError_t ec = cudaStreamEndCapture(c->cap_stream, &graph);
         if (r != MTP_OK) {
             if (graph) cudaGraphDestroy(graph);
@@ -794,13 +844,16 @@ int copy_out(void* dst, const void* src, size_t bytes, cudaStream_t s) {
     return MTP_OK;
 }
 
-int slot_set(mtp_ctx* c, int slot, int len, int pend, int rem, int done, int active, int gen) {
+int slot_set(mtp_ctx* c, int slot, int len, int pend, int rem, int done, int active, int gen, int prompt_left = -1,
+             int prompt_nph = -1) {
     SlotSet ss;
     ss.slot = slot;
     ss.seq_len = c->d_len; ss.n_pending = c->d_npend; ss.remaining = c->d_remaining;
     ss.done = c->d_done; ss.active = c->d_active; ss.gen_count = c->d_gen_count;
+    ss.prompt_left = c->d_prompt_left; ss.prompt_nph = c->d_prompt_nph;
     ss.set_len = len; ss.set_pending = pend; ss.set_remaining = rem;
     ss.set_done = done; ss.set_active = active; ss.set_gen = gen;
+    ss.set_prompt_left = prompt_left; ss.set_prompt_nph = prompt_nph;
     CUDA_TRY(launch_slot_set(ss, c->stream));
     return MTP_OK;
 }
@@ -1107,7 +1160,7 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
                              sb, sh));
     }
     const int lb = std::max(B, MAX_ROWS);
-    const int row_cap = (std::max(std::max(MAX_ROWS, B * nm), PREFILL_ROWS) + 7) / 8 * 8;  // rows of one pass
+    const int row_cap = (B * nm + PREFILL_ROWS + 7) / 8 * 8;  // rows of one pass (slots' rows + the prefill lane)
     if ((r = c->alloc(&c->d_pe, (size_t)cf.max_ctx * d)) ||
         (r = c->alloc(&c->d_kv, (size_t)c->n_pages * c->page_elems)) ||
         (r = c->alloc(&c->d_block_table, (size_t)B * c->pages_per_seq)) ||
@@ -1123,9 +1176,12 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
         (r = c->alloc(&c->d_out_tokens, (size_t)B * nm)) || (r = c->alloc(&c->d_out_accepted, B)) ||
         (r = c->alloc(&c->d_row_seq, row_cap)) || (r = c->alloc(&c->d_row_pos, row_cap)) ||
         (r = c->alloc(&c->d_row_last, row_cap)) || (r = c->alloc(&c->d_err, 1)) || (r = c->alloc(&c->d_kept, B)) ||
+        (r = c->alloc(&c->d_prompt_left, B)) || (r = c->alloc(&c->d_prompt_nph, B)) ||
+        (r = c->alloc(&c->d_lane_take, B)) ||
         (r = setup_batched(c)) || (r = setup_step_kernel(c)))
         return bail(r);
     c->h_block_table.assign((size_t)B * c->pages_per_seq, -1);
+    c->h_prompt_left.assign(B, 0);
     if (cudaMemcpy(c->d_block_table, c->h_block_table.data(), c->h_block_table.size() * sizeof(int),
                    cudaMemcpyHostToDevice) != cudaSuccess)
         return bail(fail(MTP_ERR_CUDA, "block table upload failed"));
@@ -1221,9 +1277,10 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
     return MTP_OK;
 }
 
-MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic, int n_ac,
-                        int max_new_tokens) {
-    g_err.clear();
+// Validation, page reservation and the prompt's copy to the device, shared by
+// mtp_prefill and mtp_admit; *T_out = prompt length.
+static int take_prompt(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic, int n_ac,
+                int max_new_tokens, long long* T_out) {
     MTP_TRY(check_slot(c, slot));
     const mtp_config& cf = c->cfg;
     if (n_ph < 0 || n_ac < 0 || n_ph + n_ac < 1) return fail(MTP_ERR_INVALID, "empty prompt");
@@ -1262,7 +1319,19 @@ MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph,
     int* prompt = c->d_prompt + (size_t)slot * cf.max_ctx;
     if (n_ph) CUDA_TRY(cudaMemcpyAsync(prompt, phonemes, n_ph * sizeof(int), cudaMemcpyDefault, s));
     if (n_ac) CUDA_TRY(cudaMemcpyAsync(prompt + n_ph, acoustic, n_ac * sizeof(int), cudaMemcpyDefault, s));
-    MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0));
+    *T_out = T;
+    return MTP_OK;
+}
+
+MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic, int n_ac,
+                        int max_new_tokens) {
+    g_err.clear();
+    long long T = 0;
+    MTP_TRY(take_prompt(c, slot, phonemes, n_ph, acoustic, n_ac, max_new_tokens, &T));
+    const mtp_config& cf = c->cfg;
+    cudaStream_t s = c->stream;
+    c->h_prompt_left[slot] = 0;
+    MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0, 0, n_ph));
     Prof* prof = nullptr;
     float* final_x = nullptr;
     if (c->use_batched && c->batched_ok) {  // chunks of PREFILL_ROWS positions through the batched path
@@ -1301,9 +1370,49 @@ MTP_API int mtp_release(mtp_ctx* c, int slot) {
     CUDA_TRY(cudaMemcpyAsync(c->d_block_table + (size_t)slot * c->pages_per_seq,
                              c->h_block_table.data() + (size_t)slot * c->pages_per_seq,
                              c->pages_per_seq * sizeof(int), cudaMemcpyHostToDevice, c->stream));
-    MTP_TRY(slot_set(c, slot, 0, 0, 0, 0, 0, 0));
+    MTP_TRY(slot_set(c, slot, 0, 0, 0, 0, 0, 0, 0));
+    c->h_prompt_left[slot] = 0;
     CUDA_TRY(cudaStreamSynchronize(c->stream));
     return MTP_OK;
+}
+
+// The prefill lane can serve admitted prompts: batched path, ACCEPT_ALL.
+static bool lane_usable(const mtp_ctx* c) {
+    return c->use_batched && c->batched_ok && c->cfg.accept_policy == MTP_ACCEPT_ALL;
+}
+
+MTP_API int mtp_admit(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph, const int32_t* acoustic, int n_ac,
+                      int max_new_tokens) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (!lane_usable(c)) return mtp_prefill(c, slot, phonemes, n_ph, acoustic, n_ac, max_new_tokens);
+    long long T = 0;
+    MTP_TRY(take_prompt(c, slot, phonemes, n_ph, acoustic, n_ac, max_new_tokens, &T));
+    MTP_TRY(slot_set(c, slot, 0, 0, max_new_tokens, 0, 1, 0, (int)T, n_ph));
+    c->h_prompt_left[slot] = (int)T;
+    return MTP_OK;
+}
+
+MTP_API int mtp_prefill_pending(mtp_ctx* c) {
+    g_err.clear();
+    MTP_TRY(check_ctx(c));
+    if (!lane_pending(c)) return 0;
+    if (!lane_usable(c)) return fail(MTP_ERR_INVALID, "admitted prompts need the batched path");
+    const mtp_config& cf = c->cfg;
+    cudaStream_t s = c->stream;
+    const int P = c->bm_max / 8 * 8;  // prompt rows per pass, in attention groups of 8 positions
+    int passes = 0;
+    while (lane_pending(c)) {
+        MTP_TRY(enqueue_lane_plan(c, 0, P, 8, s, c->use_pdl, nullptr));
+        MTP_TRY(run_layers_batched(c, P, 8, P / 8, PLAN_ROWS, s, c->use_pdl, nullptr));
+        Prof* prof = nullptr;
+        LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, P, nullptr, s,
+                                            c->use_pdl));
+        lane_mirror(c, P, 8);
+        ++passes;
+    }
+    MTP_TRY(check_device_error(c));
+    return passes;
 }
 
 MTP_API int mtp_decode_step(mtp_ctx* c, int n, int k, int32_t* out_tokens, int32_t* out_accepted,
@@ -1311,7 +1420,10 @@ MTP_API int mtp_decode_step(mtp_ctx* c, int n, int k, int32_t* out_tokens, int32
     g_err.clear();
     MTP_TRY(check_ctx(c));
     MTP_TRY(check_nk(c, n, k));
-    MTP_TRY(run_step(c, n, k));
+    const bool lane = lane_pending(c);
+    if (lane && !lane_usable(c)) return fail(MTP_ERR_INVALID, "admitted prompts need the batched path");
+    MTP_TRY(run_step(c, n, k, lane));
+    if (lane) lane_mirror(c, lane_rows(n), n);
     const int B = c->cfg.max_batch, nm = c->cfg.n_heads_max;
     if (out_tokens)
         CUDA_TRY(cudaMemcpy2DAsync(out_tokens, n * sizeof(int), c->d_out_tokens, nm * sizeof(int), n * sizeof(int), B,
@@ -1334,6 +1446,12 @@ MTP_API int mtp_generate(mtp_ctx* c, int n, int k, int32_t* out_tokens, int out_
     // step until EOS or the budget) finishes in one round, VERIFY_GREEDY (1..n) in a few.
     std::vector<int> rem, done, active;
     int steps = 0;
+    // admitted prompts first: steps with a prefill lane (the other slots decode meanwhile)
+    if (lane_pending(c) && !lane_usable(c)) return fail(MTP_ERR_INVALID, "admitted prompts need the batched path");
+    for (; lane_pending(c); ++steps) {
+        MTP_TRY(run_step(c, n, k, true));
+        lane_mirror(c, lane_rows(n), n);
+    }
     for (;;) {
         MTP_TRY(read_slot_ints(c, c->d_remaining, rem));
         MTP_TRY(read_slot_ints(c, c->d_done, done));

@@ -378,7 +378,9 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     __syncthreads();
     pdl_wait();
     trace_wait(a.trace);
-    if (do_accept && (!s_st[0] || s_st[1])) {
+    // a slot still running its prompt (admitted, prefilled in the lane of the steps) selects nothing yet
+    const bool prefilling = do_accept && a.prompt_left && (a.prompt_left[b] > 0 || (a.lane && a.lane_take[b] > 0));
+    if (do_accept && (!s_st[0] || s_st[1] || prefilling)) {
         if (threadIdx.x < a.n_max) a.out_tokens[(size_t)b * a.n_max + threadIdx.x] = -1;
         if (threadIdx.x == 0) a.out_accepted[b] = 0;
         return;

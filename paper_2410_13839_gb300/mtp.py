@@ -110,6 +110,18 @@ def mtp_release(ctx: int, slot: int) -> None:
     check(lib.mtp_release(ctx, slot))
 
 
+def mtp_admit(ctx: int, slot: int, phonemes, acoustic, max_new_tokens: int) -> None:
+    """Admit a prompt without running it: the next decode steps prefill it in their lane."""
+    ph = _as_i32(phonemes)
+    ac = _as_i32(acoustic)
+    check(lib.mtp_admit(ctx, slot, _ptr(ph), _len(ph), _ptr(ac), _len(ac), max_new_tokens))
+
+
+def mtp_prefill_pending(ctx: int) -> int:
+    """Run every admitted prompt now, many slots' prompt rows per pass; returns the passes."""
+    return check(lib.mtp_prefill_pending(ctx))
+
+
 def mtp_decode_step(ctx: int, n_heads: int, top_k: int, out_tokens=None, out_accepted=None,
                     out_done=None) -> None:
     check(lib.mtp_decode_step(ctx, n_heads, top_k, _ptr(out_tokens), _ptr(out_accepted), _ptr(out_done)))
@@ -259,6 +271,9 @@ class MTPDecoder:
 
     def prefill(self, slot, phonemes, acoustic, max_new_tokens):
         mtp_prefill(self.ctx, slot, phonemes, acoustic, max_new_tokens)
+
+    def admit(self, slot, phonemes, acoustic, max_new_tokens):
+        mtp_admit(self.ctx, slot, phonemes, acoustic, max_new_tokens)
 
     def decode_step(self, n_heads, top_k):
         b = self.config.max_batch
