@@ -275,11 +275,25 @@ def run_c5(mtp, ctx, stream):
     vit_s = ev[2].elapsed_time(ev[3]) / 1e3 / calls
     head_bytes = C5_N * V * d * 2
     flops = 2.0 * C5_BATCH * C5_N * V * d
+    gathers = C5_LATTICES * (C5_N - 1) * C5_K * C5_K
     return {"workload": "isolated heads + Viterbi: 256 bf16 hidden rows N(0,1), n=8 heads x V=1025 with "
                         "log-softmax and top-16; Viterbi + acceptance over 10^4 lattices of 8 x 16",
             "heads_topk_us": heads_s * 1e6, "heads_gbs": head_bytes / heads_s / 1e9,
             "heads_tflops": flops / heads_s / 1e12, "viterbi_us": vit_s * 1e6,
-            "viterbi_lattices_per_s": C5_LATTICES / vit_s}
+            "viterbi_lattices_per_s": C5_LATTICES / vit_s,
+            "viterbi_roofline": {
+                "bound": "l2_tag_requests", "achieved": gathers / vit_s / 1e9, "peak": L2_TAG_REQUESTS_PEAK,
+                "unit": "G gathers/s", "frac": gathers / vit_s / 1e9 / L2_TAG_REQUESTS_PEAK,
+                "traffic": VITERBI_C5_TAG_REQUESTS, "gathers_per_call": gathers,
+                "peak_source": "ncu: lts__t_tag_requests.sum.per_second / its % of peak (GB300)"}}
+
+
+# The stand-alone Viterbi gathers (n-1) k^2 transition scores per lattice, 4 bytes
+# each at arbitrary ids from a table resident in L2: one L2 tag lookup per
+# gather, so the L2's tag-request rate bounds it.  ncu on GB300: 236 requests/ns
+# at 62.5 % of peak -> 378 G requests/s; 15.1 M requests per C5 call.
+L2_TAG_REQUESTS_PEAK = 378.0
+VITERBI_C5_TAG_REQUESTS = 15_144_000
 
 
 def run_sweep(mtp, stream):
@@ -405,8 +419,8 @@ def cpu_baseline(max_steps: int = 60, single_steps: int = 16):
     return out
 
 
-KERNEL_SOURCES = ("paper_2410_13839_gb300/csrc/layer_fused.cu", "paper_2410_13839_gb300/csrc/common.cuh",
-                  "paper_2410_13839_gb300/csrc/kernels.cuh")
+KERNEL_SOURCES = ("paper_2410_13839_gb300/csrc/layer_fused.cu", "paper_2410_13839_gb300/csrc/frag.cuh",
+                  "paper_2410_13839_gb300/csrc/common.cuh")
 
 
 def kernel_source_sha1() -> str:
@@ -645,6 +659,37 @@ def run_profile_b32():
 PROFILE_B32_STEPS = 12
 
 
+def run_profile_select():
+    """Kernel captures of the selection kernels (not a measurement): three mtp_viterbi
+    calls on the C5 lattices (10^4 x 8 x 16), then four B=1 decode steps of the
+    VALL-E-sized model (prompt 64 + 225, n=4, top_k=4), each one select_kernel launch."""
+    import torch
+    from paper_2410_13839_gb300 import build
+    build.build()
+    from paper_2410_13839_gb300 import mtp
+    V = MODEL.codec_vocab
+    c_ids, c_lp = c5_lattices(C5_LATTICES, C5_N, C5_K, V)
+    t_ids, t_lp = torch.from_numpy(c_ids).cuda(), torch.from_numpy(c_lp).cuda()
+    t_q = torch.from_numpy(synth.transition_log_q(V)).cuda()
+    path = torch.zeros((C5_LATTICES, C5_N), dtype=torch.int32, device="cuda")
+    acc = torch.zeros(C5_LATTICES, dtype=torch.int32, device="cuda")
+    s = torch.cuda.current_stream()
+    for _ in range(3):
+        mtp.mtp_viterbi(C5_LATTICES, C5_N, C5_K, V, MODEL.eos_id, t_ids, t_lp, t_q, None, path, None, acc, None, s)
+    torch.cuda.synchronize()
+    w = synth.make_weights(MODEL)
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, 1, 1100)
+    try:
+        ph, ac = synth.make_prompt(0, 64, 225, MODEL.phone_vocab)
+        dec.prefill(0, ph, ac, 750)
+        for _ in range(4):
+            dec.decode_step(4, 4)
+        torch.cuda.synchronize()
+    finally:
+        dec.close()
+    print(json.dumps({"profile_select": "done", "viterbi_calls": 3, "decode_steps": 4}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -658,12 +703,16 @@ def main():
     ap.add_argument("--no-c5", action="store_true", help="skip the isolated heads + Viterbi microbenchmark")
     ap.add_argument("--profile-b32", action="store_true",
                     help="only run a small batch-32 decode for kernel captures (prints no measurement)")
+    ap.add_argument("--profile-select", action="store_true",
+                    help="only run the Viterbi and selection kernels for captures (prints no measurement)")
     args = ap.parse_args()
     if args.oracle_rate_steps:
         value, sample = _oracle_rate(args.oracle_rate_steps)
         print(json.dumps({"value": value, "sample": sample}), flush=True)
     elif args.profile_b32:
         run_profile_b32()
+    elif args.profile_select:
+        run_profile_select()
     elif args.impl == "reference":
         run_reference(args)
     else:

@@ -318,6 +318,14 @@ MTP_API int mtp_step_bytes(mtp_ctx* ctx, int n_heads, uint64_t* out_bytes);
 #define MTP_DEVICE_ERR_WAIT 1
 MTP_API int mtp_selftest_bounded_wait(int32_t* err_word, void* cuda_stream);
 
+/* Self-test of the persistent step kernel's grid barrier bound: one CTA
+ * arrives at a grid barrier that expects two arrivals.  Its poll loop gives up
+ * after its limit (about a second), ORs MTP_DEVICE_ERR_WAIT into *err_word,
+ * and the kernel returns; the barrier's counter is left at zero.
+ *   err_word  int32, device memory
+ * Errors: MTP_ERR_INVALID (null), MTP_ERR_CUDA. */
+MTP_API int mtp_selftest_grid_barrier(int32_t* err_word, void* cuda_stream);
+
 /* ---- stand-alone operators (device pointers, caller's stream) ---------- */
 
 /* Viterbi selection over candidate lattices (Sec. III-C, reading A: the

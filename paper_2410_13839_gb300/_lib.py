@@ -83,6 +83,7 @@ def _load() -> ctypes.CDLL:
         "mtp_viterbi": (i32, [i32, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
         "mtp_heads_topk": (i32, [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]),
         "mtp_selftest_bounded_wait": (i32, [vp, vp]),
+        "mtp_selftest_grid_barrier": (i32, [vp, vp]),
         "mtp_attention_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),
         "mtp_attention": (i32, [ctypes.POINTER(MtpAttentionArgs), vp, sz, vp]),
         "mtp_attention_noalloc": (i32, [ctypes.POINTER(MtpAttentionArgs), vp]),

@@ -171,6 +171,8 @@ int step_ring_stages(int d, int mt);
 // Clusters of SK_CLUSTER CTAs that can be resident at once (the 8-row footprint).
 cudaError_t step_kernel_configure(int d, int* max_clusters);
 cudaError_t launch_step_kernel(const StepArgs& a, int grid, cudaStream_t s, bool pdl);
+// one CTA at a grid barrier that never completes: the bounded wait sets err and returns
+cudaError_t launch_selftest_grid_barrier(int* err, cudaStream_t s);
 
 // --------------------------------------------------------------- embed ----
 struct EmbedArgs {

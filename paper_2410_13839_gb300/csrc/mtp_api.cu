@@ -1649,6 +1649,13 @@ MTP_API int mtp_selftest_bounded_wait(int32_t* err_word, void* cuda_stream) {
     return MTP_OK;
 }
 
+MTP_API int mtp_selftest_grid_barrier(int32_t* err_word, void* cuda_stream) {
+    g_err.clear();
+    if (!err_word) return fail(MTP_ERR_INVALID, "selftest: null error word");
+    CUDA_TRY(launch_selftest_grid_barrier(err_word, static_cast<cudaStream_t>(cuda_stream)));
+    return MTP_OK;
+}
+
 MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden_dtype, int n, int k,
                            int32_t* out_ids, float* out_logp, float* out_logits, float* out_lse) {
     g_err.clear();

@@ -121,11 +121,8 @@ __device__ __forceinline__ void gather_transitions(const int* ids, int n, int k,
 // Viterbi over ids/lp [n][k] with transitions lq [n-1][k][k] and backpointers
 // bp [MAX_NHEADS][32] (all shared memory); lane 0 writes the results.  The
 // selection kernel runs it once per step with a cold instruction cache and
-// keeps the loops rolled (UNROLL = 1: its time follows the instructions it
-// fetches); the stand-alone kernel, warm over many lattices, unrolls the
-// candidate loop (the comparisons stay in order: the lowest i keeps ties).
-template <int UNROLL>
-__device__ void viterbi_warp_t(const int* ids, const float* lp, const float* lq, int n, int k, int* bp, int* path,
+// keeps the loops rolled (its time follows the instructions it fetches).
+__device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, int n, int k, int* bp, int* path,
                                float* score) {
     const int lane = threadIdx.x & 31;
     const bool on = lane < k;
@@ -135,7 +132,7 @@ __device__ void viterbi_warp_t(const int* ids, const float* lp, const float* lq,
         const float* lqt = lq + (size_t)(t - 1) * k * k + (on ? lane : 0);
         float best = 0.f;
         int arg = 0;
-#pragma unroll (UNROLL)
+#pragma unroll 1
         for (int i = 0; i < k; ++i) {
             const float di = __shfl_sync(FULL_MASK, delta, i);
             const float val = __fadd_rn(di, lqt[i * k]);
@@ -415,14 +412,14 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
     } else {
         gather_transitions(s_ids, n, k, a.log_q, a.V, s_lq, threadIdx.x, blockDim.x);
         __syncthreads();
-        if (warp == 0) viterbi_warp_t<1>(s_ids, s_lp, s_lq, n, k, s_bp, s_path, &s_score);
+        if (warp == 0) viterbi_warp(s_ids, s_lp, s_lq, n, k, s_bp, s_path, &s_score);
     }
     __syncthreads();
     trace_mark(a.trace, 1);  // path
     if (warp != 0) return;
 
     // Acceptance and the slot's bookkeeping, one lane per token (short code:
-    // see viterbi_warp_t).
+    // see viterbi_warp).
     const int lane = threadIdx.x & 31;
     const int rem = s_st[2], gc = s_st[3];
     int n_emit;  // tokens this step emits (before the EOS / budget cut), s_emit
@@ -493,39 +490,121 @@ __global__ void __launch_bounds__(256) verify_kernel(const VerifyArgs a) {
     for (int i = threadIdx.x; i < a.d; i += blockDim.x) a.h_last[(size_t)b * a.d + i] = src[i];
 }
 
-// Stand-alone Viterbi: one warp per lattice, VIT_WARPS lattices per block;
-// dynamic shared memory holds each warp's transition table.
-constexpr int VIT_WARPS = 4;
+// Stand-alone Viterbi: a group of KP lanes per lattice (KP = k rounded up to
+// a power of two, 32 / KP lattices per warp), lane j = candidate j.  Each lane
+// loads its own column of the transition scores, lq[i][j] = log_q[c_{t-1,i}][c_{t,j}]
+// for every i, straight into registers: k independent L2 gathers per
+// position, issued one position ahead of the recursion that consumes them, and
+// no shared memory to limit how many warps an SM holds.  The ids of the
+// previous position come from the group's lanes by shuffle.  The recursion,
+// its add order and its tie rules are those of viterbi_warp; acceptance is
+// accept_all's rule (cut after the first EOS and at the remaining budget).
+constexpr int VIT_THREADS = 256;
 
-__global__ void __launch_bounds__(VIT_WARPS * 32) viterbi_kernel(const ViterbiArgs a) {
-    extern __shared__ float vit_lq[];
-    __shared__ int s_ids[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
-    __shared__ float s_lp[VIT_WARPS][MAX_NHEADS * MAX_TOPK];
-    __shared__ int s_path[VIT_WARPS][MAX_NHEADS];
-    __shared__ int s_bp[VIT_WARPS][MAX_NHEADS * 32];
-    __shared__ float s_score[VIT_WARPS];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.x * VIT_WARPS + warp;
-    if (b >= a.batch) return;  // whole warp leaves together
-    const int nk = a.n * a.k;
-    for (int i = lane; i < nk; i += 32) {
-        s_ids[warp][i] = a.cand_ids[(size_t)b * nk + i];
-        s_lp[warp][i] = a.cand_logp[(size_t)b * nk + i];
+template <int KP>
+__device__ __forceinline__ void vit_load_column(const ViterbiArgs& a, int id_prev, int id_cur, bool on,
+                                                float* q) {
+    const int V = a.vocab;
+    const bool cj_ok = on && id_cur >= 0 && id_cur < V;
+#pragma unroll
+    for (int i = 0; i < KP; ++i) {
+        const int ci = __shfl_sync(FULL_MASK, id_prev, i, KP);
+        q[i] = (cj_ok && i < a.k && ci >= 0 && ci < V) ? __ldg(a.log_q + (size_t)ci * V + id_cur) : -INFINITY;
     }
-    __syncwarp();
-    float* lq = vit_lq + (size_t)warp * (a.n - 1) * a.k * a.k;
-    gather_transitions(s_ids[warp], a.n, a.k, a.log_q, a.vocab, lq, lane, 32);
-    __syncwarp();
-    viterbi_warp_t<4>(s_ids[warp], s_lp[warp], lq, a.n, a.k, s_bp[warp], s_path[warp], &s_score[warp]);
-    __syncwarp();
-    if (lane != 0) return;
-    int acc, done;
-    const int rem = a.remaining ? a.remaining[b] : a.n;
-    accept_all(s_path[warp], a.n, a.eos_id, rem, acc, done);
-    for (int t = 0; t < a.n; ++t) a.path[(size_t)b * a.n + t] = s_path[warp][t];
-    if (a.score) a.score[b] = s_score[warp];
+}
+
+template <int KP>
+__global__ void __launch_bounds__(VIT_THREADS, KP >= 32 ? 2 : 4) viterbi_kernel(const ViterbiArgs a) {
+    constexpr int G = 32 / KP;  // lattices per warp
+    const int lane = threadIdx.x & 31, j = lane & (KP - 1);
+    const int b = (blockIdx.x * (VIT_THREADS / 32) + (threadIdx.x >> 5)) * G + lane / KP;
+    const bool live = b < a.batch;  // the whole warp stays for the shuffles
+    const int n = a.n, k = a.k;
+    const bool on = live && j < k;
+    int id[MAX_NHEADS];
+    float lp[MAX_NHEADS];
+#pragma unroll
+    for (int t = 0; t < MAX_NHEADS; ++t) {
+        id[t] = -1;
+        lp[t] = -INFINITY;
+        if (on && t < n) {
+            id[t] = a.cand_ids[((size_t)b * n + t) * k + j];
+            lp[t] = a.cand_logp[((size_t)b * n + t) * k + j];
+        }
+    }
+    float qa[KP], qb[KP];
+    int bp[MAX_NHEADS];
+    if (n > 1) vit_load_column<KP>(a, id[0], id[1], on, qa);
+    float delta = on ? lp[0] : -INFINITY;
+#pragma unroll
+    for (int t = 1; t < MAX_NHEADS; ++t) {
+        bp[t] = 0;
+        if (t < n) {
+            float* cur = (t & 1) ? qa : qb;
+            if (t + 1 < n) vit_load_column<KP>(a, id[t], id[t + 1], on, (t & 1) ? qb : qa);
+            float best = 0.f;
+            int arg = 0;
+#pragma unroll
+            for (int i = 0; i < KP; ++i) {
+                const float di = __shfl_sync(FULL_MASK, delta, i, KP);
+                if (i < k) {
+                    const float val = __fadd_rn(di, cur[i]);
+                    if (i == 0 || val > best) {
+                        best = val;
+                        arg = i;
+                    }
+                }
+            }
+            delta = on ? __fadd_rn(best, lp[t]) : -INFINITY;
+            bp[t] = arg;
+        }
+    }
+    // best final state: the lowest j of the maximum, within the group
+    float bv = delta;
+    int bj = on ? j : 0x7fffffff;
+#pragma unroll
+    for (int o = KP / 2; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(FULL_MASK, bv, o);
+        const int oi = __shfl_xor_sync(FULL_MASK, bj, o);
+        if (ov > bv || (ov == bv && oi < bj)) {
+            bv = ov;
+            bj = oi;
+        }
+    }
+    int state = live ? bj : 0;
+    int path[MAX_NHEADS];
+#pragma unroll
+    for (int t = MAX_NHEADS - 1; t >= 0; --t) {
+        path[t] = -1;
+        if (t < n) {
+            path[t] = __shfl_sync(FULL_MASK, id[t], state, KP);
+            if (t > 0) state = __shfl_sync(FULL_MASK, bp[t], state, KP);
+        }
+    }
+    if (!live || j != 0) return;
+    int acc = n;
+    bool cut = false;
+#pragma unroll
+    for (int t = 0; t < MAX_NHEADS; ++t)
+        if (t < n && !cut && path[t] == a.eos_id) {
+            acc = t + 1;
+            cut = true;
+        }
+    const int rem = a.remaining ? a.remaining[b] : n;
+    acc = min(acc, max(rem, 0));
+#pragma unroll
+    for (int t = 0; t < MAX_NHEADS; ++t)
+        if (t < n) a.path[(size_t)b * n + t] = path[t];
+    if (a.score) a.score[b] = bv;
     a.accepted[b] = acc;
     if (a.rollback) a.rollback[b] = 0;
+}
+
+template <int KP>
+cudaError_t launch_viterbi_kp(const ViterbiArgs& a, cudaStream_t s) {
+    constexpr int per_block = VIT_THREADS / 32 * (32 / KP);
+    viterbi_kernel<KP><<<(a.batch + per_block - 1) / per_block, VIT_THREADS, 0, s>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -562,12 +641,12 @@ cudaError_t launch_verify(const VerifyArgs& a, int slots, cudaStream_t s, bool p
 cudaError_t launch_viterbi(const ViterbiArgs& a, cudaStream_t s) {
     if (a.n < 1 || a.n > MAX_NHEADS || a.k < 1 || a.k > MAX_TOPK || a.batch < 0) return cudaErrorInvalidValue;
     if (a.batch == 0) return cudaSuccess;
-    const size_t smem = (size_t)VIT_WARPS * (a.n - 1) * a.k * a.k * sizeof(float);
-    cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(viterbi_kernel),
-                                       (size_t)VIT_WARPS * (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK * sizeof(float));
-    if (e != cudaSuccess) return e;
-    viterbi_kernel<<<(a.batch + VIT_WARPS - 1) / VIT_WARPS, VIT_WARPS * 32, smem, s>>>(a);
-    return cudaGetLastError();
+    if (a.k <= 1) return launch_viterbi_kp<1>(a, s);
+    if (a.k <= 2) return launch_viterbi_kp<2>(a, s);
+    if (a.k <= 4) return launch_viterbi_kp<4>(a, s);
+    if (a.k <= 8) return launch_viterbi_kp<8>(a, s);
+    if (a.k <= 16) return launch_viterbi_kp<16>(a, s);
+    return launch_viterbi_kp<32>(a, s);
 }
 
 }  // namespace mtp

@@ -1309,6 +1309,20 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(THREADS, 1) step_ke
     }
 }
 
+// Self-test of the grid barrier's bound: the one CTA of the launch waits for
+// two arrivals, only its own comes, the wait gives up after its poll limit,
+// sets the error word and the CTA returns.  The counter is reset on the way out.
+__device__ unsigned g_selftest_grid_ctr;
+
+__global__ void __launch_bounds__(THREADS) selftest_grid_kernel(int* err) {
+    __shared__ int s_abort;
+    if (threadIdx.x == 0) s_abort = 0;
+    __syncthreads();
+    if (threadIdx.x >= NTHREADS) return;  // the producer warp takes no part in grid barriers
+    grid_sync(&g_selftest_grid_ctr, 2u, err, &s_abort);
+    if (threadIdx.x == 0) atomicExch(&g_selftest_grid_ctr, 0u);
+}
+
 }  // namespace
 
 int step_ring_stages(int d, int mt) {
@@ -1366,6 +1380,11 @@ cudaError_t launch_step_kernel(const StepArgs& a, int grid, cudaStream_t s, bool
     if (a.rows <= 2) return launch_step_t<2>(a, grid, s, pdl);
     if (a.rows <= 4) return launch_step_t<4>(a, grid, s, pdl);
     return launch_step_t<8>(a, grid, s, pdl);
+}
+
+cudaError_t launch_selftest_grid_barrier(int* err, cudaStream_t s) {
+    selftest_grid_kernel<<<1, THREADS, 0, s>>>(err);
+    return cudaGetLastError();
 }
 
 }  // namespace mtp

@@ -196,6 +196,11 @@ def mtp_selftest_bounded_wait(err_word, stream=None) -> None:
     check(lib.mtp_selftest_bounded_wait(_ptr(err_word), _stream_handle(stream)))
 
 
+def mtp_selftest_grid_barrier(err_word, stream=None) -> None:
+    """One CTA at a grid barrier that never completes; its bounded wait sets err_word."""
+    check(lib.mtp_selftest_grid_barrier(_ptr(err_word), _stream_handle(stream)))
+
+
 def mtp_heads_topk(ctx, batch, hidden, hidden_dtype, n_heads, top_k, out_ids, out_logp,
                    out_logits=None, out_lse=None) -> None:
     check(lib.mtp_heads_topk(ctx, batch, _ptr(hidden), hidden_dtype, n_heads, top_k, _ptr(out_ids),
