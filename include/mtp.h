@@ -244,6 +244,10 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        and cached keys streamed into shared-memory rings ahead of use, bounded grid
  *                        barriers between the attention and MLP phases), where the model and GPU
  *                        allow it; 0 = two block kernels per layer (default: faster on GB300 at B = 1)
+ *   MTP_OPT_PREFILL_TC   1 = prefill passes (mtp_prefill, mtp_prefill_pending) run their attention
+ *                        on the tensor cores (tcgen05: tiles of 128 prompt rows, 128-key items, S and
+ *                        P V accumulated in TMEM; default); 0 = the split-key kernel of the decode
+ *                        steps, in groups of 8 rows
  *   MTP_OPT_SEED         seed of the path draws (any 32-bit value, zero-extended; default 0).
  *                        Position t of a draw of slot b that has generated g tokens uses the
  *                        uniform (SplitMix64(x) >> 40) / 2^24, x = ((seed * P + b) * P + g) * P + t
@@ -252,7 +256,7 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
     MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8,
-    MTP_OPT_PERSISTENT = 9
+    MTP_OPT_PERSISTENT = 9, MTP_OPT_PREFILL_TC = 10
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);
@@ -278,7 +282,7 @@ typedef enum mtp_kernel_kind {
     MTP_K_EMBED = 0, MTP_K_ATTN_BLOCK = 1, MTP_K_MLP = 2, MTP_K_HEADS = 3, MTP_K_SELECT = 4,
     MTP_K_SAVE = 5, MTP_K_PACK = 6, MTP_K_GEMM = 7, MTP_K_QKV = 8, MTP_K_ATTN = 9, MTP_K_STEP = 10,
     MTP_K_STEP_ATTN = 11, MTP_K_STEP_MLP = 12,
-    MTP_K_STEP_CTA = 13, MTP_K_COUNT = 14
+    MTP_K_STEP_CTA = 13, MTP_K_ATTN_TC = 14, MTP_K_COUNT = 15
 } mtp_kernel_kind;
 
 /* Run one decode step with each kernel launched alone (no graph, no PDL)
@@ -388,6 +392,24 @@ typedef struct mtp_attention_args {
 MTP_API size_t mtp_attention_workspace_bytes(const mtp_attention_args* args);
 MTP_API int mtp_attention(const mtp_attention_args* args, void* workspace, size_t workspace_bytes,
                           void* cuda_stream);
+
+/* The same attention on the tensor cores (tcgen05), as prefill passes run it
+ * (Sec. III-A: every prompt position attends to itself and the positions before
+ * it).  Rows form tiles of 128 (rows_per_group is not used); the rows of a tile
+ * may belong to any slots, each row sees keys 0..row_pos of its own slot.  Per
+ * tile, head and 128 cached keys: S = Q K^T and O = P V on the tensor cores
+ * with fp32 accumulators in TMEM (Q and P as bf16 hi + lo pairs), the online
+ * softmax in registers; key ranges split across CTAs are merged with a
+ * log-sum-exp.  The pool must hold each key and value row in the context's
+ * cache layout: 16-byte chunk c of row t of a page at chunk position
+ * c ^ (t mod 8).  Other arguments and layouts as mtp_attention; row_seq < 0 rows
+ * are left untouched.  workspace: mtp_attention_tc_workspace_bytes(args) bytes,
+ * counters zero on the first call and left zero.
+ * Errors: MTP_ERR_INVALID (sizes, null pointers, workspace too small, q not
+ * 16-byte aligned), MTP_ERR_CUDA. */
+MTP_API size_t mtp_attention_tc_workspace_bytes(const mtp_attention_args* args);
+MTP_API int mtp_attention_tc(const mtp_attention_args* args, void* workspace, size_t workspace_bytes,
+                             void* cuda_stream);
 
 /* mtp_attention without a caller workspace and without any allocation.  The
  * paper has no counterpart: this serves callers that must not allocate GPU

@@ -31,7 +31,7 @@ MTP_OPT_LATTICE = 6
 MTP_OPT_SAMPLING = 7
 MTP_OPT_SEED = 8
 KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save", "pack", "gemm", "qkv", "attn", "step", "step_attn",
-                "step_mlp", "step_cta")
+                "step_mlp", "step_cta", "attn_tc")
 
 
 class MtpConfig(ctypes.Structure):
@@ -87,6 +87,8 @@ def _load() -> ctypes.CDLL:
         "mtp_attention_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),
         "mtp_attention": (i32, [ctypes.POINTER(MtpAttentionArgs), vp, sz, vp]),
         "mtp_attention_noalloc": (i32, [ctypes.POINTER(MtpAttentionArgs), vp]),
+        "mtp_attention_tc_workspace_bytes": (sz, [ctypes.POINTER(MtpAttentionArgs)]),
+        "mtp_attention_tc": (i32, [ctypes.POINTER(MtpAttentionArgs), vp, sz, vp]),
         "mtp_gemm_bf16x2": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, vp]),
     }
     for name, (res, args) in sig.items():

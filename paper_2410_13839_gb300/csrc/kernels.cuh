@@ -79,12 +79,19 @@ struct AttnArgs {
     int* err;
     unsigned long long* trace;
     int kv_swizzled;                                         // pages store chunk c of key row t at c ^ (t & 7)
+    int rows;                                                // attention_tc: rows of the pass (tiles of 128)
 };
 
 size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
 size_t attn_smem_bytes(int page_size);
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms);
 cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl);
+// Tensor-core (tcgen05) causal attention of prompt rows: tiles of 128 rows of
+// any slots, 128-key items, swizzled pages only; grid (n_splits, heads, tiles).
+size_t attn_tc_workspace_floats(int tiles, int n_heads, int n_splits);
+int attn_tc_tiles(int rows);
+int attn_tc_splits_for(int tiles, int n_heads, int max_keys, int num_sms);
+cudaError_t launch_attention_tc(const AttnArgs& a, cudaStream_t s, bool pdl);
 
 // ------------------------------------------------------- fused block ----
 // One transformer block over <= MAX_ROWS fed rows: attn_block (LN1, q|k|v,

@@ -114,6 +114,7 @@ struct mtp_ctx {
     int device = 0, num_sms = 0, wbytes = 2;
     int mlp_clusters = 1;  // MLP clusters co-resident in one wave
     bool use_graphs = true, use_pdl = true, use_l2_prefetch = false;
+    bool use_attn_tc = true;  // prefill passes: tensor-core attention
     std::vector<void*> allocs;
     // weights
     void* d_weights = nullptr;
@@ -322,8 +323,11 @@ int tile_index(int nt) { return nt == 32 ? 0 : (nt == 64 ? 1 : 2); }
 // projections plus row-wise kernels; the final hidden rows stay in d_bx.
 // Attention groups: `groups` runs of rpg rows, each of one slot (decode:
 // slot b's fed rows b*n.., plan PLAN_DEVICE; prefill: 8 consecutive prompt
-// positions, plan PLAN_ROWS).
-int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStream_t s, bool pdl, Prof* prof) {
+// positions, plan PLAN_ROWS).  prefill_keys > 0: a prefill pass whose rows see
+// at most that many keys; its attention runs on the tensor cores (tiles of 128
+// rows) unless that option is off.
+int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStream_t s, bool pdl, Prof* prof,
+                       int prefill_keys = 0) {
     const mtp_config& cf = c->cfg;
     const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size;
     // activation tiles: a weight tile is streamed once per activation tile.  32-row
@@ -387,8 +391,19 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         at.n_splits = std::max(1, at.n_splits);
         at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = 0;
         at.err = c->d_err; at.kv_swizzled = 1;
-        at.trace = tslot(c, MTP_K_ATTN);
-        LAUNCH(MTP_K_ATTN, launch_attention(at, groups, s, pdl));
+        if (prefill_keys > 0 && c->use_attn_tc && plan == PLAN_ROWS) {
+            // tiles of 128 rows; splits as many as the batched attention workspace holds (S = 1 uses none)
+            const int tiles = attn_tc_tiles(M);
+            const size_t ws_floats = attn_workspace_floats(c->battn_ws_units, H, 1, MAX_ROWS);
+            at.rows = M;
+            at.n_splits = std::max(1, std::min(attn_tc_splits_for(tiles, H, prefill_keys, c->num_sms),
+                                               (int)(ws_floats / attn_tc_workspace_floats(tiles, H, 1))));
+            at.trace = tslot(c, MTP_K_ATTN_TC);
+            LAUNCH(MTP_K_ATTN_TC, launch_attention_tc(at, s, pdl));
+        } else {
+            at.trace = tslot(c, MTP_K_ATTN);
+            LAUNCH(MTP_K_ATTN, launch_attention(at, groups, s, pdl));
+        }
         // x += attention W_o^T + b_o (the per-head W_o blocks are the k-chunks)
         MTP_TRY(gemm(W.wo, d, d, false, TC_ACCUM, c->d_bx, d, L.bo, d));
         // x += GELU(LN2(x) W1^T + b1) W2^T + b2 (W1's epilogue writes the GELU rows as bf16 hi + lo)
@@ -1231,6 +1246,8 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
     } else if (option == MTP_OPT_PERSISTENT) {
         changed = c->use_persistent != (value != 0);
         c->use_persistent = value != 0;
+    } else if (option == MTP_OPT_PREFILL_TC) {
+        c->use_attn_tc = value != 0;  // prefill passes are not captured
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -1272,6 +1289,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_SAMPLING: *value = c->sampling; break;
         case MTP_OPT_SEED: *value = (int32_t)c->sample_seed; break;
         case MTP_OPT_PERSISTENT: *value = c->use_persistent && c->sk_ok; break;
+        case MTP_OPT_PREFILL_TC: *value = c->use_attn_tc; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;
@@ -1342,7 +1360,7 @@ MTP_API int mtp_prefill(mtp_ctx* c, int slot, const int32_t* phonemes, int n_ph,
             e.mode = 1; e.rows = m; e.slot = slot; e.p0 = p0; e.n_ph = n_ph; e.total = (int)T;
             e.x = c->d_bx; e.zero_buf = nullptr;
             LAUNCH(MTP_K_EMBED, launch_embed(e, s, false));
-            MTP_TRY(run_layers_batched(c, rows, 8, rows / 8, PLAN_ROWS, s, c->use_pdl, prof));
+            MTP_TRY(run_layers_batched(c, rows, 8, rows / 8, PLAN_ROWS, s, c->use_pdl, prof, p0 + m));
             LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, rows,
                                                 nullptr, s, c->use_pdl));
         }
@@ -1404,7 +1422,7 @@ MTP_API int mtp_prefill_pending(mtp_ctx* c) {
     int passes = 0;
     while (lane_pending(c)) {
         MTP_TRY(enqueue_lane_plan(c, 0, P, 8, s, c->use_pdl, nullptr));
-        MTP_TRY(run_layers_batched(c, P, 8, P / 8, PLAN_ROWS, s, c->use_pdl, nullptr));
+        MTP_TRY(run_layers_batched(c, P, 8, P / 8, PLAN_ROWS, s, c->use_pdl, nullptr, cf.max_ctx));
         Prof* prof = nullptr;
         LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, cf.d_model, P, nullptr, s,
                                             c->use_pdl));
@@ -1720,6 +1738,68 @@ MTP_API int mtp_attention(const mtp_attention_args* a, void* workspace, size_t w
     if (workspace_bytes < p.need)
         return fail(MTP_ERR_INVALID, "attention: workspace %zu bytes, need %zu", workspace_bytes, p.need);
     return attention_standalone_launch(a, p, workspace, static_cast<cudaStream_t>(cuda_stream));
+}
+
+}  // extern "C"
+
+namespace {
+// Tiles, splits and workspace of mtp_attention_tc (sizes as mtp_attention; rows_per_group unused).
+int attention_tc_plan(const mtp_attention_args* a, bool check_pointers, AttnStandalonePlan* p) {
+    if (!a || a->rows < 1 || a->n_heads < 1 ||
+        (a->page_size != 16 && a->page_size != 32 && a->page_size != 64 && a->page_size != 128) || a->layers < 1 ||
+        a->layer < 0 || a->layer >= a->layers || a->bt_stride < 1 || a->max_keys < 1)
+        return fail(MTP_ERR_INVALID, "attention_tc: invalid sizes");
+    if (check_pointers && (!a->q || !a->kv_pool || !a->block_table || !a->row_seq || !a->row_pos || !a->out))
+        return fail(MTP_ERR_INVALID, "attention_tc: null pointer");
+    if (check_pointers && (reinterpret_cast<uintptr_t>(a->q) & 15))
+        return fail(MTP_ERR_INVALID, "attention_tc: q must be 16-byte aligned");
+    int dev = 0, sms = 0;
+    CUDA_TRY(cudaGetDevice(&dev));
+    CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    p->groups = attn_tc_tiles(a->rows);
+    p->splits = attn_tc_splits_for(p->groups, a->n_heads, a->max_keys, sms);
+    p->part_bytes = align256(attn_tc_workspace_floats(p->groups, a->n_heads, p->splits) * sizeof(float));
+    p->count_bytes = align256((size_t)p->groups * a->n_heads * sizeof(int));
+    p->need = p->part_bytes + p->count_bytes;
+    return MTP_OK;
+}
+}  // namespace
+
+extern "C" {
+
+MTP_API size_t mtp_attention_tc_workspace_bytes(const mtp_attention_args* a) {
+    AttnStandalonePlan p;
+    const std::string keep = g_err;  // a size query leaves the last error alone
+    const int r = attention_tc_plan(a, false, &p);
+    g_err = keep;
+    return r == MTP_OK ? p.need : 0;
+}
+
+MTP_API int mtp_attention_tc(const mtp_attention_args* a, void* workspace, size_t workspace_bytes,
+                             void* cuda_stream) {
+    g_err.clear();
+    AttnStandalonePlan p;
+    MTP_TRY(attention_tc_plan(a, true, &p));
+    if (!workspace) return fail(MTP_ERR_INVALID, "attention_tc: null workspace");
+    if (workspace_bytes < p.need)
+        return fail(MTP_ERR_INVALID, "attention_tc: workspace %zu bytes, need %zu", workspace_bytes, p.need);
+    AttnArgs at;
+    std::memset(&at, 0, sizeof(at));
+    const int d = a->n_heads * HEAD_DIM;
+    at.q = a->q; at.ldq = d;
+    at.kv_pool = reinterpret_cast<const __nv_bfloat16*>(a->kv_pool);
+    at.page_elems = (long long)a->layers * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.layer_off = (long long)a->layer * 2 * a->n_heads * a->page_size * HEAD_DIM;
+    at.block_table = a->block_table; at.bt_stride = a->bt_stride;
+    at.row_seq = a->row_seq; at.row_pos = a->row_pos;
+    at.out = a->out; at.ldo = d;
+    at.ws_part = static_cast<float*>(workspace);
+    at.ws_count = reinterpret_cast<int*>(static_cast<char*>(workspace) + p.part_bytes);
+    at.rows = a->rows; at.n_heads = a->n_heads; at.page_size = a->page_size;
+    at.n_splits = p.splits; at.plan = PLAN_ROWS; at.kv_swizzled = 1;
+    at.err = nullptr;
+    CUDA_TRY(launch_attention_tc(at, static_cast<cudaStream_t>(cuda_stream), false));
+    return MTP_OK;
 }
 
 }  // extern "C"

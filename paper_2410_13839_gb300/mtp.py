@@ -223,6 +223,15 @@ def mtp_attention(args: MtpAttentionArgs, workspace, workspace_bytes: int, strea
     check(lib.mtp_attention(ctypes.byref(args), _ptr(workspace), workspace_bytes, _stream_handle(stream)))
 
 
+def mtp_attention_tc_workspace_bytes(args: MtpAttentionArgs) -> int:
+    return int(lib.mtp_attention_tc_workspace_bytes(ctypes.byref(args)))
+
+
+def mtp_attention_tc(args: MtpAttentionArgs, workspace, workspace_bytes: int, stream=None) -> None:
+    """Tensor-core attention of prompt rows (tiles of 128 rows); the pool in the cache's swizzled layout."""
+    check(lib.mtp_attention_tc(ctypes.byref(args), _ptr(workspace), workspace_bytes, _stream_handle(stream)))
+
+
 def mtp_attention_noalloc(args: MtpAttentionArgs, stream=None) -> None:
     """mtp_attention with the library's fixed scratch array: no workspace, no allocation."""
     check(lib.mtp_attention_noalloc(ctypes.byref(args), _stream_handle(stream)))
