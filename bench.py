@@ -235,26 +235,31 @@ def c5_lattices(count: int, n: int, k: int, vocab: int, seed: int = 5):
     return ids, lp
 
 
-def run_c5(mtp, ctx, stream):
+def run_c5(mtp, stream):
     """The isolated head + Viterbi microbenchmark: n=8 heads with log-softmax and top-16
-    on 256 bf16 hidden rows N(0,1) (the context's VALL-E-sized heads), and Viterbi with
-    acceptance over 10^4 lattices of 8 positions x 16 candidates.  CUDA events, 3 warm-up
-    calls; head bytes = the 8 heads' weights once per call."""
+    on 256 bf16 hidden rows N(0,1) (VALL-E-sized heads, in a context whose row buffers
+    hold all 256 rows: one heads launch per call), and Viterbi with acceptance over 10^4
+    lattices of 8 positions x 16 candidates.  CUDA events, 3 warm-up calls; head bytes =
+    the 8 heads' weights once per call.  The heads call asks for the candidates and lse
+    only (the logits stay on chip)."""
     import torch
     d, V = MODEL.d_model, MODEL.codec_vocab
+    w = synth.make_weights(MODEL)
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, C5_BATCH // MODEL.n_heads_max, 64,
+                         stream=stream)
+    ctx = dec.ctx
     h = torch.from_numpy(synth.make_hidden(C5_BATCH, d, seed=C5_BATCH)).cuda().to(torch.bfloat16)
     ids = torch.zeros((C5_BATCH, C5_N, C5_K), dtype=torch.int32, device="cuda")
     lp = torch.zeros((C5_BATCH, C5_N, C5_K), dtype=torch.float32, device="cuda")
-    lg = torch.zeros((C5_BATCH, C5_N, V), dtype=torch.float32, device="cuda")
     lse = torch.zeros((C5_BATCH, C5_N), dtype=torch.float32, device="cuda")
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
     calls = 20
     for _ in range(3):
-        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, lg, lse)
+        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, None, lse)
     torch.cuda.synchronize()
     ev[0].record(stream)
     for _ in range(calls):
-        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, lg, lse)
+        mtp.mtp_heads_topk(ctx, C5_BATCH, h, 1, C5_N, C5_K, ids, lp, None, lse)
     ev[1].record(stream)
     torch.cuda.synchronize()
     heads_s = ev[0].elapsed_time(ev[1]) / 1e3 / calls
@@ -273,13 +278,23 @@ def run_c5(mtp, ctx, stream):
     ev[3].record(vs)
     torch.cuda.synchronize()
     vit_s = ev[2].elapsed_time(ev[3]) / 1e3 / calls
+    dec.close()
     head_bytes = C5_N * V * d * 2
+    # algorithmic bytes of one heads call: the head weights and biases, the hidden rows (bf16),
+    # the candidates (ids + logp) and lse written
+    call_bytes = head_bytes + C5_N * V * 4 + C5_BATCH * d * 2 + C5_BATCH * C5_N * (C5_K * 8 + 4)
     flops = 2.0 * C5_BATCH * C5_N * V * d
     gathers = C5_LATTICES * (C5_N - 1) * C5_K * C5_K
+    peak, peak_src = _peaks()
     return {"workload": "isolated heads + Viterbi: 256 bf16 hidden rows N(0,1), n=8 heads x V=1025 with "
                         "log-softmax and top-16; Viterbi + acceptance over 10^4 lattices of 8 x 16",
             "heads_topk_us": heads_s * 1e6, "heads_gbs": head_bytes / heads_s / 1e9,
-            "heads_tflops": flops / heads_s / 1e12, "viterbi_us": vit_s * 1e6,
+            "heads_tflops": flops / heads_s / 1e12,
+            "heads_roofline": {"bound": "hbm", "achieved": call_bytes / heads_s / 1e9, "peak": peak,
+                               "unit": "GB/s", "frac": call_bytes / heads_s / 1e9 / peak,
+                               "peak_source": peak_src, "algorithmic_bytes_per_call": call_bytes,
+                               "note": "one call = row conversion, LN_f pack and the fused heads kernel"},
+            "viterbi_us": vit_s * 1e6,
             "viterbi_lattices_per_s": C5_LATTICES / vit_s,
             "viterbi_roofline": {
                 "bound": "l2_tag_requests", "achieved": gathers / vit_s / 1e9, "peak": L2_TAG_REQUESTS_PEAK,
@@ -621,7 +636,7 @@ def run_ours(args):
             "step_timeline": {"span_us": step_span_us, "kinds": timeline,
                               "timing": "one graph-launched decode step, %globaltimer (mtp_trace_step)"}}
     if not args.no_c5:
-        line["c5"] = run_c5(mtp, ctx, stream)
+        line["c5"] = run_c5(mtp, stream)
     dec.close()
     if not args.no_b32:
         line["b32"] = run_b32(mtp, stream, max(1, min(args.warmup, 2)), max(1, min(args.steps, 3)), interleaved=True)

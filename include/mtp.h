@@ -248,6 +248,11 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        on the tensor cores (tcgen05: tiles of 128 prompt rows, 128-key items, S and
  *                        P V accumulated in TMEM; default); 0 = the split-key kernel of the decode
  *                        steps, in groups of 8 rows
+ *   MTP_OPT_HEADS_FUSED  1 = more than 8 hidden rows (batched decode steps, mtp_heads_topk) run the
+ *                        heads, log-softmax and top-k as one tensor-core kernel (LN_f rows as bf16
+ *                        hi + lo; per (tile of 128 rows, head) a cluster of 8 CTAs over vocabulary
+ *                        slices, lse merged in the cluster before the top-k; default); 0 = heads GEMM
+ *                        into memory, then the selection kernel's top-k
  *   MTP_OPT_SEED         seed of the path draws (any 32-bit value, zero-extended; default 0).
  *                        Position t of a draw of slot b that has generated g tokens uses the
  *                        uniform (SplitMix64(x) >> 40) / 2^24, x = ((seed * P + b) * P + g) * P + t
@@ -256,7 +261,7 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
     MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8,
-    MTP_OPT_PERSISTENT = 9, MTP_OPT_PREFILL_TC = 10
+    MTP_OPT_PERSISTENT = 9, MTP_OPT_PREFILL_TC = 10, MTP_OPT_HEADS_FUSED = 11
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);

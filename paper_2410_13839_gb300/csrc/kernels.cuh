@@ -242,6 +242,7 @@ struct SelectArgs {
     const int* prompt_left;   // slots with prompt tokens left select nothing (null: no admitted prompts)
     const int* lane_take;     // with `lane`: slots whose prompt rows ran in this step's lane select nothing
     int lane;
+    int pre_topk;             // 1: cand_ids / cand_logp / lse already hold the step's top-k (fused heads)
 };
 cudaError_t launch_select(const SelectArgs& a, int batch, bool do_accept, cudaStream_t s, bool pdl);
 
@@ -335,6 +336,31 @@ int tc_encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t ro
                  bool pre_swizzled);
 int tc_tile_rows(int m);          // activation rows per tile for m rows: 32, 64 or 128
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl);
+
+// ------------------------------------ fused heads + log-softmax + top-k ----
+// The n heads over m rows of LN_f(h) given as bf16 hi + lo (heads_tc.cu): per
+// (row, head) the lse and the top-k of logp = logit - lse by (logp desc, id
+// asc); logits to memory only on request.
+struct HeadsTcArgs {
+    const float* bias;            // [n_max * V]
+    int m, n, V, k;               // rows, heads, vocabulary, candidates
+    int k_chunks;                 // d / 64
+    int a_rows;                   // rows of the activation box: 32 or 64 (m <= that), else 128
+    int32_t* out_ids; float* out_logp;   // [m][n][k]
+    float* out_lse;               // [m][n] or null
+    float* out_logits; int ldl;   // [m][ldl], head i at column i * V, or null
+    float z;                      // set by launch_heads_tc: candidates are logp >= mean + z sd of the row (pruning)
+    int* err;
+    unsigned long long* trace;
+};
+struct HeadsTc {
+    CUtensorMap w128, w144;       // head weight rows [n_max * V][d]: boxes of 64 x 128 and 64 x 144 rows
+    CUtensorMap a_hi, a_lo;       // LN_f rows: boxes of 64 x a_rows rows
+    HeadsTcArgs args;
+};
+bool heads_tc_supported(int V, int k);
+int heads_tc_box_rows_wide();
+cudaError_t launch_heads_tc(const HeadsTc& g, cudaStream_t s, bool pdl);
 
 // Raise `kernel`'s dynamic shared-memory limit to at least `bytes` on the
 // current device (and, with max_shared_carveout, prefer the whole unified L1

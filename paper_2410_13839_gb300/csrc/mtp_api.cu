@@ -115,6 +115,7 @@ struct mtp_ctx {
     int mlp_clusters = 1;  // MLP clusters co-resident in one wave
     bool use_graphs = true, use_pdl = true, use_l2_prefetch = false;
     bool use_attn_tc = true;  // prefill passes: tensor-core attention
+    bool use_heads_tc = true;  // more than 8 rows: heads, log-softmax and top-k in one tensor-core kernel
     std::vector<void*> allocs;
     // weights
     void* d_weights = nullptr;
@@ -140,6 +141,8 @@ struct mtp_ctx {
     };
     std::vector<LayerMaps> lmaps;
     CUtensorMap heads_map;  // the heads [n_heads_max * V][d] as GEMM weights (batched decode)
+    CUtensorMap heads_map144;  // the same rows in boxes of 144 (the fused heads' last vocabulary slice)
+    bool heads_tc_ok = false;  // the fused heads kernel serves this model (tensor maps, vocabulary size)
     CUtensorMap amap_hi[3], amap_lo[3], umap_hi[3], umap_lo[3];  // activation tiles of 32, 64, 128 rows
     float* d_pe = nullptr;
     // KV cache
@@ -559,6 +562,10 @@ int setup_batched(mtp_ctx* c) {
     }
     bad |= tc_encode_2d(&c->heads_map, c->w_heads, (uint64_t)d, (uint64_t)cf.n_heads_max * cf.codec_vocab, 128,
                         false);
+    c->heads_tc_ok = tc_encode_2d(&c->heads_map144, c->w_heads, (uint64_t)d,
+                                  (uint64_t)cf.n_heads_max * cf.codec_vocab, (uint32_t)heads_tc_box_rows_wide(),
+                                  false) == 0 &&
+                     heads_tc_supported(cf.codec_vocab, 1);
     c->batched_ok = bad == 0;  // without tensor maps the fused path serves every batch
     return MTP_OK;
 }
@@ -611,6 +618,38 @@ int launch_heads_batched(mtp_ctx* c, const float* x, int B, int n, float* logits
     ga.k_chunks = chunks / splits; ga.epilogue = TC_ACCUM; ga.n_valid = n * V; ga.err = c->d_err;
     ga.trace = tslot(c, MTP_K_HEADS);
     LAUNCH(MTP_K_HEADS, launch_tc_gemm(g, s, pdl));
+    return MTP_OK;
+}
+
+bool heads_fused_ok(const mtp_ctx* c, int k) {
+    return c->use_heads_tc && c->batched_ok && c->heads_tc_ok && heads_tc_supported(c->cfg.codec_vocab, k);
+}
+
+// The heads fused with their log-softmax and top-k over B hidden rows x [B][d]
+// (B <= the batched buffers' rows): LN_f rows as bf16 hi + lo, then one kernel
+// that writes the candidates (ids, logp [B][n][k]), lse [B][n] and, when
+// `logits` is not null, the logits [B][n V].
+int launch_heads_fused(mtp_ctx* c, const float* x, int B, int n, int k, int32_t* ids, float* logp, float* lse,
+                       float* logits, cudaStream_t s, bool pdl, Prof* prof) {
+    const mtp_config& cf = c->cfg;
+    const int d = cf.d_model, V = cf.codec_vocab;
+    PackArgs pa;
+    std::memset(&pa, 0, sizeof(pa));
+    pa.mode = PACK_LN; pa.x = x; pa.ldx = d; pa.gamma = c->lnf_g; pa.beta = c->lnf_b;
+    pa.eps = cf.ln_eps; pa.row_seq = nullptr; pa.hi = c->d_ahi; pa.lo = c->d_alo; pa.k = d; pa.m = B;
+    pa.trace = tslot(c, MTP_K_PACK);
+    LAUNCH(MTP_K_PACK, launch_pack_rows(pa, s, pdl));
+    HeadsTc g;
+    std::memset(&g, 0, sizeof(g));
+    g.w128 = c->heads_map; g.w144 = c->heads_map144;
+    const int ar = tc_tile_rows(B);  // 32, 64 or 128 activation rows per stage
+    g.a_hi = c->amap_hi[tile_index(ar)]; g.a_lo = c->amap_lo[tile_index(ar)];
+    HeadsTcArgs& ha = g.args;
+    ha.bias = c->b_heads; ha.m = B; ha.n = n; ha.V = V; ha.k = k; ha.k_chunks = d / 64; ha.a_rows = ar;
+    ha.out_ids = ids; ha.out_logp = logp; ha.out_lse = lse; ha.out_logits = logits; ha.ldl = n * V;
+    ha.err = c->d_err;
+    ha.trace = tslot(c, MTP_K_HEADS);
+    LAUNCH(MTP_K_HEADS, launch_heads_tc(g, s, pdl));
     return MTP_OK;
 }
 
@@ -735,8 +774,14 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
             LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
         }
-        MTP_TRY(launch_heads_batched(c, c->d_h_last, B, n, c->d_logits, s, pdl, prof));
+        const bool fused = heads_fused_ok(c, k);
+        if (fused)  // candidates, lse and the logits (kept for mtp_debug_logits and the union lattice)
+            MTP_TRY(launch_heads_fused(c, c->d_h_last, B, n, k, c->d_cand_ids, c->d_cand_logp, c->d_lse, c->d_logits,
+                                       s, pdl, prof));
+        else
+            MTP_TRY(launch_heads_batched(c, c->d_h_last, B, n, c->d_logits, s, pdl, prof));
         SelectArgs sa = select_base(c, n, k);
+        sa.pre_topk = fused ? 1 : 0;
         sa.lane = lane ? 1 : 0;
         sa.trace = tslot(c, MTP_K_SELECT);
         LAUNCH(MTP_K_SELECT, launch_select(sa, B, true, s, pdl));
@@ -1248,6 +1293,9 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
         c->use_persistent = value != 0;
     } else if (option == MTP_OPT_PREFILL_TC) {
         c->use_attn_tc = value != 0;  // prefill passes are not captured
+    } else if (option == MTP_OPT_HEADS_FUSED) {
+        changed = c->use_heads_tc != (value != 0);
+        c->use_heads_tc = value != 0;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -1290,6 +1338,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_SEED: *value = (int32_t)c->sample_seed; break;
         case MTP_OPT_PERSISTENT: *value = c->use_persistent && c->sk_ok; break;
         case MTP_OPT_PREFILL_TC: *value = c->use_attn_tc; break;
+        case MTP_OPT_HEADS_FUSED: *value = c->use_heads_tc && c->heads_tc_ok && c->batched_ok; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;
@@ -1689,10 +1738,21 @@ MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden
     // (of the context's logits rows when the caller passes no logits / lse buffers)
     const int lrows = std::max(c->cfg.max_batch, MAX_ROWS);
     const int tc_rows = out_logits && out_lse ? c->bm_max : std::min(c->bm_max, lrows);
-    const bool tc = c->use_batched && c->batched_ok && batch > MAX_ROWS && tc_rows > MAX_ROWS;
-    const int chunk = tc ? tc_rows : MAX_ROWS;
+    // the fused heads need no logits buffer: chunks of every batched row
+    const bool fused = c->use_batched && c->batched_ok && batch > MAX_ROWS && heads_fused_ok(c, k);
+    const bool tc = !fused && c->use_batched && c->batched_ok && batch > MAX_ROWS && tc_rows > MAX_ROWS;
+    const int chunk = fused ? c->bm_max : (tc ? tc_rows : MAX_ROWS);
     for (int b0 = 0; b0 < batch; b0 += chunk) {
         const int m = std::min(chunk, batch - b0);
+        if (fused) {
+            const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
+            CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,
+                                         hidden_dtype == MTP_BF16, c->d_bx, m, d, s));
+            MTP_TRY(launch_heads_fused(c, c->d_bx, m, n, k, out_ids + (size_t)b0 * n * k,
+                                       out_logp + (size_t)b0 * n * k, out_lse ? out_lse + (size_t)b0 * n : nullptr,
+                                       out_logits ? out_logits + (size_t)b0 * n * V : nullptr, s, false, prof));
+            continue;
+        }
         if (tc) {
             const size_t es = hidden_dtype == MTP_BF16 ? 2 : 4;
             CUDA_TRY(launch_convert_rows(static_cast<const char*>(hidden) + (size_t)b0 * d * es,

@@ -382,7 +382,12 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a, int do_
         if (threadIdx.x == 0) a.out_accepted[b] = 0;
         return;
     }
-    if (warp < n) {
+    if (a.pre_topk) {  // the heads kernel ranked them already
+        for (int i = threadIdx.x; i < n * k; i += blockDim.x) {
+            s_ids[i] = a.cand_ids[(size_t)bl * n * k + i];
+            s_lp[i] = a.cand_logp[(size_t)bl * n * k + i];
+        }
+    } else if (warp < n) {
         const size_t row = (size_t)bl * n + warp;
         head_topk_warp(a.logits + row * a.V, a.V, k, s_ids + warp * k, s_lp + warp * k, a.lse + row);
     }
