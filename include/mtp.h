@@ -246,8 +246,15 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        allow it; 0 = two block kernels per layer (default: faster on GB300 at B = 1)
  *   MTP_OPT_PREFILL_TC   1 = prefill passes (mtp_prefill, mtp_prefill_pending) run their attention
  *                        on the tensor cores (tcgen05: tiles of 128 prompt rows, 128-key items, S and
- *                        P V accumulated in TMEM; default); 0 = the split-key kernel of the decode
- *                        steps, in groups of 8 rows
+ *                        P V accumulated in TMEM); 0 = the split-key kernel of the decode steps, in
+ *                        groups of 8 rows (default: on GB300 the serving prompts prefill faster so,
+ *                        42 vs 58 ms at B = 32, 125 vs 144 ms at B = 128)
+ *   MTP_OPT_GEMM_CLUSTER 1 = the batched path's projections at up to 128 fed rows run as one
+ *                        activation tile per weight tile, their K split over the CTAs of a cluster
+ *                        (up to 8) that sum the partial tiles in distributed shared memory, each
+ *                        CTA finishing its share of the rows (q|k|v append, GELU pack, residual
+ *                        add); more splits than a cluster holds add by atomics (default); 0 =
+ *                        tiles of 32 rows, K split only where the output is accumulated
  *   MTP_OPT_HEADS_FUSED  1 = more than 8 hidden rows (batched decode steps, mtp_heads_topk) run the
  *                        heads, log-softmax and top-k as one tensor-core kernel (LN_f rows as bf16
  *                        hi + lo; per (tile of 128 rows, head) a cluster of 8 CTAs over vocabulary
@@ -261,7 +268,7 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
 typedef enum mtp_option {
     MTP_OPT_GRAPHS = 0, MTP_OPT_PDL = 1, MTP_OPT_L2_PREFETCH = 2, MTP_OPT_MLP_CLUSTERS = 3, MTP_OPT_BATCHED = 4,
     MTP_OPT_GEMM_SPLITS = 5, MTP_OPT_LATTICE = 6, MTP_OPT_SAMPLING = 7, MTP_OPT_SEED = 8,
-    MTP_OPT_PERSISTENT = 9, MTP_OPT_PREFILL_TC = 10, MTP_OPT_HEADS_FUSED = 11
+    MTP_OPT_PERSISTENT = 9, MTP_OPT_PREFILL_TC = 10, MTP_OPT_HEADS_FUSED = 11, MTP_OPT_GEMM_CLUSTER = 12
 } mtp_option;
 MTP_API int mtp_set_option(mtp_ctx* ctx, int option, int value);
 MTP_API int mtp_get_option(mtp_ctx* ctx, int option, int32_t* value);

@@ -33,6 +33,7 @@ MTP_OPT_SEED = 8
 MTP_OPT_PERSISTENT = 9
 MTP_OPT_PREFILL_TC = 10
 MTP_OPT_HEADS_FUSED = 11
+MTP_OPT_GEMM_CLUSTER = 12
 KERNEL_KINDS = ("embed", "attn_block", "mlp", "heads", "select", "save", "pack", "gemm", "qkv", "attn", "step", "step_attn",
                 "step_mlp", "step_cta", "attn_tc")
 

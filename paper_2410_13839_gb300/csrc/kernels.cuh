@@ -322,6 +322,9 @@ struct TcGemmArgs {
     const int* block_table; int bt_stride;
     __nv_bfloat16* pack_hi; __nv_bfloat16* pack_lo;  // TC_GELU_PACK: [m][n_w]
     int n_valid;                  // TC_ACCUM: 0, or only features < n_valid are added (element atomics, any ldo)
+    int cluster_reduce;           // 0/1: none; c in 2..8: each c consecutive K splits of a tile are one cluster
+                                  // that sums its partials in DSMEM, each CTA finishing 1/c of the rows
+                                  // (any epilogue; more splits than c only for TC_ACCUM, added by atomics)
     int* err;
     unsigned long long* trace;
 };
@@ -336,6 +339,8 @@ int tc_encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t ro
                  bool pre_swizzled);
 int tc_tile_rows(int m);          // activation rows per tile for m rows: 32, 64 or 128
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl);
+constexpr int TC_CLUSTER_SPLITS = 4;  // K splits one cluster sums in the batched path (clusters of 8 at one CTA per
+                                      // SM: only 15 fit this GPU at once)
 
 // ------------------------------------ fused heads + log-softmax + top-k ----
 // The n heads over m rows of LN_f(h) given as bf16 hi + lo (heads_tc.cu): per

@@ -114,8 +114,9 @@ struct mtp_ctx {
     int device = 0, num_sms = 0, wbytes = 2;
     int mlp_clusters = 1;  // MLP clusters co-resident in one wave
     bool use_graphs = true, use_pdl = true, use_l2_prefetch = false;
-    bool use_attn_tc = true;  // prefill passes: tensor-core attention
+    bool use_attn_tc = false;  // prefill passes: tensor-core attention (option; measured slower, see mtp.h)
     bool use_heads_tc = true;  // more than 8 rows: heads, log-softmax and top-k in one tensor-core kernel
+    bool gemm_cluster = true;  // batched projections: one 128-row activation tile, K splits summed in clusters
     std::vector<void*> allocs;
     // weights
     void* d_weights = nullptr;
@@ -337,7 +338,12 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
     // tiles keep enough CTAs streaming where K is short (q|k|v and W1 finish their
     // rows in the epilogue, one K split; W_o splits K); W2 (K = 4 d) takes whole
     // 128-row tiles and splits its long K instead
-    auto tile_rows = [&](int k) { return std::min(k > 1024 ? 128 : 32, tc_tile_rows(M)); };
+    // with cluster-reduced K splits (option, default), up to 128 rows run as one activation tile:
+    // every weight byte is streamed once, the splits give the parallelism
+    auto tile_rows = [&](int k, int epilogue) {
+        return c->gemm_cluster && M <= 128 && epilogue != TC_ACCUM ? tc_tile_rows(M)
+                                                                    : std::min(k > 1024 ? 128 : 32, tc_tile_rows(M));
+    };
     for (int l = 0; l < cf.layers; ++l) {
         const Layer& L = c->layers[l];
         const mtp_ctx::LayerMaps& W = c->lmaps[l];
@@ -354,15 +360,22 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         };
         auto gemm = [&](const CUtensorMap& w, int n_w, int k, bool a_is_u, int epilogue, float* out, int ldo,
                         const float* bias, int w_rows_per_kchunk) -> int {
-            const int nt = tile_rows(k), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
+            const int nt = tile_rows(k, epilogue), ti = tile_index(nt), ntiles = (M + nt - 1) / nt;
             TcGemm g;
             std::memset(&g, 0, sizeof(g));
             g.w = w;
             g.a_hi = a_is_u ? c->umap_hi[ti] : c->amap_hi[ti];
             g.a_lo = a_is_u ? c->umap_lo[ti] : c->amap_lo[ti];
             g.n_w = n_w; g.nt = nt;
-            g.splits = epilogue == TC_ACCUM ? gemm_splits(c, n_w, k, ntiles) : 1;
+            int sc = 1;
+            if (c->gemm_cluster && epilogue != TC_ACCUM) {  // K splits summed in a cluster, then the epilogue
+                g.splits = std::min(gemm_splits(c, n_w, k, ntiles), TC_CLUSTER_SPLITS);
+                sc = g.splits;
+            } else {  // accumulated outputs: K splits added by atomics
+                g.splits = epilogue == TC_ACCUM ? gemm_splits(c, n_w, k, ntiles) : 1;
+            }
             TcGemmArgs& ga = g.args;
+            ga.cluster_reduce = sc;
             ga.out = out; ga.ldo = ldo; ga.bias = bias; ga.m = M;
             ga.k_chunks = k / 64 / g.splits; ga.w_rows_per_kchunk = w_rows_per_kchunk;
             ga.epilogue = epilogue; ga.err = c->d_err;
@@ -1293,6 +1306,9 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
         c->use_persistent = value != 0;
     } else if (option == MTP_OPT_PREFILL_TC) {
         c->use_attn_tc = value != 0;  // prefill passes are not captured
+    } else if (option == MTP_OPT_GEMM_CLUSTER) {
+        changed = c->gemm_cluster != (value != 0);
+        c->gemm_cluster = value != 0;
     } else if (option == MTP_OPT_HEADS_FUSED) {
         changed = c->use_heads_tc != (value != 0);
         c->use_heads_tc = value != 0;
@@ -1339,6 +1355,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_PERSISTENT: *value = c->use_persistent && c->sk_ok; break;
         case MTP_OPT_PREFILL_TC: *value = c->use_attn_tc; break;
         case MTP_OPT_HEADS_FUSED: *value = c->use_heads_tc && c->heads_tc_ok && c->batched_ok; break;
+        case MTP_OPT_GEMM_CLUSTER: *value = c->gemm_cluster; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
     return MTP_OK;

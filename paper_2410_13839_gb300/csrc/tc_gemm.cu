@@ -39,6 +39,7 @@ constexpr int TC_K = 64;       // k per stage: one 128-byte swizzle row of bf16
 __host__ __device__ constexpr int tc_stages(int nt) { return nt <= 32 ? 8 : (nt <= 64 ? 6 : 4); }
 constexpr int TC_MAX_STAGES = 8;
 constexpr int TC_THREADS = 128;
+constexpr int TC_MAX_CLUSTER_SPLITS = 8;  // K splits reduced in one (portable) cluster
 constexpr uint32_t TC_W_BYTES = TC_M * TC_K * 2;
 
 // ---- PTX wrappers (tcgen05, TMA) ----
@@ -49,6 +50,13 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
+// Shared-memory address `saddr` of this CTA mapped to the CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t mapa_rank(uint32_t saddr, int rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
 // K-major, M = 128, N = nt.
 __host__ __device__ constexpr uint32_t tc_idesc(int nt) {
@@ -183,11 +191,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
     const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
     tc_fence_after();
-    if (fin && s_ok) {
-        // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them),
-        // then float4 rows of T -> out, coalesced
-        constexpr int TP = TC_M + 4;  // row pitch (floats)
-        float* T = reinterpret_cast<float*>(smem);
+    // K splits reduced in a cluster: Sc consecutive splits of this tile are one cluster; each
+    // stages its partial tile, then sums one Sc-th of the activation rows over the cluster's tiles
+    // (DSMEM) and runs the epilogue on those rows only.  Clusters of the same tile (TC_ACCUM with
+    // more splits than one cluster holds) still add their sums with atomics.
+    const int Sc = a.cluster_reduce > 1 ? a.cluster_reduce : 1;
+    const bool creduce = Sc > 1;
+    const int rank = split % Sc;
+    const bool good = fin && s_ok;
+    constexpr int TP = TC_M + 4;  // row pitch of the staged tile (floats)
+    float* T = reinterpret_cast<float*>(smem);
+    if (good) {
+        // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them)
 #pragma unroll 1
         for (int j0 = 0; j0 < NT; j0 += 32) {
             float v[32];
@@ -195,22 +210,70 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) T[(j0 + j) * TP + warp * 32 + lane] = v[j];
         }
-        __syncthreads();
+    }
+    int jbeg = 0, jend = NT;  // activation rows of the tile this CTA finishes
+    if (creduce) {
+        cluster_arrive_release();  // every split's partial tile is staged
+        cluster_wait();
+        jbeg = rank * NT / Sc;
+        jend = (rank + 1) * NT / Sc;
+        if (good) {
+            // RB float4 items per thread and round: every peer's RB loads are in flight together
+            constexpr int RB = 8;
+            const int items = (jend - jbeg) * (TC_M / 4);
+            for (int i0 = tid; i0 < items; i0 += RB * TC_THREADS) {
+                float4 acc[RB];
+                uint32_t off[RB];
+#pragma unroll
+                for (int q = 0; q < RB; ++q) {
+                    const int i = min(i0 + q * TC_THREADS, items - 1);  // past the end: a repeat, not stored
+                    float* t = T + (jbeg + i / (TC_M / 4)) * TP + (i % (TC_M / 4)) * 4;
+                    off[q] = smem_addr(t);
+                    acc[q] = *reinterpret_cast<const float4*>(t);
+                }
+                for (int r = 1; r < Sc; ++r) {  // the peers in rank order after this one
+                    const int p = (rank + r) % Sc;
+                    float4 u[RB];
+#pragma unroll
+                    for (int q = 0; q < RB; ++q) u[q] = ld_dsmem4(mapa_rank(off[q], p));
+#pragma unroll
+                    for (int q = 0; q < RB; ++q) {
+                        acc[q].x += u[q].x;
+                        acc[q].y += u[q].y;
+                        acc[q].z += u[q].z;
+                        acc[q].w += u[q].w;
+                    }
+                }
+#pragma unroll
+                for (int q = 0; q < RB; ++q)
+                    if (i0 + q * TC_THREADS < items) {
+                        const int i = i0 + q * TC_THREADS;
+                        float* t = T + (jbeg + i / (TC_M / 4)) * TP + (i % (TC_M / 4)) * 4;
+                        *reinterpret_cast<float4*>(t) = acc[q];
+                    }
+            }
+        }
+        cluster_arrive_relaxed();  // done reading the peers' tiles (waited for before leaving)
+    }
+    __syncthreads();
+    if (good) {
+        // float4 rows of T -> out, coalesced
         const int rows = min(NT, a.m - arow);
+        const bool add_bias = a.bias && split < Sc;  // the tile's first cluster (or split 0) adds it
         const int P = a.page_size, H = a.n_heads, d = H * HEAD_DIM;
+        const int j1 = min(jend, rows);
         if constexpr (PART) {  // TC_ACCUM of features < n_valid only, element atomics (rows of any pitch)
-            for (int i = tid; i < rows * TC_M; i += TC_THREADS) {
-                const int j = i / TC_M, fl = i % TC_M, f = tile * TC_M + fl;
+            for (int i = tid; i < (j1 - jbeg) * TC_M; i += TC_THREADS) {
+                const int j = jbeg + i / TC_M, fl = i % TC_M, f = tile * TC_M + fl;
                 if (f < a.n_valid)
-                    atomicAdd(a.out + (size_t)(arow + j) * a.ldo + f,
-                              T[j * TP + fl] + (a.bias && split == 0 ? a.bias[f] : 0.f));
+                    atomicAdd(a.out + (size_t)(arow + j) * a.ldo + f, T[j * TP + fl] + (add_bias ? a.bias[f] : 0.f));
             }
         } else
-        for (int i = tid; i < rows * (TC_M / 4); i += TC_THREADS) {
-            const int j = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
+        for (int i = tid; i < (j1 - jbeg) * (TC_M / 4); i += TC_THREADS) {
+            const int j = jbeg + i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
             const int f = tile * TC_M + f4, n = arow + j;
             float4 y = *reinterpret_cast<const float4*>(T + j * TP + f4);
-            if (a.bias && split == 0) {
+            if (add_bias) {
                 y.x += a.bias[f];
                 y.y += a.bias[f + 1];
                 y.z += a.bias[f + 2];
@@ -257,6 +320,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         // the MMAs may still be running: wait for them (bounded) before freeing TMEM
         mbar_wait(&done, 0, nullptr);
     }
+    if (creduce) cluster_wait();  // the peers are done with this CTA's tile
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, TMEM_COLS);
@@ -296,11 +360,18 @@ cudaError_t launch_kern(K kern, const TcGemm& g, cudaStream_t s, bool pdl) {
     cfg.blockDim = dim3(TC_THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (g.args.cluster_reduce > 1) {  // consecutive K splits of a tile form one cluster
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = 1;
+        attr[1].val.clusterDim.y = g.args.cluster_reduce;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
+    }
     return cudaLaunchKernelEx(&cfg, kern, g.w, g.a_hi, g.a_lo, g.args);
 }
 
@@ -333,7 +404,9 @@ int tc_tile_rows(int m) { return m <= 32 ? 32 : (m <= 64 ? 64 : 128); }
 
 cudaError_t launch_tc_gemm(const TcGemm& g, cudaStream_t s, bool pdl) {
     if (g.n_w % TC_M || g.args.k_chunks < 1 || g.splits < 1 || g.args.m < 1) return cudaErrorInvalidValue;
-    if (g.args.epilogue != TC_ACCUM && g.splits != 1) return cudaErrorInvalidValue;
+    const int sc = g.args.cluster_reduce > 1 ? g.args.cluster_reduce : 1;
+    if (sc > TC_MAX_CLUSTER_SPLITS || g.splits % sc) return cudaErrorInvalidValue;
+    if (g.args.epilogue != TC_ACCUM && g.splits != sc) return cudaErrorInvalidValue;  // one cluster finishes a tile
     switch (g.nt) {
         case 32: return launch_nt<32>(g, s, pdl);
         case 64: return launch_nt<64>(g, s, pdl);
