@@ -255,11 +255,12 @@ MTP_API int mtp_debug_lattice(mtp_ctx* ctx, int32_t* out_ids, float* out_logp, i
  *                        CTA finishing its share of the rows (q|k|v append, GELU pack, residual
  *                        add); more splits than a cluster holds add by atomics (default); 0 =
  *                        tiles of 32 rows, K split only where the output is accumulated
- *   MTP_OPT_HEADS_FUSED  1 = more than 8 hidden rows (batched decode steps, mtp_heads_topk) run the
- *                        heads, log-softmax and top-k as one tensor-core kernel (LN_f rows as bf16
- *                        hi + lo; per (tile of 128 rows, head) a cluster of 8 CTAs over vocabulary
- *                        slices, lse merged in the cluster before the top-k; default); 0 = heads GEMM
- *                        into memory, then the selection kernel's top-k
+ *   MTP_OPT_HEADS_FUSED  heads, log-softmax and top-k of more than 8 hidden rows as one tensor-core
+ *                        kernel (LN_f rows as bf16 hi + lo; per (tile of 128 rows, head) a cluster of
+ *                        8 CTAs over vocabulary slices, lse merged in the cluster before the top-k):
+ *                        0 = never (heads GEMM into memory, then the selection kernel's top-k);
+ *                        1 = in mtp_heads_topk (default: 65.8 vs 94.6 us for 256 rows, n = 8, top-16);
+ *                        2 = also in batched decode steps (measured 1.2 % slower per step at B = 32)
  *   MTP_OPT_SEED         seed of the path draws (any 32-bit value, zero-extended; default 0).
  *                        Position t of a draw of slot b that has generated g tokens uses the
  *                        uniform (SplitMix64(x) >> 40) / 2^24, x = ((seed * P + b) * P + g) * P + t

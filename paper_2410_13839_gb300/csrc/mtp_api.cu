@@ -115,7 +115,7 @@ struct mtp_ctx {
     int mlp_clusters = 1;  // MLP clusters co-resident in one wave
     bool use_graphs = true, use_pdl = true, use_l2_prefetch = false;
     bool use_attn_tc = false;  // prefill passes: tensor-core attention (option; measured slower, see mtp.h)
-    bool use_heads_tc = true;  // more than 8 rows: heads, log-softmax and top-k in one tensor-core kernel
+    int use_heads_tc = 1;  // fused heads kernel: 0 never, 1 stand-alone heads calls, 2 also batched decode steps
     bool gemm_cluster = true;  // batched projections: one 128-row activation tile, K splits summed in clusters
     std::vector<void*> allocs;
     // weights
@@ -634,8 +634,9 @@ int launch_heads_batched(mtp_ctx* c, const float* x, int B, int n, float* logits
     return MTP_OK;
 }
 
-bool heads_fused_ok(const mtp_ctx* c, int k) {
-    return c->use_heads_tc && c->batched_ok && c->heads_tc_ok && heads_tc_supported(c->cfg.codec_vocab, k);
+bool heads_fused_ok(const mtp_ctx* c, int k, bool decode_step) {
+    return c->use_heads_tc >= (decode_step ? 2 : 1) && c->batched_ok && c->heads_tc_ok &&
+           heads_tc_supported(c->cfg.codec_vocab, k);
 }
 
 // The heads fused with their log-softmax and top-k over B hidden rows x [B][d]
@@ -787,7 +788,7 @@ int enqueue_step(mtp_ctx* c, int n, int k, cudaStream_t s, bool pdl, Prof* prof,
             unsigned long long* tr = tslot(c, MTP_K_SAVE);
             LAUNCH(MTP_K_SAVE, launch_save_last(c->d_bx, c->d_row_seq, c->d_row_last, c->d_h_last, d, M, tr, s, pdl));
         }
-        const bool fused = heads_fused_ok(c, k);
+        const bool fused = heads_fused_ok(c, k, true);
         if (fused)  // candidates, lse and the logits (kept for mtp_debug_logits and the union lattice)
             MTP_TRY(launch_heads_fused(c, c->d_h_last, B, n, k, c->d_cand_ids, c->d_cand_logp, c->d_lse, c->d_logits,
                                        s, pdl, prof));
@@ -1310,8 +1311,9 @@ MTP_API int mtp_set_option(mtp_ctx* c, int option, int value) {
         changed = c->gemm_cluster != (value != 0);
         c->gemm_cluster = value != 0;
     } else if (option == MTP_OPT_HEADS_FUSED) {
-        changed = c->use_heads_tc != (value != 0);
-        c->use_heads_tc = value != 0;
+        if (value < 0 || value > 2) return fail(MTP_ERR_INVALID, "heads option %d: 0, 1 or 2", value);
+        changed = c->use_heads_tc != value;
+        c->use_heads_tc = value;
     } else if (option == MTP_OPT_BATCHED) {
         changed = c->use_batched != (value != 0);
         c->use_batched = value != 0;
@@ -1354,7 +1356,7 @@ MTP_API int mtp_get_option(mtp_ctx* c, int option, int32_t* value) {
         case MTP_OPT_SEED: *value = (int32_t)c->sample_seed; break;
         case MTP_OPT_PERSISTENT: *value = c->use_persistent && c->sk_ok; break;
         case MTP_OPT_PREFILL_TC: *value = c->use_attn_tc; break;
-        case MTP_OPT_HEADS_FUSED: *value = c->use_heads_tc && c->heads_tc_ok && c->batched_ok; break;
+        case MTP_OPT_HEADS_FUSED: *value = c->heads_tc_ok && c->batched_ok ? c->use_heads_tc : 0; break;
         case MTP_OPT_GEMM_CLUSTER: *value = c->gemm_cluster; break;
         default: return fail(MTP_ERR_INVALID, "unknown option %d", option);
     }
@@ -1756,7 +1758,7 @@ MTP_API int mtp_heads_topk(mtp_ctx* c, int batch, const void* hidden, int hidden
     const int lrows = std::max(c->cfg.max_batch, MAX_ROWS);
     const int tc_rows = out_logits && out_lse ? c->bm_max : std::min(c->bm_max, lrows);
     // the fused heads need no logits buffer: chunks of every batched row
-    const bool fused = c->use_batched && c->batched_ok && batch > MAX_ROWS && heads_fused_ok(c, k);
+    const bool fused = c->use_batched && c->batched_ok && batch > MAX_ROWS && heads_fused_ok(c, k, false);
     const bool tc = !fused && c->use_batched && c->batched_ok && batch > MAX_ROWS && tc_rows > MAX_ROWS;
     const int chunk = fused ? c->bm_max : (tc ? tc_rows : MAX_ROWS);
     for (int b0 = 0; b0 < batch; b0 += chunk) {

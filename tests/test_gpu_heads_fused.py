@@ -137,3 +137,50 @@ def test_tiny_model_and_ties():
                     assert ids[b, i, :len(top)].tolist() == top.tolist()
     finally:
         dec.close()
+
+
+def test_decode_steps_with_fused_heads():
+    """Batched decode steps (B = 12, n = 4, top-4) with the fused heads (option 2) against the same
+    teacher-forced steps with the GEMM + selection top-k (option 0) and the oracle: logits within 5e-4
+    of each other (two summation orders of the same bf16 hi/lo products over d = 1024; logits up to ~4)
+    and within the bf16 bar of the oracle; each run's candidates exact on its own logp
+    rows; paths equal wherever the candidates are."""
+    from oracle.mtp import MTPOracle
+    mtp = lib_module()
+    model = synth.VALLE
+    B, n, k, steps = 12, 4, 4, 4
+    prompts = [synth.make_prompt(300 + b, 20 + 3 * b, 60 + 5 * b, model.phone_vocab) for b in range(B)]
+    runs = []
+    w = None
+    for opt in (2, 0):
+        dec, w = decoder(model, max_batch=B, max_ctx=256)
+        try:
+            mtp.mtp_set_option(dec.ctx, OPT_HEADS_FUSED, opt)
+            assert mtp.mtp_get_option(dec.ctx, OPT_HEADS_FUSED) == opt
+            for b, (ph, ac) in enumerate(prompts):
+                dec.prefill(b, ph, ac, 64)
+            rec = []
+            for t in range(steps):
+                if t:  # teacher-forced: both runs feed the same tokens (the first run's path)
+                    for b in range(B):
+                        mtp.mtp_set_teacher_tokens(dec.ctx, b, runs[0][t - 1][3][b] if opt == 0 else rec[-1][3][b])
+                dec.decode_step(n, k)
+                lg, lse = dec.logits(n)
+                ids, lp, path = dec.lattice(n, k)
+                rec.append((lg.copy(), lse.copy(), (ids.copy(), lp.copy()), path.copy()))
+            runs.append(rec)
+        finally:
+            dec.close()
+    o = MTPOracle(model, w)
+    ph, ac = prompts[0]
+    o.prefill(ph, ac, 64)
+    assert_logits_close(runs[0][0][0][0], o.step(n, k).logits, "slot 0, step 0")
+    for t in range(steps):
+        (lg_f, lse_f, (ids_f, lp_f), path_f), (lg_u, lse_u, (ids_u, lp_u), path_u) = runs[0][t], runs[1][t]
+        assert np.abs(lg_f - lg_u).max() < 5e-4
+        for b in range(B):
+            r_ids, r_vals = S.top_k_rows(logp32(lg_f[b], lse_f[b]), k)
+            assert np.array_equal(ids_f[b], r_ids), f"step {t} slot {b}"
+            assert np.array_equal(lp_f[b].view(np.uint32), r_vals.view(np.uint32))
+            if np.array_equal(ids_f[b], ids_u[b]):
+                assert np.array_equal(path_f[b], path_u[b])
