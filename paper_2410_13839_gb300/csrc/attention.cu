@@ -32,7 +32,8 @@ constexpr int ATT_THREADS = 128;  // four warps: four CTAs per SM
 constexpr int ATT_STAGES = 3;    // staging slots of the key/value ring (three 64-key slots keep ~48 KB in flight)
 constexpr int RPG = MAX_ROWS;    // rows per group, upper bound
 constexpr int PART = 2 + HEAD_DIM;  // (max, sum, out[64]) per row and split
-constexpr int MAX_SPLITS = 32;     // one warp lane per split in the merge
+constexpr int MAX_SPLITS = ATTN_MAX_SPLITS;  // one warp lane per split in the merge
+static_assert(MAX_SPLITS <= 32, "the merge takes one lane per split");
 static_assert(HEAD_DIM == 64, "score scale 0.125 assumes 64-wide heads");
 
 
@@ -477,7 +478,7 @@ int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int nu
 
 cudaError_t launch_attention(const AttnArgs& a, int groups, cudaStream_t s, bool pdl) {
     if (a.rows_per_group < 1 || a.rows_per_group > RPG || half_keys(a.page_size) % a.page_size != 0 ||
-        a.n_splits < 1)
+        a.n_splits < 1 || a.n_splits > MAX_SPLITS)
         return cudaErrorInvalidValue;
     const size_t smem = attn_smem_bytes(a.page_size);
     cudaError_t e = ensure_kernel_smem(reinterpret_cast<const void*>(attn_kernel), smem);

@@ -82,6 +82,8 @@ struct AttnArgs {
     int rows;                                                // attention_tc: rows of the pass (tiles of 128)
 };
 
+constexpr int ATTN_CTAS_PER_SM = 4;  // attn_kernel: 128 threads x 128 registers, ~51 KB of shared memory
+constexpr int ATTN_MAX_SPLITS = 32;  // key splits one launch merges
 size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
 size_t attn_smem_bytes(int page_size);
 int attn_splits_for(int groups, int n_heads, int page_size, int max_keys, int num_sms);

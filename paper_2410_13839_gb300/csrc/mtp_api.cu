@@ -402,9 +402,19 @@ int run_layers_batched(mtp_ctx* c, int M, int rpg, int groups, int plan, cudaStr
         at.out_hi = c->d_ahi; at.out_lo = c->d_alo; at.ldb = d;  // straight into W_o's operand
         at.ws_part = c->d_bws; at.ws_count = c->d_bwc;
         at.rows_per_group = rpg; at.n_heads = H; at.page_size = P;
-        at.n_splits = std::min(attn_splits_for(groups, H, P, cf.max_ctx, c->num_sms),
-                               c->battn_ws_units / std::max(1, groups));
-        at.n_splits = std::max(1, at.n_splits);
+        // key splits.  Decode steps: about 2.5 waves of CTAs at four per SM, so the slots with the
+        // longest contexts do not set the launch's length (B = 32 serving: 3 splits, 888 vs 972 us
+        // per step with one; B = 128: one split, two measured 5.6 % slower).  Prefill passes: one
+        // wave (their groups of 8 positions have similar key counts; the decode rule measured 13 %
+        // slower at B = 32).
+        {
+            int want = attn_splits_for(groups, H, P, cf.max_ctx, c->num_sms);
+            if (plan == PLAN_DEVICE) {
+                const double waves = 2.5 * ATTN_CTAS_PER_SM * c->num_sms / std::max(1, groups * H);
+                want = std::min({(int)std::lround(waves), (cf.max_ctx + P - 1) / P, ATTN_MAX_SPLITS});
+            }
+            at.n_splits = std::max(1, std::min(want, c->battn_ws_units / std::max(1, groups)));
+        }
         at.plan = plan; at.seq_len = c->d_len; at.seq_new = c->d_npend; at.seq_base = 0;
         at.err = c->d_err; at.kv_swizzled = 1;
         if (prefill_keys > 0 && c->use_attn_tc && plan == PLAN_ROWS) {
