@@ -50,6 +50,14 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
+// Bulk copy of `bytes` from this CTA's shared memory to shared memory of a CTA of the cluster
+// (dst, bar: shared::cluster addresses), completing on that CTA's barrier.  16-byte aligned.
+__device__ __forceinline__ void bulk_copy_s2s_cluster(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "r"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 // Shared-memory address `saddr` of this CTA mapped to the CTA of cluster rank `rank`.
 __device__ __forceinline__ uint32_t mapa_rank(uint32_t saddr, int rank) {
     uint32_t r;
@@ -71,7 +79,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     constexpr uint32_t A_BYTES = NT * TC_K * 2, STAGE = TC_W_BYTES + 2 * A_BYTES;
     constexpr uint32_t TMEM_COLS = NT < 32 ? 32 : NT;
     constexpr int TC_STAGES = tc_stages(NT);
-    __shared__ uint64_t full[TC_MAX_STAGES], empty[TC_MAX_STAGES], done;
+    __shared__ uint64_t full[TC_MAX_STAGES], empty[TC_MAX_STAGES], done, red_bar;
     __shared__ uint32_t tmem_base;
     __shared__ int s_ok;
     __shared__ long long s_rowbase[NT];  // TC_QKV: element offset of the row's key row in its page (-1: none)
@@ -94,6 +102,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             mbar_init(&empty[s], 1);
         }
         mbar_init(&done, 1);
+        mbar_init(&red_bar, 1);
         fence_barrier_init();
         s_ok = 1;
     }
@@ -213,50 +222,47 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     int jbeg = 0, jend = NT;  // activation rows of the tile this CTA finishes
     if (creduce) {
-        cluster_arrive_release();  // every split's partial tile is staged
-        cluster_wait();
+        // each CTA pushes the rows that another CTA finishes to that CTA (one bulk copy per peer,
+        // completing on the receiver's barrier), then sums the Sc partial copies of its own rows
         jbeg = rank * NT / Sc;
         jend = (rank + 1) * NT / Sc;
-        if (good) {
-            // RB float4 items per thread and round: every peer's RB loads are in flight together
-            constexpr int RB = 8;
-            const int items = (jend - jbeg) * (TC_M / 4);
-            for (int i0 = tid; i0 < items; i0 += RB * TC_THREADS) {
-                float4 acc[RB];
-                uint32_t off[RB];
-#pragma unroll
-                for (int q = 0; q < RB; ++q) {
-                    const int i = min(i0 + q * TC_THREADS, items - 1);  // past the end: a repeat, not stored
-                    float* t = T + (jbeg + i / (TC_M / 4)) * TP + (i % (TC_M / 4)) * 4;
-                    off[q] = smem_addr(t);
-                    acc[q] = *reinterpret_cast<const float4*>(t);
-                }
-                for (int r = 1; r < Sc; ++r) {  // the peers in rank order after this one
-                    const int p = (rank + r) % Sc;
-                    float4 u[RB];
-#pragma unroll
-                    for (int q = 0; q < RB; ++q) u[q] = ld_dsmem4(mapa_rank(off[q], p));
-#pragma unroll
-                    for (int q = 0; q < RB; ++q) {
-                        acc[q].x += u[q].x;
-                        acc[q].y += u[q].y;
-                        acc[q].z += u[q].z;
-                        acc[q].w += u[q].w;
-                    }
-                }
-#pragma unroll
-                for (int q = 0; q < RB; ++q)
-                    if (i0 + q * TC_THREADS < items) {
-                        const int i = i0 + q * TC_THREADS;
-                        float* t = T + (jbeg + i / (TC_M / 4)) * TP + (i % (TC_M / 4)) * 4;
-                        *reinterpret_cast<float4*>(t) = acc[q];
-                    }
+        const uint32_t seg = (uint32_t)(NT / Sc) * TP * 4;  // bytes of one CTA's share of rows
+        float* recv = T + (size_t)NT * TP;                  // [Sc][NT / Sc][TP]: slot = sender's rank
+        if (tid == 0) mbar_arrive_expect_tx(&red_bar, seg * (uint32_t)(Sc - 1));
+        __syncthreads();
+        cluster_arrive_release();  // every split's partial tile is staged and every receiver armed
+        cluster_wait();
+        if (tid == 0 && good) {
+            fence_proxy_async();  // the tile was written by this CTA's threads
+            for (int r = 1; r < Sc; ++r) {
+                const int p = (rank + r) % Sc;
+                bulk_copy_s2s_cluster(mapa_rank(smem_addr(recv + (size_t)rank * (NT / Sc) * TP), p),
+                                      smem_addr(T + (size_t)p * (NT / Sc) * TP), seg,
+                                      mapa_rank(smem_addr(&red_bar), p));
             }
         }
-        cluster_arrive_relaxed();  // done reading the peers' tiles (waited for before leaving)
+        const bool got = mbar_wait(&red_bar, 0, a.err);
+        if (good && got) {
+            for (int i = tid; i < (jend - jbeg) * (TC_M / 4); i += TC_THREADS) {
+                const int jl = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
+                float* t = T + (size_t)(jbeg + jl) * TP + f4;
+                float4 acc = *reinterpret_cast<const float4*>(t);
+                for (int src = 0; src < Sc; ++src) {  // the other splits, in rank order
+                    if (src == rank) continue;
+                    const float4 u = *reinterpret_cast<const float4*>(recv + ((size_t)src * (NT / Sc) + jl) * TP + f4);
+                    acc.x += u.x;
+                    acc.y += u.y;
+                    acc.z += u.z;
+                    acc.w += u.w;
+                }
+                *reinterpret_cast<float4*>(t) = acc;
+            }
+        }
+        if (!got) s_ok = 0;
+        cluster_arrive_relaxed();  // this CTA's pushes have landed (waited for before leaving)
     }
     __syncthreads();
-    if (good) {
+    if (good && s_ok) {
         // float4 rows of T -> out, coalesced
         const int rows = min(NT, a.m - arow);
         const bool add_bias = a.bias && split < Sc;  // the tile's first cluster (or split 0) adds it
@@ -268,17 +274,23 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 if (f < a.n_valid)
                     atomicAdd(a.out + (size_t)(arow + j) * a.ldo + f, T[j * TP + fl] + (add_bias ? a.bias[f] : 0.f));
             }
-        } else
+        } else {
+        // every item of this thread has the same 4 features (TC_THREADS is a multiple of TC_M / 4):
+        // their bias is read once, ahead of the stores
+        static_assert(TC_THREADS % (TC_M / 4) == 0, "one feature quad per thread");
+        float4 bq = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (add_bias) {
+            const int f = tile * TC_M + (tid % (TC_M / 4)) * 4;
+            bq = make_float4(__ldg(a.bias + f), __ldg(a.bias + f + 1), __ldg(a.bias + f + 2), __ldg(a.bias + f + 3));
+        }
         for (int i = tid; i < (j1 - jbeg) * (TC_M / 4); i += TC_THREADS) {
             const int j = jbeg + i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
             const int f = tile * TC_M + f4, n = arow + j;
             float4 y = *reinterpret_cast<const float4*>(T + j * TP + f4);
-            if (add_bias) {
-                y.x += a.bias[f];
-                y.y += a.bias[f + 1];
-                y.z += a.bias[f + 2];
-                y.w += a.bias[f + 3];
-            }
+            y.x += bq.x;
+            y.y += bq.y;
+            y.z += bq.z;
+            y.w += bq.w;
             if (a.epilogue == TC_ACCUM) {
                 atomicAdd(reinterpret_cast<float4*>(a.out + (size_t)n * a.ldo + f), y);
             } else if (a.epilogue == TC_STORE) {
@@ -315,6 +327,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 *reinterpret_cast<uint2*>(a.pack_hi + (size_t)n * a.ldo + f) = make_uint2(hi[0], hi[1]);
                 *reinterpret_cast<uint2*>(a.pack_lo + (size_t)n * a.ldo + f) = make_uint2(lo[0], lo[1]);
             }
+        }
         }
     } else if (!fin) {
         // the MMAs may still be running: wait for them (bounded) before freeing TMEM
