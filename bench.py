@@ -674,6 +674,36 @@ def run_profile_b32():
 PROFILE_B32_STEPS = 12
 
 
+def run_profile_b32_serving():
+    """Kernel captures at serving context lengths (not a measurement): the 32 batched-serving
+    prompts admitted and prefilled together (mtp_prefill_pending), then
+    PROFILE_SERVING_STEPS decode steps, so the contexts reach ~1,200 keys.  Prints how many
+    attention launches (attn_kernel) ran before the last step: a capture of the last step's
+    first attention skips that many."""
+    import torch
+    from paper_2410_13839_gb300 import build
+    build.build()
+    from paper_2410_13839_gb300 import mtp
+    seqs = b32_sequences(B32)
+    max_ctx = max(len(p) + len(a) + g for p, a, g in seqs) + MODEL.n_heads_max + 8
+    w = synth.make_weights(MODEL)
+    stream = torch.cuda.Stream()
+    dec = mtp.MTPDecoder(MODEL, w, synth.weight_names(MODEL), synth.is_matrix, B32, max_ctx, stream=stream)
+    for b, (p, a, g) in enumerate(seqs):
+        mtp.mtp_admit(dec.ctx, b, p, a, g)
+    passes = mtp.mtp_prefill_pending(dec.ctx)
+    for _ in range(PROFILE_SERVING_STEPS):
+        mtp.mtp_decode_step(dec.ctx, N_HEADS, TOP_K)
+    torch.cuda.synchronize()
+    dec.close()
+    before_last = (passes + PROFILE_SERVING_STEPS - 1) * MODEL.layers
+    print(json.dumps({"profile_b32_serving": "done", "prefill_passes": passes, "decode_steps": PROFILE_SERVING_STEPS,
+                      "attention_launches_before_last_step": before_last}), flush=True)
+
+
+PROFILE_SERVING_STEPS = 200
+
+
 def run_profile_select():
     """Kernel captures of the selection kernels (not a measurement): three mtp_viterbi
     calls on the C5 lattices (10^4 x 8 x 16), then four B=1 decode steps of the
@@ -718,6 +748,8 @@ def main():
     ap.add_argument("--no-c5", action="store_true", help="skip the isolated heads + Viterbi microbenchmark")
     ap.add_argument("--profile-b32", action="store_true",
                     help="only run a small batch-32 decode for kernel captures (prints no measurement)")
+    ap.add_argument("--profile-b32-serving", action="store_true",
+                    help="only run the batch-32 serving prompts and 200 decode steps for captures (no measurement)")
     ap.add_argument("--profile-select", action="store_true",
                     help="only run the Viterbi and selection kernels for captures (prints no measurement)")
     args = ap.parse_args()
@@ -726,6 +758,8 @@ def main():
         print(json.dumps({"value": value, "sample": sample}), flush=True)
     elif args.profile_b32:
         run_profile_b32()
+    elif args.profile_b32_serving:
+        run_profile_b32_serving()
     elif args.profile_select:
         run_profile_select()
     elif args.impl == "reference":
