@@ -27,9 +27,19 @@ def _prompts(model, batch, seed0):
     return out
 
 
-def batched_teacher_forced(model, batch, n, k, max_new, max_steps, seed0=300, batched=1):
+def _serving_prompts(model, batch):
+    """The batched-serving recipe: U[32,128] phonemes + U[150,450] acoustic tokens (seeds 2000 + i)."""
+    out = []
+    for i in range(batch):
+        n_ph = synth.make_lengths(i, 32, 128, "serve_phonemes")
+        n_ac = synth.make_lengths(i, 150, 450, "serve_acoustic")
+        out.append(synth.make_prompt(i, n_ph, n_ac, model.phone_vocab))
+    return out
+
+
+def batched_teacher_forced(model, batch, n, k, max_new, max_steps, seed0=300, batched=1, prompts=None):
     mtp = lib_module()
-    prompts = _prompts(model, batch, seed0)
+    prompts = prompts if prompts is not None else _prompts(model, batch, seed0)
     max_ctx = max(len(p) + len(a) for p, a in prompts) + max_new + model.n_heads_max + 3
     dec, w = decoder(model, max_batch=batch, max_ctx=max_ctx)
     logs = []
@@ -84,6 +94,15 @@ def test_batched_equals_fused_passes():
 
 def test_batched_valle_b32():
     batched_teacher_forced(synth.VALLE, batch=32, n=4, k=4, max_new=16, max_steps=2, seed0=500)
+
+
+def test_batched_valle_b32_serving_prompts():
+    """VALL-E-sized B=32 with the serving workload's prompt lengths (182-578 positions: two to
+    five 128-position prefill chunks per slot; decode contexts of several key pages per split)."""
+    prompts = _serving_prompts(synth.VALLE, 32)
+    lens = [len(p) + len(a) for p, a in prompts]
+    assert min(lens) > 128 and max(lens) > 3 * 128
+    batched_teacher_forced(synth.VALLE, batch=32, n=4, k=4, max_new=8, max_steps=2, prompts=prompts)
 
 
 def test_batched_tiny_bf16_b128():
