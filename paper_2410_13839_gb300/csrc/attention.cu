@@ -418,6 +418,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
     }
     __threadfence();
     __syncthreads();
+    trace_mark(a.trace, 2);  // split partials written
     if (tid == 0) s_last = atomicAdd(a.ws_count + g * H + h, 1) == S - 1;
     __syncthreads();
     if (!s_last) return;

@@ -14,8 +14,9 @@
 // and of both activation parts into a 4-stage shared-memory ring with TMA
 // (128-byte swizzled tiles), a second elected thread issues tcgen05.mma
 // into a TMEM accumulator (128 lanes x NT fp32 columns) and releases each
-// stage with tcgen05.commit, and the four warps read the accumulator back
-// with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31, i.e. weight rows) and
+// stage with tcgen05.commit, and the eight warps read the accumulator back
+// with tcgen05.ld (warps w and w + 4 own TMEM lanes 32w..32w+31, i.e. weight
+// rows, and take alternate 32-column chunks) and
 // store or atomically add it to out.  Grid: (N_w / 128 weight tiles, K
 // splits, activation tiles).  The weight copies of the first stages are
 // issued before griddepcontrol.wait; the activation copies after it.
@@ -38,7 +39,10 @@ constexpr int TC_K = 64;       // k per stage: one 128-byte swizzle row of bf16
 // ring stages per activation tile size: about 190 KB of copies in flight per CTA
 __host__ __device__ constexpr int tc_stages(int nt) { return nt <= 32 ? 8 : (nt <= 64 ? 6 : 4); }
 constexpr int TC_MAX_STAGES = 8;
-constexpr int TC_THREADS = 128;
+// 8 warps: two elected lanes run the ring; in the epilogue warps w and w + 4 share TMEM lane
+// quarter w % 4 and take alternate 32-column chunks, and every row loop has twice the threads
+// (the epilogue is instruction-latency bound: one warp per scheduler hid nothing)
+constexpr int TC_THREADS = 256;
 constexpr int TC_MAX_CLUSTER_SPLITS = 8;  // K splits reduced in one (portable) cluster
 constexpr uint32_t TC_W_BYTES = TC_M * TC_K * 2;
 
@@ -198,8 +202,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (warp < 2) __syncwarp();
 
     // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
-    const bool fin = __syncthreads_and(mbar_wait(&done, 0, a.err)) != 0;  // uniform: the epilogue synchronises
+    // one thread polls (a poll costs each polling thread, even on a completed phase); the block
+    // barrier hands the result to the others
+    const bool fin = __syncthreads_and(tid == 0 ? mbar_wait(&done, 0, a.err) : true) != 0;
     tc_fence_after();
+    trace_mark(a.trace, 0);  // accumulator complete
     // K splits reduced in a cluster: Sc consecutive splits of this tile are one cluster; each
     // stages its partial tile, then sums one Sc-th of the activation rows over the cluster's tiles
     // (DSMEM) and runs the epilogue on those rows only.  Clusters of the same tile (TC_ACCUM with
@@ -213,13 +220,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (good) {
         // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them)
 #pragma unroll 1
-        for (int j0 = 0; j0 < NT; j0 += 32) {
+        const int quarter = warp & 3;  // the TMEM lanes (weight rows) this warp may read
+        for (int j0 = (warp >> 2) * 32; j0 < NT; j0 += (TC_THREADS / 128) * 32) {
             float v[32];
-            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)j0, v);
+            tmem_ld32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)j0, v);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) T[(j0 + j) * TP + warp * 32 + lane] = v[j];
+            for (int j = 0; j < 32; ++j) T[(j0 + j) * TP + quarter * 32 + lane] = v[j];
         }
     }
+    trace_mark(a.trace, 1);  // thread 0's rows staged
     int jbeg = 0, jend = NT;  // activation rows of the tile this CTA finishes
     if (creduce) {
         // each CTA pushes the rows that another CTA finishes to that CTA (one bulk copy per peer,
@@ -232,28 +241,33 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         __syncthreads();
         cluster_arrive_release();  // every split's partial tile is staged and every receiver armed
         cluster_wait();
-        if (tid == 0 && good) {
+        trace_mark(a.trace, 2);  // the cluster's tiles staged
+        if (tid < Sc - 1 && good) {  // one copy per issuing thread
             fence_proxy_async();  // the tile was written by this CTA's threads
-            for (int r = 1; r < Sc; ++r) {
-                const int p = (rank + r) % Sc;
-                bulk_copy_s2s_cluster(mapa_rank(smem_addr(recv + (size_t)rank * (NT / Sc) * TP), p),
-                                      smem_addr(T + (size_t)p * (NT / Sc) * TP), seg,
-                                      mapa_rank(smem_addr(&red_bar), p));
-            }
+            const int p = (rank + 1 + tid) % Sc;
+            bulk_copy_s2s_cluster(mapa_rank(smem_addr(recv + (size_t)rank * (NT / Sc) * TP), p),
+                                  smem_addr(T + (size_t)p * (NT / Sc) * TP), seg, mapa_rank(smem_addr(&red_bar), p));
         }
-        const bool got = mbar_wait(&red_bar, 0, a.err);
+        const bool got = __syncthreads_and(tid == 0 ? mbar_wait(&red_bar, 0, a.err) : true) != 0;
+        trace_mark(a.trace, 3);  // the peers' partial rows received
         if (good && got) {
             for (int i = tid; i < (jend - jbeg) * (TC_M / 4); i += TC_THREADS) {
                 const int jl = i / (TC_M / 4), f4 = (i % (TC_M / 4)) * 4;
                 float* t = T + (size_t)(jbeg + jl) * TP + f4;
-                float4 acc = *reinterpret_cast<const float4*>(t);
-                for (int src = 0; src < Sc; ++src) {  // the other splits, in rank order
-                    if (src == rank) continue;
-                    const float4 u = *reinterpret_cast<const float4*>(recv + ((size_t)src * (NT / Sc) + jl) * TP + f4);
-                    acc.x += u.x;
-                    acc.y += u.y;
-                    acc.z += u.z;
-                    acc.w += u.w;
+                float4 part[TC_MAX_CLUSTER_SPLITS];
+#pragma unroll
+                for (int src = 0; src < TC_MAX_CLUSTER_SPLITS; ++src)  // every partial loaded before any is added
+                    if (src < Sc)
+                        part[src] = *reinterpret_cast<const float4*>(
+                            src == rank ? t : recv + ((size_t)src * (NT / Sc) + jl) * TP + f4);
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int src = 0; src < TC_MAX_CLUSTER_SPLITS; ++src) {  // every split's partial, in rank order
+                    if (src >= Sc) continue;
+                    acc.x += part[src].x;
+                    acc.y += part[src].y;
+                    acc.z += part[src].z;
+                    acc.w += part[src].w;
                 }
                 *reinterpret_cast<float4*>(t) = acc;
             }
@@ -262,6 +276,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         cluster_arrive_relaxed();  // this CTA's pushes have landed (waited for before leaving)
     }
     __syncthreads();
+    trace_mark(a.trace, 4);  // rows to finish summed
     if (good && s_ok) {
         // float4 rows of T -> out, coalesced
         const int rows = min(NT, a.m - arow);
@@ -329,6 +344,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             }
         }
         }
+        trace_mark(a.trace, 5);  // thread 0's stores issued
     } else if (!fin) {
         // the MMAs may still be running: wait for them (bounded) before freeing TMEM
         mbar_wait(&done, 0, nullptr);
