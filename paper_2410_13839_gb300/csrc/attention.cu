@@ -58,6 +58,13 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
+// The transpose of the 8 x 8 b16 matrix whose row lane / 4, columns 2 (lane % 4) and + 1, this
+// lane holds in r: returns the same elements of the transposed matrix.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t r) {
+    uint32_t d;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(r));
+    return d;
+}
 // x0, x1 as bf16 pairs hi + lo (hi + lo = x to about 2^-16 relative; low halves hold x0)
 __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
     const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
@@ -243,23 +250,35 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
     }
     __syncthreads();
 
-    // per-warp tensor-core tiles: fragment rows = fed rows (rows >= RPG zero)
-    const int qrow = lane >> 2, c2 = (lane & 3) * 2;
-    const bool qon = qrow < RPG && s_act[qrow];
-    const int qpos = qon ? s_pos[qrow] : -1;
-    uint32_t qhi[4][2], qlo[4][2];
+    // per-warp tensor-core tiles with the keys as the M side: S^T = K Q^T (16 keys x the 8 query
+    // rows; the queries' bf16 hi and lo parts are two N = 8 operands) and O^T += V^T P^T (head
+    // dims x query rows, P^T's hi and lo parts added into the same accumulator).  Lane (g, c2):
+    // keys g, g + 8 of a tile and queries c2, c2 + 1 in S^T; head dims g, g + 8 of each 16-dim
+    // block and queries c2, c2 + 1 in O^T.
+    const int g8 = lane >> 2, c2 = (lane & 3) * 2;
+    bool qon[2];
+    int qpos[2];
 #pragma unroll
-    for (int ks = 0; ks < 4; ++ks)
+    for (int j = 0; j < 2; ++j) {
+        qon[j] = s_act[c2 + j] != 0;
+        qpos[j] = qon[j] ? s_pos[c2 + j] : -1;
+    }
+    uint32_t qhi[4][2], qlo[4][2];  // B operand of S^T: query row g8, dims ks * 16 + 8 hh + c2, + 1
+    {
+        const bool on = s_act[g8] != 0;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int k = ks * 16 + hh * 8 + c2;
-            split2(qon ? qs[qrow * HEAD_DIM + k] : 0.f, qon ? qs[qrow * HEAD_DIM + k + 1] : 0.f, qhi[ks][hh],
-                   qlo[ks][hh]);
-        }
-    float m_w = -INFINITY, l_w = 0.f;
-    float o[8][4];
+        for (int ks = 0; ks < 4; ++ks)
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
+            for (int hh = 0; hh < 2; ++hh) {
+                const int k = ks * 16 + hh * 8 + c2;
+                split2(on ? qs[g8 * HEAD_DIM + k] : 0.f, on ? qs[g8 * HEAD_DIM + k + 1] : 0.f, qhi[ks][hh],
+                       qlo[ks][hh]);
+            }
+    }
+    float m_w[2] = {-INFINITY, -INFINITY}, l_w[2] = {0.f, 0.f};
+    float o[4][4];  // O^T block dp: dims dp * 16 + g8 (0, 1) and + 8 (2, 3), queries c2 + (i & 1)
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
 #pragma unroll
         for (int i = 0; i < 4; ++i) o[j][i] = 0.f;
     const int swz = a.kv_swizzled ? 7 : 0;
@@ -277,59 +296,67 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
         const uint32_t kb = smem_addr(Ks + (size_t)half * HALF_KEYS * HEAD_DIM);
         const uint32_t vb = smem_addr(Vs + (size_t)half * HALF_KEYS * HEAD_DIM);
         for (int kt = warp * 16; kt < nk && ok; kt += (ATT_THREADS / 32) * 16) {
-            float sh[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-            float sl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};  // hi and lo parts: own chains
             {
-                const int key = kt + (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
+                // A = K rows kt..kt+15: matrices (keys 0-7 | 8-15) x (dims 0-7 | 8-15) of the k-step
+                const int key = kt + (lane & 7) + (((lane >> 3) & 1) << 3), chalf = lane >> 4;
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) {
-                    uint32_t b[4];
-                    ldsm_x4(b, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & swz)) << 4));
-                    const uint32_t ah[4] = {qhi[ks][0], 0u, qhi[ks][1], 0u};
-                    const uint32_t al[4] = {qlo[ks][0], 0u, qlo[ks][1], 0u};
-                    const uint32_t b0[2] = {b[0], b[1]}, b1[2] = {b[2], b[3]};
-                    mma_bf16(sh[0], ah, b0);
-                    mma_bf16(sl[0], al, b0);
-                    mma_bf16(sh[1], ah, b1);
-                    mma_bf16(sl[1], al, b1);
+                    uint32_t ka[4];
+                    ldsm_x4(ka, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & swz)) << 4));
+                    const uint32_t bh[2] = {qhi[ks][0], qhi[ks][1]}, bl[2] = {qlo[ks][0], qlo[ks][1]};
+                    mma_bf16(sh, ka, bh);
+                    mma_bf16(sl, ka, bl);
                 }
             }
-            // this lane's scores: row qrow, keys kt + {c2, c2 + 1, 8 + c2, 9 + c2} of the batch
-            float sv[4] = {sh[0][0] + sl[0][0], sh[0][1] + sl[0][1], sh[1][0] + sl[1][0], sh[1][1] + sl[1][1]};
-            float tmax = -INFINITY;
+            // this lane's scores: keys kt + g8 (i = 0, 1) and kt + g8 + 8 (i = 2, 3), query c2 + (i & 1)
+            float sv[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int kp = bp * P + kt + (q >> 1) * 8 + c2 + (q & 1);
-                sv[q] = qon && kp <= qpos ? sv[q] : -INFINITY;
-                tmax = fmaxf(tmax, sv[q]);
+            for (int i = 0; i < 4; ++i) {
+                const int kp = bp * P + kt + g8 + (i >> 1) * 8, j = i & 1;
+                const float v = sh[i] + sl[i];
+                sv[i] = qon[j] && kp <= qpos[j] && kp < K_tot ? v : -INFINITY;
             }
-            tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 1));
-            tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 2));
-            const float m_new = fmaxf(m_w, tmax);
-            const float corr = m_new == -INFINITY ? 1.f : (m_w == -INFINITY ? 0.f : expf(m_w - m_new));
+            float t0 = fmaxf(sv[0], sv[2]), t1 = fmaxf(sv[1], sv[3]);  // over the tile's keys: lanes g8
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                t0 = fmaxf(t0, __shfl_xor_sync(FULL_MASK, t0, off));
+                t1 = fmaxf(t1, __shfl_xor_sync(FULL_MASK, t1, off));
+            }
+            const float mn[2] = {fmaxf(m_w[0], t0), fmaxf(m_w[1], t1)};
+            float corr[2];
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+                corr[j] = mn[j] == -INFINITY ? 1.f : (m_w[j] == -INFINITY ? 0.f : expf(m_w[j] - mn[j]));
             float pv[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) pv[q] = sv[q] == -INFINITY ? 0.f : expf(sv[q] - m_new);
-            l_w = l_w * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
-            m_w = m_new;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                o[j][0] *= corr;
-                o[j][1] *= corr;
-            }
-            uint32_t ph[4] = {0u, 0u, 0u, 0u}, pl[4] = {0u, 0u, 0u, 0u};
-            split2(pv[0], pv[1], ph[0], pl[0]);
-            split2(pv[2], pv[3], ph[2], pl[2]);
-            const int vkey = kt + (lane & 7) + (((lane >> 3) & 1) << 3), vhalf = lane >> 4;
+            for (int i = 0; i < 4; ++i) pv[i] = sv[i] == -INFINITY ? 0.f : expf(sv[i] - mn[i & 1]);
+            l_w[0] = l_w[0] * corr[0] + (pv[0] + pv[2]);
+            l_w[1] = l_w[1] * corr[1] + (pv[1] + pv[3]);
+            m_w[0] = mn[0];
+            m_w[1] = mn[1];
 #pragma unroll
             for (int dp = 0; dp < 4; ++dp) {
-                uint32_t v[4];
-                ldsm_x4_t(v, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & swz)) << 4));
-                const uint32_t v0[2] = {v[0], v[1]}, v1[2] = {v[2], v[3]};
-                mma_bf16(o[2 * dp], ph, v0);
-                mma_bf16(o[2 * dp], pl, v0);
-                mma_bf16(o[2 * dp + 1], ph, v1);
-                mma_bf16(o[2 * dp + 1], pl, v1);
+                o[dp][0] *= corr[0];
+                o[dp][1] *= corr[1];
+                o[dp][2] *= corr[0];
+                o[dp][3] *= corr[1];
+            }
+            // P^T as the B operand (keys x queries): this lane holds rows g8 (keys) and columns c2 (queries)
+            // of each 8 x 8 block; its transpose is the operand's layout (query g8, keys c2, c2 + 1)
+            uint32_t ph0, pl0, ph1, pl1;
+            split2(pv[0], pv[1], ph0, pl0);  // keys g8
+            split2(pv[2], pv[3], ph1, pl1);  // keys g8 + 8
+            const uint32_t bph[2] = {movmatrix_trans(ph0), movmatrix_trans(ph1)};
+            const uint32_t bpl[2] = {movmatrix_trans(pl0), movmatrix_trans(pl1)};
+            // A = V^T: matrices (dims 0-7 | 8-15 of block dp) x (keys 0-7 | 8-15), from the key rows
+            const int vkey = kt + (lane & 7) + ((lane >> 4) << 3), vhalf = (lane >> 3) & 1;
+#pragma unroll
+            for (int dp = 0; dp < 4; ++dp) {
+                uint32_t va[4];
+                ldsm_x4_t(va, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & swz)) << 4));
+                mma_bf16(o[dp], va, bph);
+                mma_bf16(o[dp], va, bpl);
             }
         }
         __syncthreads();  // every warp is done with this slot
@@ -348,17 +375,23 @@ __global__ void __launch_bounds__(ATT_THREADS, 4) attn_kernel(const AttnArgs a) 
     }
     // merge the warps' (max, sum, out) per row through the staging area:
     // warp j then holds row j's (m_run, l_run) and output dims 2 lane, 2 lane + 1
-    l_w += __shfl_xor_sync(FULL_MASK, l_w, 1);
-    l_w += __shfl_xor_sync(FULL_MASK, l_w, 2);
+#pragma unroll
+    for (int j = 0; j < 2; ++j)  // each lane summed its own keys; the query's keys span lanes g8
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) l_w[j] += __shfl_xor_sync(FULL_MASK, l_w[j], off);
     float* wst = reinterpret_cast<float*>(Ks);  // [warps][RPG][PART]
-    if (qrow < RPG) {
-        float* ws = wst + ((size_t)warp * RPG + qrow) * PART;
-        if (c2 == 0) {
-            ws[0] = m_w;
-            ws[1] = l_w;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        float* ws = wst + ((size_t)warp * RPG + c2 + j) * PART;
+        if (g8 == 0) {
+            ws[0] = m_w[j];
+            ws[1] = l_w[j];
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) *reinterpret_cast<float2*>(ws + 2 + j * 8 + c2) = make_float2(o[j][0], o[j][1]);
+        for (int dp = 0; dp < 4; ++dp) {
+            ws[2 + dp * 16 + g8] = o[dp][j];
+            ws[2 + dp * 16 + g8 + 8] = o[dp][2 + j];
+        }
     }
     __syncthreads();
     constexpr int NW = ATT_THREADS / 32;
