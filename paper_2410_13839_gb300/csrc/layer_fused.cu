@@ -642,25 +642,38 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     // of a batch; S = Q K^T (fed rows as the M = 16 side, rows >= MT zero)
     // and O += P V with online-softmax state in registers.  Q and P enter as
     // bf16 hi + lo pairs (two MMAs), which keeps them to fp32 accuracy.
-    const int qrow = lane >> 2, c2 = (lane & 3) * 2;
-    const bool qon = qrow < MT && qrow < a.M && s_seq[min(qrow, MT - 1)] >= 0;
-    const int qpos = qon ? s_pos[qrow] : -1;
-    const int qgrp = qrow / rpg;
-    uint32_t qhi[4][2], qlo[4][2];  // A-fragment registers 0 and 2 of each k-step (rows g + 8 are zero)
+    // Keys as the MMA's M side: S^T = K Q^T over 16-key tiles (the fed rows' bf16 hi and lo parts
+    // as two N = 8 operands) and O^T += V^T P^T (head dims x fed rows; P^T's hi and lo parts into
+    // one accumulator).  Lane (g8, c2): keys g8, g8 + 8 of a tile and rows c2, c2 + 1 in S^T; head
+    // dims g8, g8 + 8 of each 16-dim block and rows c2, c2 + 1 in O^T.
+    const int g8 = lane >> 2, c2 = (lane & 3) * 2;
+    bool qon[2];
+    int qpos[2], qgrp[2];
 #pragma unroll
-    for (int ks = 0; ks < 4; ++ks)
+    for (int j = 0; j < 2; ++j) {
+        const int r = c2 + j;
+        qon[j] = r < MT && r < a.M && s_seq[min(r, MT - 1)] >= 0;
+        qpos[j] = qon[j] ? s_pos[min(r, MT - 1)] : -1;
+        qgrp[j] = r / rpg;
+    }
+    uint32_t qhi[4][2], qlo[4][2];  // B operand of S^T: fed row g8, dims ks * 16 + 8 hh + c2, + 1
+    {
+        const bool on = g8 < MT && g8 < a.M && s_seq[min(g8, MT - 1)] >= 0;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int k = ks * 16 + hh * 8 + c2;
-            // the query scaled by 1/sqrt(64) (exact in binary)
-            const float q0 = qon ? qkvf[k * MT + qrow] * 0.125f : 0.f;
-            const float q1 = qon ? qkvf[(k + 1) * MT + qrow] * 0.125f : 0.f;
-            split_bf16x2(q0, q1, qhi[ks][hh], qlo[ks][hh]);
-        }
-    float m_run = -INFINITY, l_run = 0.f;
-    float o[8][4];
+        for (int ks = 0; ks < 4; ++ks)
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
+            for (int hh = 0; hh < 2; ++hh) {
+                const int k = ks * 16 + hh * 8 + c2;
+                // the query scaled by 1/sqrt(64) (exact in binary)
+                const float q0 = on ? qkvf[k * MT + g8] * 0.125f : 0.f;
+                const float q1 = on ? qkvf[(k + 1) * MT + g8] * 0.125f : 0.f;
+                split_bf16x2(q0, q1, qhi[ks][hh], qlo[ks][hh]);
+            }
+    }
+    float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+    float o[4][4];  // O^T block dp: dims dp * 16 + g8 (0, 1) and + 8 (2, 3), fed rows c2 + (i & 1)
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
 #pragma unroll
         for (int i = 0; i < 4; ++i) o[j][i] = 0.f;
     const int G = (a.M + rpg - 1) / rpg;
@@ -704,79 +717,92 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
             for (int kt = warp * 16; kt < nk; kt += NWARPS * 16) {
                 const int r0 = kt % P;  // first key row of the tile in its page
                 const uint32_t kb = smem_addr(slot_keys(kt / P)), vb = kb + P * HEAD_DIM * 2;
-                float sfr[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-                float sfl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};  // lo parts: own chains
+                float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};  // hi and lo parts: own chains
                 {
-                    const int key = r0 + (lane & 7) + ((lane >> 4) << 3), chalf = (lane >> 3) & 1;
+                    // A = K rows: matrices (keys 0-7 | 8-15) x (dims 0-7 | 8-15) of the k-step
+                    const int key = r0 + (lane & 7) + (((lane >> 3) & 1) << 3), chalf = lane >> 4;
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks) {
-                        uint32_t b[4];
-                        ldsm_x4(b, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & 7)) << 4));
-                        const uint32_t ah[4] = {qhi[ks][0], 0u, qhi[ks][1], 0u};
-                        const uint32_t al[4] = {qlo[ks][0], 0u, qlo[ks][1], 0u};
-                        const uint32_t b0[2] = {b[0], b[1]}, b1[2] = {b[2], b[3]};
-                        mma_bf16(sfr[0], ah, b0);
-                        mma_bf16(sfl[0], al, b0);
-                        mma_bf16(sfr[1], ah, b1);
-                        mma_bf16(sfl[1], al, b1);
+                        uint32_t ka[4];
+                        ldsm_x4(ka, kb + key * 128 + ((uint32_t)((2 * ks + chalf) ^ (key & 7)) << 4));
+                        const uint32_t bh[2] = {qhi[ks][0], qhi[ks][1]}, bl[2] = {qlo[ks][0], qlo[ks][1]};
+                        mma_bf16(sh, ka, bh);
+                        mma_bf16(sl, ka, bl);
                     }
                 }
-                // this lane's scores: row qrow, keys kt + {c2, c2 + 1, 8 + c2, 9 + c2} of the batch
-                float sv[4] = {sfr[0][0] + sfl[0][0], sfr[0][1] + sfl[0][1], sfr[1][0] + sfl[1][0],
-                               sfr[1][1] + sfl[1][1]};
-                float tmax = -INFINITY;
+                // this lane's scores: keys kt + g8 (i = 0, 1) and kt + g8 + 8 (i = 2, 3), fed row c2 + (i & 1)
+                float sv[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const int kp = bp * P + kt + (i >> 1) * 8 + c2 + (i & 1);
-                    const bool vis = qon && qgrp == g && kp <= qpos && kp < K_tot;
-                    sv[i] = vis ? sv[i] : -INFINITY;
-                    tmax = fmaxf(tmax, sv[i]);
+                    const int kp = bp * P + kt + g8 + (i >> 1) * 8, j = i & 1;
+                    const bool vis = qon[j] && qgrp[j] == g && kp <= qpos[j] && kp < K_tot;
+                    sv[i] = vis ? sh[i] + sl[i] : -INFINITY;
                 }
-                tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 1));
-                tmax = fmaxf(tmax, __shfl_xor_sync(FULL_MASK, tmax, 2));
-                const float m_new = fmaxf(m_run, tmax);
-                const float corr = m_new == -INFINITY ? 1.f : (m_run == -INFINITY ? 0.f : expf(m_run - m_new));
+                float t0 = fmaxf(sv[0], sv[2]), t1 = fmaxf(sv[1], sv[3]);  // over the tile's keys: lanes g8
+#pragma unroll
+                for (int off = 4; off < 32; off <<= 1) {
+                    t0 = fmaxf(t0, __shfl_xor_sync(FULL_MASK, t0, off));
+                    t1 = fmaxf(t1, __shfl_xor_sync(FULL_MASK, t1, off));
+                }
+                const float mn[2] = {fmaxf(m_run[0], t0), fmaxf(m_run[1], t1)};
+                float corr[2];
+#pragma unroll
+                for (int j = 0; j < 2; ++j)
+                    corr[j] = mn[j] == -INFINITY ? 1.f : (m_run[j] == -INFINITY ? 0.f : expf(m_run[j] - mn[j]));
                 float pv[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) pv[i] = sv[i] == -INFINITY ? 0.f : expf(sv[i] - m_new);
-                l_run = l_run * corr + ((pv[0] + pv[1]) + (pv[2] + pv[3]));
-                m_run = m_new;
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    o[j][0] *= corr;
-                    o[j][1] *= corr;
-                }
-                uint32_t ph[4] = {0u, 0u, 0u, 0u}, pl[4] = {0u, 0u, 0u, 0u};
-                split_bf16x2(pv[0], pv[1], ph[0], pl[0]);
-                split_bf16x2(pv[2], pv[3], ph[2], pl[2]);
-                const int vkey = r0 + (lane & 7) + (((lane >> 3) & 1) << 3), vhalf = lane >> 4;
+                for (int i = 0; i < 4; ++i) pv[i] = sv[i] == -INFINITY ? 0.f : expf(sv[i] - mn[i & 1]);
+                l_run[0] = l_run[0] * corr[0] + (pv[0] + pv[2]);
+                l_run[1] = l_run[1] * corr[1] + (pv[1] + pv[3]);
+                m_run[0] = mn[0];
+                m_run[1] = mn[1];
 #pragma unroll
                 for (int dp = 0; dp < 4; ++dp) {
-                    uint32_t v[4];
-                    ldsm_x4_t(v, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & 7)) << 4));
-                    const uint32_t v0[2] = {v[0], v[1]}, v1[2] = {v[2], v[3]};
-                    mma_bf16(o[2 * dp], ph, v0);
-                    mma_bf16(o[2 * dp], pl, v0);
-                    mma_bf16(o[2 * dp + 1], ph, v1);
-                    mma_bf16(o[2 * dp + 1], pl, v1);
+                    o[dp][0] *= corr[0];
+                    o[dp][1] *= corr[1];
+                    o[dp][2] *= corr[0];
+                    o[dp][3] *= corr[1];
+                }
+                // P^T as the B operand: this lane holds rows g8 (keys), columns c2 (fed rows) of each
+                // 8 x 8 block; its transpose is the operand's layout (fed row g8, keys c2, c2 + 1)
+                uint32_t ph0, pl0, ph1, pl1;
+                split_bf16x2(pv[0], pv[1], ph0, pl0);  // keys g8
+                split_bf16x2(pv[2], pv[3], ph1, pl1);  // keys g8 + 8
+                const uint32_t bph[2] = {movmatrix_trans(ph0), movmatrix_trans(ph1)};
+                const uint32_t bpl[2] = {movmatrix_trans(pl0), movmatrix_trans(pl1)};
+                // A = V^T: matrices (dims 0-7 | 8-15 of block dp) x (keys 0-7 | 8-15), from the key rows
+                const int vkey = r0 + (lane & 7) + ((lane >> 4) << 3), vhalf = (lane >> 3) & 1;
+#pragma unroll
+                for (int dp = 0; dp < 4; ++dp) {
+                    uint32_t va[4];
+                    ldsm_x4_t(va, vb + vkey * 128 + ((uint32_t)((2 * dp + vhalf) ^ (vkey & 7)) << 4));
+                    mma_bf16(o[dp], va, bph);
+                    mma_bf16(o[dp], va, bpl);
                 }
             }
         }
     }
     // merge the warps' (max, sum, out) states into part through the weight
     // area (free once every warp is past its last tile): [NWARPS][MT][PARTW]
-    l_run += __shfl_xor_sync(FULL_MASK, l_run, 1);
-    l_run += __shfl_xor_sync(FULL_MASK, l_run, 2);
+#pragma unroll
+    for (int j = 0; j < 2; ++j)  // each lane summed its own keys; a row's keys span lanes g8
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) l_run[j] += __shfl_xor_sync(FULL_MASK, l_run[j], off);
     __syncthreads();
     float* wst = reinterpret_cast<float*>(smem + L.wqkv);
-    if (qrow < MT) {
-        float* ws = wst + ((size_t)warp * MT + qrow) * PARTW;
-        if (c2 == 0) {
-            ws[0] = m_run;
-            ws[1] = l_run;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        if (c2 + j >= MT) continue;
+        float* ws = wst + ((size_t)warp * MT + c2 + j) * PARTW;
+        if (g8 == 0) {
+            ws[0] = m_run[j];
+            ws[1] = l_run[j];
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) *reinterpret_cast<float2*>(ws + 2 + j * 8 + c2) = make_float2(o[j][0], o[j][1]);
+        for (int dp = 0; dp < 4; ++dp) {
+            ws[2 + dp * 16 + g8] = o[dp][j];
+            ws[2 + dp * 16 + g8 + 8] = o[dp][2 + j];
+        }
     }
     __syncthreads();
     if (tid < NWARPS * MT) {  // weight of warp w's state in row m: exp(max_w - common max)
