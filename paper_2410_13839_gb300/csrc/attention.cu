@@ -4,12 +4,13 @@
 // Grid (split, head, group).  A group is the rows of one slot (the n tokens
 // fed this step, or 8 consecutive positions of a prefill chunk).  Each CTA
 // takes a contiguous range of pages of its slot and streams their keys and
-// values for its head through two halves of shared memory with
-// cp.async.bulk (one half is filled while the other is read).  Each warp
-// takes 16-key tiles: S = Q K^T and O += P V on the tensor cores (mma.sync;
-// the fed rows are the M side, Q and P enter as bf16 hi + lo pairs, which
-// keeps them to fp32 accuracy) with its online-softmax state in registers;
-// the warps' states are merged in shared memory.  Partial results (max,
+// values for its head through a ring of three shared-memory slots with
+// cp.async.bulk (two are in flight while one is read).  Each warp takes
+// 16-key tiles on the tensor cores (mma.sync) with the keys as the M side:
+// S^T = K Q^T and O^T += V^T P^T, the fed rows' Q and P entering as bf16
+// hi + lo pairs (two N = 8 operands), which keeps them to fp32 accuracy, and
+// its online-softmax state in registers; the warps' states are merged in
+// shared memory.  Partial results (max,
 // sum, unnormalised output) of the splits are merged with a log-sum-exp by
 // the CTA that finishes last (an atomic counter per group and head, reset by
 // that CTA), so no second kernel is needed.

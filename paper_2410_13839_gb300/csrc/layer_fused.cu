@@ -639,8 +639,7 @@ __global__ void __cluster_dims__(CA, 1, 1) __launch_bounds__(NTHREADS, 2) attn_b
     trace_mark(a.trace, 4);  // gathered
     // ---- 4. attention over this CTA's split of each group's keys ----
     // Flash-attention style on the tensor cores: each warp takes 16-key tiles
-    // of a batch; S = Q K^T (fed rows as the M = 16 side, rows >= MT zero)
-    // and O += P V with online-softmax state in registers.  Q and P enter as
+    // of a batch with online-softmax state in registers; Q and P enter as
     // bf16 hi + lo pairs (two MMAs), which keeps them to fp32 accuracy.
     // Keys as the MMA's M side: S^T = K Q^T over 16-key tiles (the fed rows' bf16 hi and lo parts
     // as two N = 8 operands) and O^T += V^T P^T (head dims x fed rows; P^T's hi and lo parts into

@@ -201,7 +201,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     if (warp < 2) __syncwarp();
 
-    // epilogue: thread = weight row f (TMEM lane), 32 activation rows per load
+    // epilogue: lane = weight row f (TMEM lane of the warp's quarter), 32 activation rows per load
     // one thread polls (a poll costs each polling thread, even on a completed phase); the block
     // barrier hands the result to the others
     const bool fin = __syncthreads_and(tid == 0 ? mbar_wait(&done, 0, a.err) : true) != 0;
