@@ -24,9 +24,14 @@ a transposed operand or a wrong head layout breaks); with every block matrix
 and bias zero the decoder returns tok_phone[id] + PE(p) on the phoneme span
 and tok_codec[id] + PE(p) on the codec span, the sinusoid written out in
 scalar form (tests/test_oracle_heads_embed.py; swapped or shared tables
-rejected).  Beyond these, the composition of the
-block is "parity unpinned" against any printed value: the paper prints no
-activation, logit or worked example of the model.
+rejected); the whole block stack against PyTorch's pre-LN transformer
+encoder layer (torch.nn.TransformerEncoderLayer, norm_first, exact GELU)
+loaded with the same weights, for a whole prompt and a prompt fed in chunks
+through the cache, to float64 rounding (tests/test_oracle_block_torch.py;
+a transposed W_o, heads split across the wrong axis, the tanh GELU and a
+skipped LN2 rejected).  No pin ties the block to printed values: the paper
+prints no activation, logit or worked example of the model, so what these
+pins fix is the reading above, not numbers from the paper.
 """
 from __future__ import annotations
 
