@@ -82,7 +82,7 @@ struct AttnArgs {
     int rows;                                                // attention_tc: rows of the pass (tiles of 128)
 };
 
-constexpr int ATTN_CTAS_PER_SM = 4;  // attn_kernel: 128 threads x 128 registers, ~51 KB of shared memory
+constexpr int ATTN_CTAS_PER_SM = 4;  // attn_kernel: 128 threads x at most 128 registers, ~51 KB of shared memory
 constexpr int ATTN_MAX_SPLITS = 32;  // key splits one launch merges
 size_t attn_workspace_floats(int groups, int n_heads, int n_splits, int rows_per_group);
 size_t attn_smem_bytes(int page_size);
