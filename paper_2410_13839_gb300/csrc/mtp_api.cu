@@ -1222,7 +1222,7 @@ MTP_API int mtp_create(const mtp_config* config, const void* weights_blob, size_
     const mtp_config& cf = c->cfg;
     if ((r = upload_weights(c, weights_blob, blob_bytes)) != MTP_OK) return bail(r);
 
-    const int d = cf.d_model, F = cf.d_ffn, H = cf.n_attn_heads, P = cf.page_size, B = cf.max_batch;
+    const int d = cf.d_model, H = cf.n_attn_heads, P = cf.page_size, B = cf.max_batch;
     const int V = cf.codec_vocab, nm = cf.n_heads_max;
     c->pages_per_seq = (cf.max_ctx + P - 1) / P;
     c->n_pages = cf.n_pages > 0 ? cf.n_pages : B * c->pages_per_seq;

@@ -159,20 +159,6 @@ __device__ void viterbi_warp(const int* ids, const float* lp, const float* lq, i
     }
 }
 
-// ACCEPT_ALL: cut after the first EOS and at the budget.
-__device__ __forceinline__ void accept_all(const int* path, int n, int eos, int remaining, int& a, int& done) {
-    a = n;
-    bool eos_in = false;
-    for (int t = 0; t < n; ++t)
-        if (path[t] == eos) {
-            a = t + 1;
-            eos_in = true;
-            break;
-        }
-    a = min(a, max(remaining, 0));
-    done = (eos_in && a >= 1 && path[a - 1] == eos) || remaining - a <= 0;
-}
-
 constexpr int MS = MAX_NHEADS * MAX_TOPK;  // most states of a union lattice
 constexpr int LQ_FLOATS = (MAX_NHEADS - 1) * MAX_TOPK * MAX_TOPK;  // select_kernel's scratch
 static_assert((2 + MAX_NHEADS + 2 + MAX_NHEADS) * MS <= LQ_FLOATS, "union Viterbi scratch");
@@ -503,7 +489,7 @@ __global__ void __launch_bounds__(256) verify_kernel(const VerifyArgs a) {
 // no shared memory to limit how many warps an SM holds.  The ids of the
 // previous position come from the group's lanes by shuffle.  The recursion,
 // its add order and its tie rules are those of viterbi_warp; acceptance is
-// accept_all's rule (cut after the first EOS and at the remaining budget).
+// the ACCEPT_ALL rule (cut after the first EOS and at the remaining budget).
 constexpr int VIT_THREADS = 256;
 
 template <int KP>

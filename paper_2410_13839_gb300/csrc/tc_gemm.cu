@@ -219,7 +219,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     float* T = reinterpret_cast<float*>(smem);
     if (good) {
         // accumulator -> shared tile T[n][f] (the stages are free: every MMA has read them)
-#pragma unroll 1
         const int quarter = warp & 3;  // the TMEM lanes (weight rows) this warp may read
         for (int j0 = (warp >> 2) * 32; j0 < NT; j0 += (TC_THREADS / 128) * 32) {
             float v[32];
